@@ -1,0 +1,138 @@
+"""Python access to the plain CPU oracle (``oracle.c``).
+
+TEST INFRASTRUCTURE ONLY.  Only the tests, ``__graft_entry__.smoke()`` and the
+CPU-baseline leg of ``bench.py`` may import this module.  The product path (the
+CUDA library and its binding) never touches it.
+
+What the oracle computes, and the passage each part follows:
+
+* ``gilbert_order(Mt, Nt)`` -- the generalized Hilbert curve over the Mt x Nt
+  output-tile grid (Sec. II-B, Fig. 2; ``create_sfc_map`` / ``map_sfc_index``
+  of Listing 1).  ``out[s] = tm * Nt + tn``.
+* ``gemm_f64(A, B)`` -- C = A * B by definition, fp64 accumulation over the
+  bf16 inputs widened exactly (Sec. II-A, Listing 1).
+* ``gemm_sub_f64(A, B, rows, cols, k0, k1)`` -- selected rows/columns, optionally
+  one K range (one layer's partial product of the K split, Sec. II-C/D).
+* ``round_bf16(x)`` -- one-step round-to-nearest-even of doubles to bf16.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "oracle.c")
+_LIB = os.path.join(_HERE, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile ``oracle.c`` into ``liboracle.so`` beside it (gcc, OpenMP)."""
+    if not force and os.path.exists(_LIB) and os.path.getmtime(_LIB) >= os.path.getmtime(_SRC):
+        return _LIB
+    tmp = _LIB + ".tmp%d" % os.getpid()
+    cmd = ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fopenmp",
+           "-ffp-contract=off", "-o", tmp, _SRC, "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, _LIB)
+    return _LIB
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        lib = ctypes.CDLL(build())
+        i32p = ctypes.POINTER(ctypes.c_int32)
+        u16p = ctypes.c_void_p
+        i64 = ctypes.c_int64
+        lib.oracle_gilbert_order.argtypes = [ctypes.c_int, ctypes.c_int, i32p]
+        lib.oracle_gilbert_order.restype = ctypes.c_int
+        lib.oracle_gemm_f64.argtypes = [i64, i64, i64, u16p, i64, u16p, i64, ctypes.c_void_p, i64]
+        lib.oracle_gemm_f64.restype = None
+        lib.oracle_gemm_sub_f64.argtypes = [ctypes.c_void_p, i64, ctypes.c_void_p, i64, i64, i64,
+                                            u16p, i64, u16p, i64, ctypes.c_void_p]
+        lib.oracle_gemm_sub_f64.restype = None
+        lib.oracle_round_bf16.argtypes = [ctypes.c_double]
+        lib.oracle_round_bf16.restype = ctypes.c_uint16
+        lib.oracle_round_bf16_array.argtypes = [ctypes.c_void_p, i64, ctypes.c_void_p]
+        lib.oracle_round_bf16_array.restype = None
+        _lib = lib
+        return lib
+
+
+def gilbert_order(Mt: int, Nt: int) -> np.ndarray:
+    """Curve permutation: ``out[s] = tm * Nt + tn`` (int32, length Mt*Nt)."""
+    out = np.empty(Mt * Nt, dtype=np.int32)
+    rc = _load().oracle_gilbert_order(int(Mt), int(Nt),
+                                      out.ctypes.data_as(ctypes.POINTER(ctypes.c_int32)))
+    if rc != 0:
+        raise RuntimeError("oracle_gilbert_order(%d, %d) failed with %d" % (Mt, Nt, rc))
+    return out
+
+
+def _bf16_bits(x) -> np.ndarray:
+    """Accept a torch bf16 tensor or a uint16 array of bf16 bit patterns."""
+    if hasattr(x, "dtype") and str(x.dtype) == "torch.bfloat16":
+        import torch
+        return x.detach().cpu().contiguous().view(torch.int16).numpy().view(np.uint16)
+    arr = np.ascontiguousarray(x)
+    if arr.dtype != np.uint16:
+        raise TypeError("expected bf16 bit patterns (uint16) or a torch.bfloat16 tensor")
+    return arr
+
+
+def gemm_f64(A, B) -> np.ndarray:
+    """C = A @ B in fp64 over bf16 inputs (row-major, dense)."""
+    a = _bf16_bits(A)
+    b = _bf16_bits(B)
+    M, K = a.shape
+    K2, N = b.shape
+    if K != K2:
+        raise ValueError("inner dimensions differ")
+    C = np.empty((M, N), dtype=np.float64)
+    _load().oracle_gemm_f64(M, N, K, a.ctypes.data, K, b.ctypes.data, N, C.ctypes.data, N)
+    return C
+
+
+def gemm_sub_f64(A, B, rows=None, cols=None, k0: int = 0, k1: int | None = None) -> np.ndarray:
+    """Rows ``rows`` x columns ``cols`` of A[:, k0:k1] @ B[k0:k1, :] in fp64."""
+    a = _bf16_bits(A)
+    b = _bf16_bits(B)
+    M, K = a.shape
+    N = b.shape[1]
+    rows = np.arange(M, dtype=np.int64) if rows is None else np.ascontiguousarray(rows, dtype=np.int64)
+    cols = np.arange(N, dtype=np.int64) if cols is None else np.ascontiguousarray(cols, dtype=np.int64)
+    if k1 is None:
+        k1 = K
+    if not (0 <= k0 <= k1 <= K):
+        raise ValueError("bad k range")
+    if rows.size and (rows.min() < 0 or rows.max() >= M):
+        raise ValueError("row index out of range")
+    if cols.size and (cols.min() < 0 or cols.max() >= N):
+        raise ValueError("column index out of range")
+    out = np.empty((rows.size, cols.size), dtype=np.float64)
+    _load().oracle_gemm_sub_f64(rows.ctypes.data, rows.size, cols.ctypes.data, cols.size,
+                                int(k0), int(k1), a.ctypes.data, K, b.ctypes.data, N,
+                                out.ctypes.data)
+    return out
+
+
+def round_bf16_bits(x) -> np.ndarray:
+    """Round doubles to bf16 (nearest, ties to even); uint16 bit patterns."""
+    flat = np.ascontiguousarray(np.asarray(x, dtype=np.float64).ravel())
+    bits = np.empty(flat.size, dtype=np.uint16)
+    _load().oracle_round_bf16_array(flat.ctypes.data, flat.size, bits.ctypes.data)
+    return bits.reshape(np.shape(x))
+
+
+def round_bf16(x) -> np.ndarray:
+    """Round doubles to bf16 (nearest, ties to even), returned as float64 values."""
+    bits = round_bf16_bits(x)
+    return (bits.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
