@@ -1,0 +1,170 @@
+/*
+ * sfc_gemm.h -- C ABI of the space-filling-curve (SFC) bf16 GEMM for GB300.
+ *
+ * The library computes C = A * B (A: M x K, B: K x N, C: M x N, all row-major)
+ * the way Sec. II-D and Listing 1 of "Space Filling Curves is All You Need:
+ * Communication-Avoiding Matrix Multiplication Made Simple" describe it:
+ *
+ *   - the output is blocked into bm x bn tiles, an Mt x Nt grid (Sec. II-A);
+ *   - the tiles are ordered along a generalized Hilbert curve that works for
+ *     any grid shape (Sec. II-B, Fig. 2);
+ *   - the task space of Mt*Nt*ca_c items is handed to the workers in contiguous
+ *     blocks; item i belongs to K layer i / (Mt*Nt) and curve position
+ *     i % (Mt*Nt) (Listing 1, the parallel loop and its index arithmetic);
+ *   - with ca_c > 1 ("K_layers", the replication factor c of the 2.5D/3D
+ *     communication-avoiding scheme, Sec. II-C/II-D) each layer contracts its
+ *     own share of K into an fp32 copy of C, and the copies are summed at the
+ *     end in layer order 0..c-1 (Listing 1, the final reduction).
+ *
+ * Here a worker is a CUDA thread block resident on one SM of a persistent
+ * kernel; the tile contraction (the paper's batch-reduce GEMM, Sec. II-A) runs
+ * on the tcgen05 tensor cores with fp32 accumulation in tensor memory.
+ *
+ * Conventions for every entry point:
+ *   - sizes and leading dimensions are in ELEMENTS; lda >= K, ldb >= N, ldc >= N;
+ *   - A, B, C and workspace are DEVICE pointers owned by the caller; the
+ *     library never frees them and keeps no reference after the call returns;
+ *   - calls that take a stream are asynchronous on that stream (NULL = the
+ *     legacy default stream); arguments are validated on the host first and a
+ *     validation error launches nothing;
+ *   - every function returns an sfc_status_t (0 = success) unless noted.
+ *
+ * Thread safety: entry points may be called from several host threads; each
+ * call only reads immutable library state after a one-time per-device set-up.
+ */
+#ifndef SFC_GEMM_H
+#define SFC_GEMM_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    SFC_OK = 0,
+    SFC_ERR_INVALID_ARG = -1,  /* bad size, null pointer, bad enum, ca_c out of range  */
+    SFC_ERR_UNALIGNED = -2,    /* A/B base not 16-byte aligned or lda/ldb not a multiple of 8 */
+    SFC_ERR_WORKSPACE = -3,    /* workspace smaller than sfc_gemm_workspace_size(...)  */
+    SFC_ERR_CUDA = -4,         /* a CUDA runtime call failed (see sfc_last_cuda_error) */
+    SFC_ERR_TIMEOUT = -5,      /* a device-side wait gave up (reported by sfc_get_device_status) */
+    SFC_ERR_UNSUPPORTED = -6   /* no usable sm_103 device, or an option this build lacks */
+} sfc_status_t;
+
+typedef enum { SFC_F32 = 0, SFC_BF16 = 1 } sfc_dtype_t;
+
+/* Order of the output tiles along which workers take their items.
+ * SFC:    generalized Hilbert curve (Sec. II-B) -- the method.
+ * RASTER: row-major tile order s -> (s / Nt, s % Nt), a comparison baseline. */
+typedef enum { SFC_ORDER_SFC = 0, SFC_ORDER_RASTER = 1 } sfc_order_t;
+
+/* How items are dealt to the P persistent workers.
+ * SEGMENT: worker p takes the contiguous block [p*W/P, (p+1)*W/P) of the W
+ *          items, the static block partition of Listing 1's parallel loop.
+ * WAVE:    worker p takes items p, p+P, p+2P, ...: consecutive curve positions
+ *          run at the same time on different SMs, so each wave of P tiles is a
+ *          compact patch of the grid and A/B panels are shared through L2.
+ * AUTO:    the library picks (currently WAVE). */
+typedef enum { SFC_ASSIGN_SEGMENT = 0, SFC_ASSIGN_WAVE = 1, SFC_ASSIGN_AUTO = 2 } sfc_assign_t;
+
+/* Output tile width.  AUTO picks per shape; 128 and 256 force it. bm is 128. */
+typedef enum { SFC_TILE_AUTO = 0, SFC_TILE_N128 = 128, SFC_TILE_N256 = 256 } sfc_tile_t;
+
+/*
+ * sfc_tile_order -- the curve permutation over an Mt x Nt tile grid
+ * (Sec. II-B; create_sfc_map / map_sfc_index of Listing 1).
+ *   out_idx: HOST array of Mt*Nt int32, filled with out_idx[s] = tm*Nt + tn for
+ *            curve position s.  The curve starts at tile (0,0), consecutive
+ *            positions are edge-adjacent tiles.  Host-only, no GPU needed.
+ * Errors: SFC_ERR_INVALID_ARG if Mt < 1, Nt < 1, Mt*Nt > 2^31-1 or out_idx NULL.
+ */
+int sfc_tile_order(int Mt, int Nt, int32_t *out_idx);
+
+/*
+ * sfc_tile_order_device -- the same permutation computed by the GPU decoder
+ * that the GEMM kernel itself uses (one thread per curve position).
+ *   out_idx_dev: DEVICE array of Mt*Nt int32.  Asynchronous on `stream`.
+ * Errors: as sfc_tile_order, plus SFC_ERR_CUDA.
+ */
+int sfc_tile_order_device(int Mt, int Nt, int32_t *out_idx_dev, void *stream);
+
+/*
+ * sfc_gemm_workspace_size -- bytes of fp32 workspace sfc_gemm_ex needs for the
+ * ca_c partial copies of C (Listing 1's C[K_layers][...], Sec. II-D):
+ * 0 when ca_c == 1, else ca_c * M * round_up(N, 4) * 4.  Returns 0 for invalid
+ * arguments.
+ */
+size_t sfc_gemm_workspace_size(int64_t M, int64_t N, int64_t K, int ca_c);
+
+/*
+ * sfc_gemm -- C = A * B with bf16 A, B, fp32 accumulation and fp32 output,
+ * curve order, automatic assignment and tile width.
+ *   A: bf16, M x K, row stride lda.   B: bf16, K x N, row stride ldb.
+ *   C: fp32, M x N, row stride ldc.   Written, never read (beta = 0).
+ *   ca_c: number of K layers, 1 <= ca_c <= ceil(K/64).  Layer l contracts K
+ *         tiles [floor(l*Kt/ca_c), floor((l+1)*Kt/ca_c)) of the Kt = ceil(K/64)
+ *         64-wide K tiles.  For ca_c > 1 the library takes its fp32 workspace
+ *         from a stream-ordered pool (cudaMallocAsync / cudaFreeAsync on
+ *         `stream`).
+ *   stream: a cudaStream_t passed as void*.
+ * Requirements: A and B 16-byte aligned, lda and ldb multiples of 8 (the tile
+ * loads use the Tensor Memory Accelerator).  C may have any alignment.
+ * Errors: SFC_ERR_INVALID_ARG, SFC_ERR_UNALIGNED, SFC_ERR_CUDA, SFC_ERR_UNSUPPORTED.
+ */
+int sfc_gemm(int64_t M, int64_t N, int64_t K,
+             const void *A, const void *B, void *C,
+             int64_t lda, int64_t ldb, int64_t ldc,
+             int ca_c, void *stream);
+
+/*
+ * sfc_gemm_ex -- sfc_gemm with every knob exposed.
+ *   c_dtype:   SFC_F32 or SFC_BF16 (bf16 output is the fp32 result rounded to
+ *              nearest, ties to even).
+ *   order, assign, tile: see the enums above.
+ *   workspace / workspace_bytes: caller-owned DEVICE scratch of at least
+ *              sfc_gemm_workspace_size(M, N, K, ca_c) bytes, 16-byte aligned;
+ *              may be NULL when ca_c == 1, or NULL to use the stream-ordered
+ *              pool as sfc_gemm does.  Its contents on return are unspecified.
+ * Errors: as sfc_gemm, plus SFC_ERR_WORKSPACE.
+ */
+int sfc_gemm_ex(int64_t M, int64_t N, int64_t K,
+                const void *A, const void *B, void *C,
+                int64_t lda, int64_t ldb, int64_t ldc,
+                int ca_c, sfc_dtype_t c_dtype,
+                sfc_order_t order, sfc_assign_t assign, sfc_tile_t tile,
+                void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ * sfc_get_device_status -- synchronizes `stream`, then returns and clears the
+ * device error word that kernels set when a bounded wait gives up
+ * (SFC_ERR_TIMEOUT), or SFC_ERR_CUDA if the synchronization itself failed.
+ * SFC_OK if no kernel reported a problem since the last call.
+ */
+int sfc_get_device_status(void *stream);
+
+/* sfc_last_cuda_error -- the cudaError_t code behind the most recent
+ * SFC_ERR_CUDA on the calling thread (0 if none). */
+int sfc_last_cuda_error(void);
+
+/* sfc_num_workers -- number of persistent workers (SMs) used on the current
+ * device, or a negative sfc_status_t. */
+int sfc_num_workers(void);
+
+/*
+ * sfc_debug_force_timeout -- test hook for the failure path: launches one GEMM
+ * worker on a tiny problem whose MMA stage waits on a barrier that nothing
+ * arrives at, with a wait limit of `limit_ms` milliseconds (1..1000).  The
+ * kernel gives up, records SFC_ERR_TIMEOUT in the device error word, drains
+ * its in-flight copies, frees its tensor memory and returns; the context stays
+ * usable.  Read the outcome with sfc_get_device_status.
+ *   A, B: DEVICE bf16 buffers of at least 128*64 and 64*128 elements;
+ *   C:    DEVICE fp32 buffer of at least 128*128 elements.
+ */
+int sfc_debug_force_timeout(const void *A, const void *B, void *C, int limit_ms, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* SFC_GEMM_H */

@@ -1,0 +1,199 @@
+"""ctypes binding of ``libsfcgemm.so`` (C ABI declared in ``include/sfc_gemm.h``).
+
+Argument marshalling only: every step of the GEMM runs in the library's CUDA
+kernels.  PyTorch provides device memory and streams.  If the library is
+missing, every call raises :class:`SfcLibraryMissing` -- there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import numpy as np
+
+from . import build_lib
+
+SFC_OK = 0
+SFC_ERR_INVALID_ARG = -1
+SFC_ERR_UNALIGNED = -2
+SFC_ERR_WORKSPACE = -3
+SFC_ERR_CUDA = -4
+SFC_ERR_TIMEOUT = -5
+SFC_ERR_UNSUPPORTED = -6
+_NAMES = {0: "SFC_OK", -1: "SFC_ERR_INVALID_ARG", -2: "SFC_ERR_UNALIGNED", -3: "SFC_ERR_WORKSPACE",
+          -4: "SFC_ERR_CUDA", -5: "SFC_ERR_TIMEOUT", -6: "SFC_ERR_UNSUPPORTED"}
+
+SFC_F32, SFC_BF16 = 0, 1
+ORDERS = {"sfc": 0, "raster": 1}
+ASSIGNS = {"segment": 0, "wave": 1, "auto": 2}
+TILES = {0: 0, "auto": 0, 128: 128, 256: 256}
+
+EXPORTS = ("sfc_tile_order", "sfc_tile_order_device", "sfc_gemm_workspace_size", "sfc_gemm", "sfc_gemm_ex",
+           "sfc_get_device_status", "sfc_last_cuda_error", "sfc_num_workers", "sfc_debug_force_timeout")
+
+
+class SfcLibraryMissing(RuntimeError):
+    pass
+
+
+class SfcError(RuntimeError):
+    def __init__(self, code: int, what: str, cuda_error: int = 0):
+        self.code = code
+        self.cuda_error = cuda_error
+        msg = "%s failed: %s" % (what, _NAMES.get(code, str(code)))
+        if code == SFC_ERR_CUDA:
+            msg += " (CUDA error %d)" % cuda_error
+        super().__init__(msg)
+
+
+_lock = threading.Lock()
+_lib = None
+
+
+def library_path() -> str:
+    return build_lib.LIB
+
+
+def load():
+    """Load the library (once).  Raises SfcLibraryMissing if it was not built."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        path = library_path()
+        if not os.path.exists(path):
+            raise SfcLibraryMissing("libsfcgemm.so is not built (%s); run "
+                                    "`python -m paper_2601_16294_gb300.build_lib`" % path)
+        lib = ctypes.CDLL(path)
+        i64, i32, vp, sz = ctypes.c_int64, ctypes.c_int, ctypes.c_void_p, ctypes.c_size_t
+        lib.sfc_tile_order.argtypes = [i32, i32, vp]
+        lib.sfc_tile_order_device.argtypes = [i32, i32, vp, vp]
+        lib.sfc_gemm_workspace_size.argtypes = [i64, i64, i64, i32]
+        lib.sfc_gemm_workspace_size.restype = sz
+        lib.sfc_gemm.argtypes = [i64, i64, i64, vp, vp, vp, i64, i64, i64, i32, vp]
+        lib.sfc_gemm_ex.argtypes = [i64, i64, i64, vp, vp, vp, i64, i64, i64, i32, i32, i32, i32, i32, vp, sz, vp]
+        lib.sfc_get_device_status.argtypes = [vp]
+        lib.sfc_last_cuda_error.argtypes = []
+        lib.sfc_num_workers.argtypes = []
+        lib.sfc_debug_force_timeout.argtypes = [vp, vp, vp, i32, vp]
+        for name in EXPORTS:
+            if name != "sfc_gemm_workspace_size":
+                getattr(lib, name).restype = ctypes.c_int
+        _lib = lib
+        return lib
+
+
+def _check(rc: int, what: str):
+    if rc != SFC_OK:
+        raise SfcError(rc, what, load().sfc_last_cuda_error() if rc == SFC_ERR_CUDA else 0)
+
+
+def _stream_ptr(stream):
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+# ------------------------------------------------------------------ curve
+
+def tile_order(Mt: int, Nt: int) -> np.ndarray:
+    """Curve permutation from the library's host decoder: out[s] = tm*Nt + tn."""
+    out = np.empty(int(Mt) * int(Nt), dtype=np.int32)
+    _check(load().sfc_tile_order(int(Mt), int(Nt), out.ctypes.data), "sfc_tile_order")
+    return out
+
+
+def tile_order_device(Mt: int, Nt: int, stream=None):
+    """Curve permutation from the GPU decoder the GEMM kernel uses (int32 CUDA tensor)."""
+    import torch
+    out = torch.empty(int(Mt) * int(Nt), dtype=torch.int32, device="cuda")
+    _check(load().sfc_tile_order_device(int(Mt), int(Nt), ctypes.c_void_p(out.data_ptr()),
+                                        _stream_ptr(stream)), "sfc_tile_order_device")
+    return out
+
+
+# ------------------------------------------------------------------- GEMM
+
+def workspace_size(M: int, N: int, K: int, ca_c: int) -> int:
+    return int(load().sfc_gemm_workspace_size(int(M), int(N), int(K), int(ca_c)))
+
+
+def num_workers() -> int:
+    n = load().sfc_num_workers()
+    if n < 0:
+        _check(n, "sfc_num_workers")
+    return n
+
+
+def _row_major_2d(t, name):
+    if t.dim() != 2 or t.stride(1) != 1:
+        raise ValueError("%s must be a 2-D row-major (unit column stride) tensor" % name)
+    return t.stride(0)
+
+
+def gemm(A, B, C=None, *, ca_c: int = 1, out_dtype=None, order: str = "sfc", assign: str = "auto",
+         tile=0, workspace=None, stream=None):
+    """C = A @ B on the GPU.  A: (M, K) bf16, B: (K, N) bf16, both CUDA, row-major
+    (row strides may be padded).  C: (M, N) fp32 or bf16 CUDA tensor, allocated
+    if not given.  ``workspace``: optional CUDA tensor of at least
+    ``workspace_size(M, N, K, ca_c)`` bytes."""
+    import torch
+    lib = load()
+    M, K = A.shape
+    K2, N = B.shape
+    if K != K2:
+        raise ValueError("inner dimensions differ: %d vs %d" % (K, K2))
+    if A.dtype != torch.bfloat16 or B.dtype != torch.bfloat16:
+        raise TypeError("A and B must be bfloat16")
+    if C is None:
+        C = torch.empty((M, N), dtype=out_dtype or torch.float32, device=A.device)
+    if C.dtype not in (torch.float32, torch.bfloat16) or tuple(C.shape) != (M, N):
+        raise ValueError("C must be (M, N) float32 or bfloat16")
+    lda = _row_major_2d(A, "A")
+    ldb = _row_major_2d(B, "B")
+    ldc = _row_major_2d(C, "C")
+    ws_ptr, ws_bytes = None, 0
+    if workspace is not None:
+        ws_ptr, ws_bytes = ctypes.c_void_p(workspace.data_ptr()), workspace.numel() * workspace.element_size()
+    rc = lib.sfc_gemm_ex(M, N, K, ctypes.c_void_p(A.data_ptr()), ctypes.c_void_p(B.data_ptr()),
+                         ctypes.c_void_p(C.data_ptr()), lda, ldb, ldc, int(ca_c),
+                         SFC_F32 if C.dtype == torch.float32 else SFC_BF16, ORDERS[order], ASSIGNS[assign],
+                         TILES[tile], ws_ptr, ws_bytes, _stream_ptr(stream))
+    _check(rc, "sfc_gemm_ex")
+    return C
+
+
+def gemm_raw(M, N, K, A_ptr, B_ptr, C_ptr, lda, ldb, ldc, ca_c=1, stream_ptr=None) -> int:
+    """Direct call of ``sfc_gemm`` with raw device pointers; returns the status code."""
+    return load().sfc_gemm(int(M), int(N), int(K), ctypes.c_void_p(A_ptr), ctypes.c_void_p(B_ptr),
+                           ctypes.c_void_p(C_ptr), int(lda), int(ldb), int(ldc), int(ca_c),
+                           ctypes.c_void_p(stream_ptr))
+
+
+def device_status(stream=None) -> int:
+    """Synchronise the stream and return (and clear) the kernels' error word."""
+    return load().sfc_get_device_status(_stream_ptr(stream))
+
+
+def debug_force_timeout(A, B, C, limit_ms: int = 20, stream=None) -> int:
+    return load().sfc_debug_force_timeout(ctypes.c_void_p(A.data_ptr()), ctypes.c_void_p(B.data_ptr()),
+                                          ctypes.c_void_p(C.data_ptr()), int(limit_ms), _stream_ptr(stream))
+
+
+def matmul_host(A_host, B_host, C_host=None, *, ca_c: int = 1, out_dtype=None, stream=None, **kw):
+    """End-to-end call from HOST tensors: copy A and B (pinned for speed) to the
+    device, run the GEMM, copy C back into ``C_host`` (allocated pinned if not
+    given).  Returns C_host after the stream has synchronised."""
+    import torch
+    s = stream or torch.cuda.current_stream()
+    with torch.cuda.stream(s):
+        A = A_host.to("cuda", non_blocking=True)
+        B = B_host.to("cuda", non_blocking=True)
+        C = gemm(A, B, ca_c=ca_c, out_dtype=out_dtype, stream=s, **kw)
+        if C_host is None:
+            C_host = torch.empty(C.shape, dtype=C.dtype, pin_memory=True)
+        C_host.copy_(C, non_blocking=True)
+    s.synchronize()
+    return C_host

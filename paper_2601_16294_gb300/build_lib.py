@@ -1,0 +1,53 @@
+"""Build ``libsfcgemm.so`` in-tree with nvcc for sm_103a.
+
+Usage: ``python -m paper_2601_16294_gb300.build_lib`` (or ``build()`` from Python).
+The library links the CUDA runtime statically and resolves the driver's
+tensor-map encoder at run time, so it loads on machines without a GPU driver.
+"""
+from __future__ import annotations
+
+import os
+import subprocess
+import sys
+
+PKG = os.path.dirname(os.path.abspath(__file__))
+ROOT = os.path.dirname(PKG)
+CSRC = os.path.join(PKG, "csrc")
+INCLUDE = os.path.join(ROOT, "include")
+LIB = os.path.join(PKG, "libsfcgemm.so")
+SOURCES = [os.path.join(CSRC, "sfc_gemm.cu")]
+DEPS = SOURCES + [os.path.join(CSRC, f) for f in ("ptx.cuh", "sfc_curve.cuh", "sfc_gemm_kernel.cuh")] + [
+    os.path.join(INCLUDE, "sfc_gemm.h")]
+
+ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
+
+
+def nvcc() -> str:
+    cand = os.path.join(os.environ.get("CUDA_HOME", "/usr/local/cuda"), "bin", "nvcc")
+    return cand if os.path.exists(cand) else "nvcc"
+
+
+def up_to_date() -> bool:
+    if not os.path.exists(LIB):
+        return False
+    t = os.path.getmtime(LIB)
+    return all(os.path.getmtime(d) <= t for d in DEPS if os.path.exists(d))
+
+
+def build(force: bool = False, verbose: bool = False) -> str:
+    if not force and up_to_date():
+        return LIB
+    tmp = LIB + ".tmp%d" % os.getpid()
+    cmd = [nvcc(), "-std=c++17", "-O3", "-lineinfo", *ARCH, "-I", INCLUDE, "-I", CSRC,
+           "-Xcompiler", "-fPIC,-fvisibility=hidden", "-shared", "-o", tmp, *SOURCES]
+    if verbose:
+        cmd.insert(1, "-Xptxas=-v")
+        print(" ".join(cmd), file=sys.stderr)
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, LIB)
+    return LIB
+
+
+if __name__ == "__main__":
+    build(force="--force" in sys.argv, verbose="-v" in sys.argv)
+    print(LIB)

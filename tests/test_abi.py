@@ -1,0 +1,131 @@
+"""C ABI checks that need no GPU: the library builds, loads and exports every
+declared entry point; its host curve decoder equals the oracle; argument
+validation returns the documented codes before touching the device; without
+a usable GPU the compute entry points fail loudly instead of falling back."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import paper_2601_16294_gb300 as sfc
+from paper_2601_16294_gb300 import binding, build_lib
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "sfc_gemm.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build_lib.build()
+    return binding.load()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"^\s*(?:int|size_t|void)\s+\**(sfc_\w+)\s*\(", text, flags=re.M)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("sfc_tile_order", "sfc_gemm", "sfc_gemm_ex", "sfc_gemm_workspace_size"):
+        assert required in names
+    assert set(names) == set(binding.EXPORTS)
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+        assert ctypes.cast(getattr(lib, name), ctypes.c_void_p).value
+
+
+@pytest.mark.parametrize("Mt", range(1, 34))
+def test_host_decoder_matches_oracle_small(lib, oracle, Mt):
+    for Nt in range(1, 34):
+        assert np.array_equal(sfc.tile_order(Mt, Nt), oracle.gilbert_order(Mt, Nt)), (Mt, Nt)
+
+
+@pytest.mark.parametrize("Mt,Nt", [(4, 4), (128, 128), (128, 64), (64, 1002), (2, 64), (24, 40), (8, 133),
+                                   (48, 6), (4, 1002), (16, 501), (1002, 64), (65, 63), (1, 1002)])
+def test_host_decoder_matches_oracle_config_grids(lib, oracle, Mt, Nt):
+    assert np.array_equal(sfc.tile_order(Mt, Nt), oracle.gilbert_order(Mt, Nt))
+
+
+def test_tile_order_rejects_bad_arguments(lib):
+    buf = np.empty(4, dtype=np.int32)
+    assert lib.sfc_tile_order(0, 4, buf.ctypes.data) == binding.SFC_ERR_INVALID_ARG
+    assert lib.sfc_tile_order(4, -1, buf.ctypes.data) == binding.SFC_ERR_INVALID_ARG
+    assert lib.sfc_tile_order(2, 2, None) == binding.SFC_ERR_INVALID_ARG
+    assert lib.sfc_tile_order(65536, 65536, buf.ctypes.data) == binding.SFC_ERR_INVALID_ARG
+
+
+def test_workspace_size(lib):
+    assert sfc.workspace_size(512, 512, 4096, 1) == 0
+    assert sfc.workspace_size(512, 512, 4096, 4) == 4 * 512 * 512 * 4
+    assert sfc.workspace_size(3, 5, 64, 2) == 2 * 3 * 8 * 4          # rows padded to 4 floats
+    assert sfc.workspace_size(0, 5, 64, 2) == 0
+    assert sfc.workspace_size(3, 5, 64, 0) == 0
+
+
+# Fake, never-dereferenced device addresses: validation runs before any CUDA call.
+PA, PB, PC = 0x10000, 0x20000, 0x30000
+
+
+def call_ex(lib, M=256, N=256, K=256, A=PA, B=PB, C=PC, lda=None, ldb=None, ldc=None, ca_c=1, dtype=0,
+            order=0, assign=2, tile=0, ws=None, ws_bytes=0):
+    lda = K if lda is None else lda
+    ldb = N if ldb is None else ldb
+    ldc = N if ldc is None else ldc
+    return lib.sfc_gemm_ex(M, N, K, ctypes.c_void_p(A), ctypes.c_void_p(B), ctypes.c_void_p(C), lda, ldb, ldc,
+                           ca_c, dtype, order, assign, tile, ctypes.c_void_p(ws) if ws else None, ws_bytes, None)
+
+
+def test_gemm_validation_codes(lib):
+    E = binding
+    assert call_ex(lib, M=0) == E.SFC_ERR_INVALID_ARG
+    assert call_ex(lib, N=-1) == E.SFC_ERR_INVALID_ARG
+    assert call_ex(lib, K=0) == E.SFC_ERR_INVALID_ARG
+    assert call_ex(lib, A=0) == E.SFC_ERR_INVALID_ARG
+    assert call_ex(lib, C=0) == E.SFC_ERR_INVALID_ARG
+    assert call_ex(lib, lda=128) == E.SFC_ERR_INVALID_ARG          # lda < K
+    assert call_ex(lib, ldc=100) == E.SFC_ERR_INVALID_ARG          # ldc < N
+    assert call_ex(lib, ca_c=0) == E.SFC_ERR_INVALID_ARG
+    assert call_ex(lib, K=256, ca_c=5) == E.SFC_ERR_INVALID_ARG    # Kt = 4 < ca_c
+    assert call_ex(lib, dtype=7) == E.SFC_ERR_INVALID_ARG
+    assert call_ex(lib, order=3) == E.SFC_ERR_INVALID_ARG
+    assert call_ex(lib, assign=9) == E.SFC_ERR_INVALID_ARG
+    assert call_ex(lib, tile=64) == E.SFC_ERR_INVALID_ARG
+    assert call_ex(lib, A=PA + 8) == E.SFC_ERR_UNALIGNED           # A not 16-byte aligned
+    assert call_ex(lib, K=100, lda=100) == E.SFC_ERR_UNALIGNED     # 200-byte rows
+    assert call_ex(lib, N=260, ldb=260, ldc=260) == E.SFC_ERR_UNALIGNED
+    need = sfc.workspace_size(256, 256, 256, 2)
+    assert call_ex(lib, ca_c=2, ws=0x40000, ws_bytes=need - 4) == E.SFC_ERR_WORKSPACE
+    assert call_ex(lib, ca_c=2, ws=0x40008, ws_bytes=need) == E.SFC_ERR_UNALIGNED
+    assert lib.sfc_gemm(256, 256, 256, None, ctypes.c_void_p(PB), ctypes.c_void_p(PC), 256, 256, 256, 1,
+                        None) == E.SFC_ERR_INVALID_ARG
+    assert lib.sfc_debug_force_timeout(ctypes.c_void_p(PA), ctypes.c_void_p(PB), ctypes.c_void_p(PC), 0,
+                                       None) == E.SFC_ERR_INVALID_ARG
+
+
+def _has_gpu():
+    try:
+        import torch
+        return torch.cuda.is_available()
+    except Exception:
+        return False
+
+
+@pytest.mark.skipif(_has_gpu(), reason="checks the no-GPU failure path")
+def test_valid_call_without_gpu_fails_loudly(lib):
+    rc = call_ex(lib)
+    assert rc in (binding.SFC_ERR_CUDA, binding.SFC_ERR_UNSUPPORTED)
+    assert lib.sfc_num_workers() < 0
+    assert lib.sfc_get_device_status(None) == binding.SFC_ERR_CUDA
+
+
+def test_missing_library_raises(monkeypatch, tmp_path):
+    monkeypatch.setattr(binding, "_lib", None)
+    monkeypatch.setattr(binding, "library_path", lambda: str(tmp_path / "absent.so"))
+    with pytest.raises(binding.SfcLibraryMissing):
+        binding.load()
