@@ -152,6 +152,35 @@ int sfc_last_cuda_error(void);
 int sfc_num_workers(void);
 
 /*
+ * sfc_gemm_noalloc -- sfc_gemm_ex for callers that must not allocate memory.
+ *
+ * The paper has no counterpart: this is a deployment convenience.  Some
+ * callers cannot call cudaMalloc or use a stream-ordered pool at all -- code
+ * running inside a framework that owns every device allocation, a real-time
+ * path where an allocation may block or fail, or a process that has already
+ * handed all device memory to its own arena.  For them this entry point takes
+ * the fp32 partial copies of C (ca_c > 1) from a fixed scratch area compiled
+ * into the library, SFC_NOALLOC_SCRATCH_BYTES bytes of device memory that
+ * every GPU which loads the library holds until the process exits.  It calls
+ * no cudaMalloc, cudaFree or allocating library routine.
+ *
+ *   Arguments as sfc_gemm_ex with order = SFC, assign and tile = AUTO.
+ *   Errors: SFC_ERR_WORKSPACE (nothing launched) when
+ *           sfc_gemm_workspace_size(M, N, K, ca_c) > SFC_NOALLOC_SCRATCH_BYTES;
+ *           otherwise as sfc_gemm_ex.
+ * The first call on each device looks up the scratch area's device address
+ * (once per device, with that device current); make that first call before
+ * any stream capture.  All calls share the one scratch area and leave their
+ * partials in it: calls whose kernels can overlap on the GPU (different
+ * streams without ordering between them) race on it, so order them.
+ */
+#define SFC_NOALLOC_SCRATCH_BYTES ((size_t)32 << 20)
+int sfc_gemm_noalloc(int64_t M, int64_t N, int64_t K,
+                     const void *A, const void *B, void *C,
+                     int64_t lda, int64_t ldb, int64_t ldc,
+                     int ca_c, sfc_dtype_t c_dtype, void *stream);
+
+/*
  * sfc_debug_force_timeout -- test hook for the failure path: launches one GEMM
  * worker on a tiny problem whose MMA stage waits on a barrier that nothing
  * arrives at, with a wait limit of `limit_ms` milliseconds (1..1000).  The

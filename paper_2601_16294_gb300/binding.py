@@ -30,7 +30,9 @@ ASSIGNS = {"segment": 0, "wave": 1, "auto": 2}
 TILES = {0: 0, "auto": 0, 128: 128, 256: 256}
 
 EXPORTS = ("sfc_tile_order", "sfc_tile_order_device", "sfc_gemm_workspace_size", "sfc_gemm", "sfc_gemm_ex",
-           "sfc_get_device_status", "sfc_last_cuda_error", "sfc_num_workers", "sfc_debug_force_timeout")
+           "sfc_get_device_status", "sfc_last_cuda_error", "sfc_num_workers", "sfc_debug_force_timeout",
+           "sfc_gemm_noalloc")
+NOALLOC_SCRATCH_BYTES = 32 << 20
 
 
 class SfcLibraryMissing(RuntimeError):
@@ -77,6 +79,7 @@ def load():
         lib.sfc_last_cuda_error.argtypes = []
         lib.sfc_num_workers.argtypes = []
         lib.sfc_debug_force_timeout.argtypes = [vp, vp, vp, i32, vp]
+        lib.sfc_gemm_noalloc.argtypes = [i64, i64, i64, vp, vp, vp, i64, i64, i64, i32, i32, vp]
         for name in EXPORTS:
             if name != "sfc_gemm_workspace_size":
                 getattr(lib, name).restype = ctypes.c_int
@@ -162,6 +165,22 @@ def gemm(A, B, C=None, *, ca_c: int = 1, out_dtype=None, order: str = "sfc", ass
                          SFC_F32 if C.dtype == torch.float32 else SFC_BF16, ORDERS[order], ASSIGNS[assign],
                          TILES[tile], ws_ptr, ws_bytes, _stream_ptr(stream))
     _check(rc, "sfc_gemm_ex")
+    return C
+
+
+def gemm_noalloc(A, B, C, *, ca_c: int = 1, stream=None):
+    """C = A @ B through ``sfc_gemm_noalloc``: the K-layer partials use the
+    library's built-in scratch area, so the call allocates nothing.  C must be
+    preallocated (fp32 or bf16).  Raises SfcError(SFC_ERR_WORKSPACE) when the
+    partials would not fit in ``NOALLOC_SCRATCH_BYTES``."""
+    import torch
+    M, K = A.shape
+    N = B.shape[1]
+    rc = load().sfc_gemm_noalloc(M, N, K, ctypes.c_void_p(A.data_ptr()), ctypes.c_void_p(B.data_ptr()),
+                                 ctypes.c_void_p(C.data_ptr()), _row_major_2d(A, "A"), _row_major_2d(B, "B"),
+                                 _row_major_2d(C, "C"), int(ca_c),
+                                 SFC_F32 if C.dtype == torch.float32 else SFC_BF16, _stream_ptr(stream))
+    _check(rc, "sfc_gemm_noalloc")
     return C
 
 

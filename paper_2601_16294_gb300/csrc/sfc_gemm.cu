@@ -336,3 +336,52 @@ SFC_API int sfc_debug_force_timeout(const void* A, const void* B, void* C, int l
                     SFC_TILE_N128, nullptr, 0, static_cast<cudaStream_t>(stream), 1,
                     static_cast<uint64_t>(limit_ms) * 1000000ull);
 }
+
+// ---------------------------------------------------------------------------
+// Allocation-free entry point.  The fp32 partial copies of C live in a fixed
+// device array of this module instead of caller or pool memory; host code
+// must not pass the array's name to a kernel (on the host it is only a
+// stand-in symbol), so its device address is looked up once per device.
+// ---------------------------------------------------------------------------
+namespace sfc {
+namespace {
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[SFC_NOALLOC_SCRATCH_BYTES];
+
+struct NoAllocScratch {
+    std::once_flag once;
+    int status = SFC_ERR_CUDA;
+    void* ptr = nullptr;
+};
+NoAllocScratch g_noalloc[kMaxDevices];
+
+int noalloc_scratch(void** ptr) {
+    int dev;
+    int rc = current_device(&dev);
+    if (rc != SFC_OK) return rc;
+    NoAllocScratch& s = g_noalloc[dev];
+    std::call_once(s.once, [&]() {
+        void* p = nullptr;
+        cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess) { s.status = cuda_fail(e); return; }
+        s.ptr = p;
+        s.status = SFC_OK;
+    });
+    if (s.status == SFC_OK) *ptr = s.ptr;
+    return s.status;
+}
+
+}  // namespace
+}  // namespace sfc
+
+SFC_API int sfc_gemm_noalloc(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void* C,
+                             int64_t lda, int64_t ldb, int64_t ldc, int ca_c, sfc_dtype_t c_dtype,
+                             void* stream) {
+    if (sfc_gemm_workspace_size(M, N, K, ca_c) > SFC_NOALLOC_SCRATCH_BYTES) return SFC_ERR_WORKSPACE;
+    void* scratch = nullptr;
+    int rc = noalloc_scratch(&scratch);
+    if (rc != SFC_OK) return rc;
+    return sfc_gemm_ex(M, N, K, A, B, C, lda, ldb, ldc, ca_c, c_dtype, SFC_ORDER_SFC, SFC_ASSIGN_AUTO,
+                       SFC_TILE_AUTO, scratch, SFC_NOALLOC_SCRATCH_BYTES, stream);
+}
+
