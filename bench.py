@@ -1,11 +1,17 @@
 #!/usr/bin/env python3
 """Benchmark of the SFC bf16 GEMM on GB300.
 
-One step = one pass of the whole hot path over the square sweep
+Default workload ("square"): one step = one pass of the whole hot path over
 M = N = K in {2048, 4096, 8192, 16384} (bf16 inputs uniform in [-1, 1] from
 seed 0, fp32 accumulation, bf16 output, ca_c = 1, tiles ordered along the
 generalized Hilbert curve).  ``value`` is the weighted harmonic mean over the
-sweep, sum(2 M N K) / sum(time), in TFLOP/s, with inputs resident in HBM.
+step's shapes, sum(2 M N K) / time, in TFLOP/s, with inputs resident in HBM.
+
+Other workloads (``--workload``) measure the remaining shape sets the same way:
+``prefill`` (LLM-prefill projections), ``irregular`` (odd tile grids),
+``highk`` (the communication-avoiding K split), ``cube512`` (the small parity
+case).  Where a shape lists several K-layer counts, each is timed and the best
+one is used in the step (the paper reports the best replication factor too).
 
 Prints one JSON line (rank 0).  ``--impl reference`` times the CPU oracle (the
 plain fp64 triple loop) on sampled rows of the same workload instead.
@@ -28,13 +34,47 @@ if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
 METRIC = "bf16 GEMM TFLOP/s & % of GB300 dense peak; weighted harmonic mean over shapes"
-WORKLOAD = ("square bf16 GEMM sweep M=N=K in {2048, 4096, 8192, 16384}, uniform [-1,1] seeded inputs, "
-            "fp32 accumulate, bf16 output, ca_c=1")
-SIZES = (2048, 4096, 8192, 16384)
-FALLBACK_PEAKS = {"bf16_tflops": 1900.0, "hbm_gbs": 6800.0}
+FALLBACK_PEAKS = {"bf16_tflops": 1900.0, "hbm_gbs": 6800.0, "bf16_tflops_sustained": 1700.0}
 KERNEL_SOURCES = ("paper_2601_16294_gb300/csrc/sfc_gemm_kernel.cuh", "paper_2601_16294_gb300/csrc/ptx.cuh",
                   "paper_2601_16294_gb300/csrc/sfc_curve.cuh", "paper_2601_16294_gb300/csrc/sfc_gemm.cu")
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic_square_sweep.json")
+CS = (1, 2, 4, 8)
+
+
+def _shape(M, N, K, kind="uniform", out="bf16", cs=(1,)):
+    return {"M": M, "N": N, "K": K, "kind": kind, "out": out, "cs": tuple(cs)}
+
+
+WORKLOADS = {
+    "square": {
+        "desc": "square bf16 GEMM sweep M=N=K in {2048, 4096, 8192, 16384}, uniform [-1,1] seeded inputs, "
+                "fp32 accumulate, bf16 output, ca_c=1",
+        "shapes": [_shape(n, n, n) for n in (2048, 4096, 8192, 16384)],
+    },
+    "prefill": {
+        "desc": "LLM-prefill-shaped bf16 GEMMs: M in {512, 2048, 8192} x (N,K) in {(4096,4096), (14336,4096), "
+                "(4096,14336), (128256,4096)}, activations N(0,1), weights N(0,0.02) stored KxN, bf16 output, "
+                "best ca_c in {1,2,4,8}",
+        "shapes": [_shape(m, n, k, "prefill", "bf16", CS) for m in (512, 2048, 8192)
+                   for (n, k) in ((4096, 4096), (14336, 4096), (4096, 14336), (128256, 4096))],
+    },
+    "irregular": {
+        "desc": "irregular shapes 3000x5000x7000, 1000x17000x2500, 6144x768x12288, 129x8191x4096, uniform [-1,1], "
+                "bf16 output, rows padded to 16 bytes, best ca_c in {1,2,4,8}",
+        "shapes": [_shape(3000, 5000, 7000, cs=CS), _shape(1000, 17000, 2500, cs=CS),
+                   _shape(6144, 768, 12288, cs=CS), _shape(129, 8191, 4096, cs=CS)],
+    },
+    "highk": {
+        "desc": "communication-avoiding high-K cases M=N in {512, 1024, 2048} x K in {32768, 65536, 131072}, "
+                "uniform [-1,1], fp32 output, ca_c in {1,2,4,8} each timed, best in the step",
+        "shapes": [_shape(m, m, k, "uniform", "f32", CS) for m in (512, 1024, 2048)
+                   for k in (32768, 65536, 131072)],
+    },
+    "cube512": {
+        "desc": "single GEMM M=N=K=512, uniform [-1,1] seed 0, fp32 output, 4x4 grid of 128x128 tiles, ca_c=1",
+        "shapes": [_shape(512, 512, 512, "uniform", "f32")],
+    },
+}
 
 
 def parse_args():
@@ -43,14 +83,28 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
+    ap.add_argument("--workload", choices=sorted(WORKLOADS), default="square")
     ap.add_argument("--order", choices=("sfc", "raster"), default="sfc")
     ap.add_argument("--assign", choices=("auto", "wave", "segment"), default="auto")
-    ap.add_argument("--sizes", type=str, default=",".join(map(str, SIZES)),
-                    help="comma-separated square sizes (default: the full sweep)")
+    ap.add_argument("--sizes", type=str, default=None,
+                    help="square workload only: comma-separated sizes instead of the full sweep")
+    ap.add_argument("--ca-c", type=int, default=None, help="force one K-layer count for every shape")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
     return ap.parse_args()
+
+
+def workload_shapes(args):
+    shapes = [dict(s) for s in WORKLOADS[args.workload]["shapes"]]
+    if args.sizes:
+        if args.workload != "square":
+            raise SystemExit("--sizes applies to the square workload only")
+        shapes = [_shape(int(n), int(n), int(n)) for n in args.sizes.split(",")]
+    if args.ca_c is not None:
+        for s in shapes:
+            s["cs"] = (args.ca_c,)
+    return shapes
 
 
 def kernel_sha() -> str:
@@ -62,15 +116,24 @@ def kernel_sha() -> str:
 
 
 def load_peaks():
-    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
-        with open(path) as f:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
             d = json.load(f)
         return {"bf16_tflops": float(d["bf16_tflops"]), "hbm_gbs": float(d["hbm_gbs"]),
                 "bf16_tflops_sustained": float(d.get("bf16_tflops_sustained", d["bf16_tflops"])),
                 "source": "measured"}
     except Exception:
-        return dict(FALLBACK_PEAKS, bf16_tflops_sustained=1700.0, source="fallback")
+        return dict(FALLBACK_PEAKS, source="fallback")
+
+
+def roofline_time_s(s, peaks):
+    """max(compute time at the dense peak, compulsory bytes at HBM bandwidth)."""
+    o = 4 if s["out"] == "f32" else 2
+    flops = 2.0 * s["M"] * s["N"] * s["K"]
+    bytes_min = 2.0 * (s["M"] * s["K"] + s["K"] * s["N"]) + o * s["M"] * s["N"]
+    t_tc = flops / (peaks["bf16_tflops"] * 1e12)
+    t_hbm = bytes_min / (peaks["hbm_gbs"] * 1e9)
+    return max(t_tc, t_hbm), ("tensor" if t_tc >= t_hbm else "hbm")
 
 
 # ------------------------------------------------------------------ distributed
@@ -112,7 +175,6 @@ class ClockSampler:
 
     def __init__(self, device_index: int, enabled: bool = True):
         self.proc = None
-        self.index = device_index
         if not enabled:
             return
         try:
@@ -132,16 +194,16 @@ class ClockSampler:
         except Exception:
             self.proc.kill()
             out, _ = self.proc.communicate()
-        rows = list(csv.reader(io.StringIO(out)))
-        sm, mx, reasons = [], [], set()
+        sm, mx, power, reasons = [], [], [], set()
         names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
-        for r in rows:
+        for r in csv.reader(io.StringIO(out)):
             r = [x.strip() for x in r]
             if len(r) < 9:
                 continue
             try:
                 sm.append(float(r[1]))
                 mx.append(float(r[2]))
+                power.append(float(r[3]))
             except ValueError:
                 continue
             for name, val in zip(names, r[5:9]):
@@ -150,36 +212,73 @@ class ClockSampler:
         if not sm:
             return None
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "samples": len(sm),
-                "reasons": sorted(reasons)}
+                "power_w_max": max(power), "reasons": sorted(reasons)}
 
 
 # ------------------------------------------------------------------- our arm
 
+def make_inputs(s, synth, torch):
+    lda = synth.pad8(s["K"])
+    ldb = synth.pad8(s["N"])
+    A, B = synth.gemm_inputs(s["M"], s["N"], s["K"], s["kind"], seed=0, lda=lda, ldb=ldb)
+
+    def dev(t):
+        full = t.as_strided((t.shape[0], t.stride(0)), (t.stride(0), 1))
+        return full.contiguous().cuda()[:, : t.shape[1]]
+
+    out_dtype = torch.float32 if s["out"] == "f32" else torch.bfloat16
+    C = torch.empty((s["M"], s["N"]), dtype=out_dtype, device="cuda")
+    return A, B, dev(A), dev(B), C
+
+
 def run_ours(args, rank, local, world):
     import torch
     import paper_2601_16294_gb300 as sfc
-    from paper_2601_16294_gb300 import binding, synth
+    from paper_2601_16294_gb300 import synth
 
     torch.cuda.set_device(local)
     sfc.load()
     stream = torch.cuda.current_stream()
-    sizes = [int(s) for s in args.sizes.split(",")]
+    shapes = workload_shapes(args)
     peaks = load_peaks()
 
     # inputs resident in HBM before timing (seeded on the CPU, copied once)
     mats = []
-    for n in sizes:
-        A, B = synth.gemm_inputs(n, n, n, "uniform", seed=0)
-        mats.append((n, A.cuda(), B.cuda(), torch.empty((n, n), dtype=torch.bfloat16, device="cuda"), A, B))
+    for s in shapes:
+        A, B, Ad, Bd, C = make_inputs(s, synth, torch)
+        mats.append({"s": s, "A": A, "B": B, "Ad": Ad, "Bd": Bd, "C": C, "c": s["cs"][0]})
     torch.cuda.synchronize()
 
-    kw = dict(ca_c=1, order=args.order, assign=args.assign, stream=stream)
+    def call(m, c):
+        sfc.gemm(m["Ad"], m["Bd"], m["C"], ca_c=c, order=args.order, assign=args.assign, stream=stream)
+
+    # pick the K-layer count per shape where several are listed (timed, warm)
+    cs_report = {}
+    for i, m in enumerate(mats):
+        if len(m["s"]["cs"]) == 1:
+            continue
+        Kt = (m["s"]["K"] + 63) // 64
+        best = None
+        for c in [c for c in m["s"]["cs"] if c <= Kt]:
+            for _ in range(2):
+                call(m, c)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for _ in range(5):
+                call(m, c)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            t = e0.elapsed_time(e1) / 5
+            cs_report.setdefault(i, {})[c] = round(t, 4)
+            if best is None or t < best[1]:
+                best = (c, t)
+        m["c"] = best[0]
 
     def step(events=None):
-        for i, (n, A, B, C, _, _) in enumerate(mats):
+        for i, m in enumerate(mats):
             if events is not None:
                 events[i][0].record(stream)
-            sfc.gemm(A, B, C, **kw)
+            call(m, m["c"])
             if events is not None:
                 events[i][1].record(stream)
 
@@ -209,46 +308,53 @@ def run_ours(args, rank, local, world):
         raise RuntimeError("device-side timeout in the timed region (status %d)" % status)
 
     elapsed_ms = max_over_ranks(t0.elapsed_time(t1), world)
-    flops_step = sum(2.0 * n ** 3 for n, *_ in mats)
+    flops_step = sum(2.0 * m["s"]["M"] * m["s"]["N"] * m["s"]["K"] for m in mats)
     value = world * flops_step * args.steps / (elapsed_ms * 1e-3) / 1e12
     ms_per_step = elapsed_ms / args.steps
 
-    # per-shape kernel times (same launches, events on the launching stream)
     per_shape = []
-    tot_kernel_ms = 0.0
-    for i, (n, *_rest) in enumerate(mats):
+    tot_ms = 0.0
+    for i, m in enumerate(mats):
+        s = m["s"]
         ts = [per_launch[k][i][0].elapsed_time(per_launch[k][i][1]) for k in range(args.steps)]
         mean = sum(ts) / len(ts)
-        tot_kernel_ms += sum(ts)
-        tf = 2.0 * n ** 3 / (mean * 1e-3) / 1e12
-        per_shape.append({"M": n, "N": n, "K": n, "ms_mean": round(mean, 4), "ms_min": round(min(ts), 4),
-                          "tflops": round(tf, 1), "frac_of_peak": round(tf / peaks["bf16_tflops"], 4)})
+        tot_ms += sum(ts)
+        flops = 2.0 * s["M"] * s["N"] * s["K"]
+        t_roof, bound = roofline_time_s(s, peaks)
+        row = {"M": s["M"], "N": s["N"], "K": s["K"], "out": s["out"], "ca_c": m["c"],
+               "ms_mean": round(mean, 4), "ms_min": round(min(ts), 4),
+               "tflops": round(flops / (mean * 1e-3) / 1e12, 1), "bound": bound,
+               "frac_of_roofline": round(t_roof / (mean * 1e-3), 4)}
+        if i in cs_report:
+            row["ms_by_ca_c"] = cs_report[i]
+        per_shape.append(row)
 
-    # roofline of the dominant kernel (the GEMM kernel: every launch in the step)
-    launches = args.steps * len(mats)
-    achieved = flops_step * args.steps / (tot_kernel_ms * 1e-3) / 1e12
+    # roofline of the dominant kernel (the GEMM kernel; the K-layer reduction,
+    # when used, is inside the same per-shape event pairs)
+    achieved = flops_step * args.steps / (tot_ms * 1e-3) / 1e12
     traffic = None
     try:
         with open(TRAFFIC_FILE) as f:
             tr = json.load(f)
-        if tr.get("kernel_sha") == kernel_sha() and tr.get("sizes") == sizes:
+        if tr.get("kernel_sha") == kernel_sha() and tr.get("workload") == args.workload and not args.sizes:
             traffic = tr["dram_bytes_per_launch"]
     except Exception:
         traffic = None
     roofline = {"bound": "tensor", "achieved": round(achieved, 1), "peak": peaks["bf16_tflops"],
                 "unit": "TFLOP/s", "frac": round(achieved / peaks["bf16_tflops"], 4), "traffic": traffic,
-                "kernel": "sfc_gemm_kernel<256,4,bf16>", "peak_source": peaks["source"] + " bf16 burst",
-                "frac_of_sustained": round(achieved / peaks["bf16_tflops_sustained"], 4)}
-
+                "kernel": "sfc_gemm_kernel", "peak_source": peaks["source"] + " dense bf16 (burst)",
+                "frac_of_sustained_peak": round(achieved / peaks["bf16_tflops_sustained"], 4)}
+    launches = args.steps * sum(1 if m["c"] == 1 else 2 for m in mats)
+    desc = WORKLOADS[args.workload]["desc"] if not args.sizes else "square sweep sizes %s" % args.sizes
     result = {
         "metric": METRIC, "value": round(value, 1), "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "data": "synthetic (seeded uniform [-1,1] bf16)",
-        "config": {"workload": WORKLOAD, "sizes": sizes, "order": args.order, "assign": args.assign,
+        "data": "synthetic (seeded %s bf16)" % ",".join(sorted({m["s"]["kind"] for m in mats})),
+        "config": {"workload": desc, "order": args.order, "assign": args.assign,
                    "parallelism": "replicas" if world > 1 else "single GPU",
-                   "l2": "inputs larger than L2 between reuses: each shape's operands are re-read only "
-                         "after the other shapes' GEMMs (>1.5 GB of traffic) have passed through L2",
+                   "l2": "inputs larger than L2 between reuses: one step runs every shape once, so a shape's "
+                         "operands are re-read only after the other shapes' traffic has passed through L2",
                    "pct_of_dense_peak": round(100.0 * value / world / peaks["bf16_tflops"], 2)},
         "roofline": roofline,
         "gpu_launches": launches,
@@ -256,11 +362,10 @@ def run_ours(args, rank, local, world):
     }
     if clock_info is not None:
         result["clocks"] = clock_info
-
     if not args.no_e2e:
         result["e2e"] = run_e2e(args, mats, stream, world)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        result["cpu_baseline"] = run_cpu_baseline(args, mats)
+        result["cpu_baseline"] = run_cpu_baseline(mats)
     return result
 
 
@@ -271,17 +376,17 @@ def run_e2e(args, mats, stream, world):
     import paper_2601_16294_gb300 as sfc
 
     host = []
-    for n, A, B, C, Acpu, Bcpu in mats:
-        host.append((n, Acpu.pin_memory(), Bcpu.pin_memory(),
-                     torch.empty((n, n), dtype=torch.bfloat16, pin_memory=True)))
-    h2d = sum(2 * 2 * n * n for n, *_ in host)
-    d2h = sum(2 * n * n for n, *_ in host)
+    for m in mats:
+        host.append((m, m["A"].contiguous().pin_memory(), m["B"].contiguous().pin_memory(),
+                     torch.empty(m["C"].shape, dtype=m["C"].dtype, pin_memory=True)))
+    h2d = sum(Ah.numel() * 2 + Bh.numel() * 2 for _, Ah, Bh, _ in host)
+    d2h = sum(Ch.numel() * Ch.element_size() for _, _, _, Ch in host)
 
     def step():
-        for n, Ah, Bh, Ch in host:
-            sfc.matmul_host(Ah, Bh, Ch, out_dtype=torch.bfloat16, stream=stream)
+        for m, Ah, Bh, Ch in host:
+            sfc.matmul_host(Ah, Bh, Ch, ca_c=m["c"], out_dtype=Ch.dtype, stream=stream)
 
-    for _ in range(max(1, min(args.warmup, 2))):
+    for _ in range(2):
         step()
     steps = max(1, min(args.steps, 5))
     barrier(world)
@@ -291,7 +396,7 @@ def run_e2e(args, mats, stream, world):
         step()
     torch.cuda.synchronize()
     el = max_over_ranks(time.perf_counter() - t, world)
-    flops = sum(2.0 * n ** 3 for n, *_ in host) * steps * world
+    flops = sum(2.0 * m["s"]["M"] * m["s"]["N"] * m["s"]["K"] for m in mats) * steps * world
     return {"value": round(flops / el / 1e12, 1), "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": steps,
             "api": "paper_2601_16294_gb300.matmul_host -> sfc_gemm_ex (C ABI)"}
@@ -312,48 +417,51 @@ def oracle_sample(mats_cpu, rows):
     oracle.build()
     flops = 0.0
     t = 0.0
-    for n, A, B in mats_cpu:
-        r = np.linspace(0, n - 1, rows).astype(np.int64)
+    for A, B in mats_cpu:
+        M, K = A.shape
+        N = B.shape[1]
+        r = np.linspace(0, M - 1, min(rows, M)).astype(np.int64)
         A_rows = A[r].contiguous()
+        Bc = B.contiguous()
         t0 = time.perf_counter()
-        oracle.gemm_f64(A_rows, B)
+        oracle.gemm_f64(A_rows, Bc)
         t += time.perf_counter() - t0
-        flops += 2.0 * rows * n * n
+        flops += 2.0 * r.size * N * K
     return flops, t
 
 
-def run_cpu_baseline(args, mats):
+def run_cpu_baseline(mats):
     """The oracle as it stands, on this host's cores, on a bounded sample of the
     workload: a 16-row probe sets the row count for about 12 s of CPU work."""
     os.environ.setdefault("OMP_NUM_THREADS", str(cpu_cores()))
-    mats_cpu = [(n, Acpu, Bcpu) for n, _, _, _, Acpu, Bcpu in mats]
-    f_probe, s_probe = oracle_sample(mats_cpu, 16)
+    mats_cpu = [(m["A"], m["B"]) for m in mats]
+    _, s_probe = oracle_sample(mats_cpu, 16)
     rows = int(min(1024, max(16, 16 * 12.0 / max(s_probe, 1e-3))))
     rows = max(16, rows // 16 * 16)
     flops, secs = oracle_sample(mats_cpu, rows)
     return {"value": round(flops / secs / 1e12, 6), "unit": "TFLOP/s",
             "cores": int(os.environ["OMP_NUM_THREADS"]), "kind": "oracle", "seconds": round(secs, 2),
-            "sample": "%d evenly spaced rows of C for each square shape (fp64 i-k-j triple loop, "
-                      "OpenMP over rows)" % rows}
+            "sample": "%d evenly spaced rows of C for each shape (fp64 i-k-j triple loop, OpenMP over rows)"
+                      % rows}
 
 
 # ------------------------------------------------------------- reference arm
 
 def run_reference(args, rank, world):
     """The CPU oracle as the reference arm: each step computes sampled rows of
-    every shape of the sweep (bounded so the run ends within minutes)."""
+    every shape of the workload (bounded so the run ends within minutes)."""
     if rank != 0:
         return None
     from paper_2601_16294_gb300 import synth
     os.environ.setdefault("OMP_NUM_THREADS", str(cpu_cores()))
-    sizes = [int(s) for s in args.sizes.split(",")]
+    shapes = workload_shapes(args)
     mats_cpu = []
-    for n in sizes:
-        A, B = synth.gemm_inputs(n, n, n, "uniform", seed=0)
-        mats_cpu.append((n, A, B))
+    for s in shapes:
+        A, B = synth.gemm_inputs(s["M"], s["N"], s["K"], s["kind"], seed=0)
+        mats_cpu.append((A, B))
     rows = 16
     for _ in range(args.warmup):
-        oracle_sample(mats_cpu, 4)
+        oracle_sample(mats_cpu, 2)
     flops = secs = 0.0
     for _ in range(args.steps):
         f, s = oracle_sample(mats_cpu, rows)
@@ -361,12 +469,12 @@ def run_reference(args, rank, world):
         secs += s
     value = flops / secs / 1e12
     cores = int(os.environ["OMP_NUM_THREADS"])
-    sample = "%d evenly spaced rows of C per square shape per step" % rows
+    sample = "%d evenly spaced rows of C per shape per step" % rows
+    desc = WORKLOADS[args.workload]["desc"] if not args.sizes else "square sweep sizes %s" % args.sizes
     return {"impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": "TFLOP/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(1e3 * secs / args.steps, 2),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic (seeded uniform [-1,1] bf16)",
-            "config": {"workload": WORKLOAD, "sizes": sizes, "sample": sample},
+            "data": "synthetic (seeded bf16)", "config": {"workload": desc, "sample": sample},
             "cpu_baseline": {"value": round(value, 6), "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": round(value, 6), "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},

@@ -68,8 +68,18 @@ typedef enum { SFC_ORDER_SFC = 0, SFC_ORDER_RASTER = 1 } sfc_order_t;
  * AUTO:    the library picks (currently WAVE). */
 typedef enum { SFC_ASSIGN_SEGMENT = 0, SFC_ASSIGN_WAVE = 1, SFC_ASSIGN_AUTO = 2 } sfc_assign_t;
 
-/* Output tile width.  AUTO picks per shape; 128 and 256 force it. bm is 128. */
-typedef enum { SFC_TILE_AUTO = 0, SFC_TILE_N128 = 128, SFC_TILE_N256 = 256 } sfc_tile_t;
+/* Output tile shape and the hardware that computes it.
+ * N128 / N256:           128 x 128 / 128 x 256 tiles, one SM each.
+ * PAIR_N128 / PAIR_N256: 256 x 128 / 256 x 256 tiles computed by a pair of SMs
+ *                        (a 2-CTA cluster; each SM loads half of A and half of B).
+ * AUTO picks per shape from the tile count and the number of workers. */
+typedef enum {
+    SFC_TILE_AUTO = 0,
+    SFC_TILE_N128 = 128,
+    SFC_TILE_N256 = 256,
+    SFC_TILE_PAIR_N128 = 1128,
+    SFC_TILE_PAIR_N256 = 1256
+} sfc_tile_t;
 
 /*
  * sfc_tile_order -- the curve permutation over an Mt x Nt tile grid
@@ -110,6 +120,12 @@ size_t sfc_gemm_workspace_size(int64_t M, int64_t N, int64_t K, int ca_c);
  *   stream: a cudaStream_t passed as void*.
  * Requirements: A and B 16-byte aligned, lda and ldb multiples of 8 (the tile
  * loads use the Tensor Memory Accelerator).  C may have any alignment.
+ * Accuracy: products are exact and summed in fp32; the tensor core's running
+ * sum is restarted every 4096 values of k and the partial sums are added with
+ * round-to-nearest fp32 adds, which bounds the error growth of very long K.
+ * (Experiments only: the environment variable SFC_GEMM_CHUNK_SLABS, read once
+ * per device, sets that restart interval in units of 64 values of k; 0 turns
+ * the restarts off.)
  * Errors: SFC_ERR_INVALID_ARG, SFC_ERR_UNALIGNED, SFC_ERR_CUDA, SFC_ERR_UNSUPPORTED.
  */
 int sfc_gemm(int64_t M, int64_t N, int64_t K,

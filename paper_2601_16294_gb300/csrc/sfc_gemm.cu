@@ -6,11 +6,13 @@
 
 #include <atomic>
 #include <cstdint>
+#include <cstdlib>
 #include <cstring>
 #include <mutex>
 
 #include "sfc_gemm.h"
 #include "sfc_gemm_kernel.cuh"
+#include "sfc_gemm_pair_kernel.cuh"
 
 #define SFC_API extern "C" __attribute__((visibility("default")))
 
@@ -29,10 +31,74 @@ int cuda_fail(cudaError_t e) {
 
 // ---------------------------------------------------------- per-device state
 
+// Kernel variants.  Stage counts fill ~192 KB of shared memory per block.
+enum Variant { kSingle128 = 0, kSingle256 = 1, kPair128 = 2, kPair256 = 3, kNumVariants = 4 };
+constexpr int kStagesSingle256 = 4;  // 48 KB stages
+constexpr int kStagesSingle128 = 6;  // 32 KB stages
+constexpr int kStagesPair256 = 6;    // 32 KB stages per CTA
+constexpr int kStagesPair128 = 8;    // 24 KB stages per CTA
+constexpr int kDefaultChunkSlabs = 64;  // 4096 values of k per tensor-memory accumulation chain
+
+constexpr int variant_bn(int v) { return (v == kSingle128 || v == kPair128) ? 128 : 256; }
+constexpr bool variant_pair(int v) { return v == kPair128 || v == kPair256; }
+
+template <int BN, int STAGES>
+constexpr int single_smem() { return RingLayout<(kBM + BN) * kBK * 2, STAGES>::kDynamicBytes; }
+template <int BN, int STAGES>
+constexpr int pair_smem() { return RingLayout<PairStage<BN>::kBytes, STAGES>::kDynamicBytes; }
+
+template <typename OutT>
+struct Kernels {
+    static constexpr void (*single128)(CUtensorMap, CUtensorMap, GemmParams) =
+        sfc_gemm_kernel<128, kStagesSingle128, OutT>;
+    static constexpr void (*single256)(CUtensorMap, CUtensorMap, GemmParams) =
+        sfc_gemm_kernel<256, kStagesSingle256, OutT>;
+    static constexpr void (*pair128)(CUtensorMap, CUtensorMap, GemmParams) =
+        sfc_gemm_pair_kernel<128, kStagesPair128, OutT>;
+    static constexpr void (*pair256)(CUtensorMap, CUtensorMap, GemmParams) =
+        sfc_gemm_pair_kernel<256, kStagesPair256, OutT>;
+    static void (*get(int v))(CUtensorMap, CUtensorMap, GemmParams) {
+        switch (v) {
+            case kSingle128: return single128;
+            case kSingle256: return single256;
+            case kPair128: return pair128;
+            default: return pair256;
+        }
+    }
+};
+
+constexpr int variant_smem(int v) {
+    return v == kSingle128   ? single_smem<128, kStagesSingle128>()
+           : v == kSingle256 ? single_smem<256, kStagesSingle256>()
+           : v == kPair128   ? pair_smem<128, kStagesPair128>()
+                             : pair_smem<256, kStagesPair256>();
+}
+
+cudaLaunchConfig_t launch_config(int v, int grid, cudaStream_t s, cudaLaunchAttribute* attr) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid, 1, 1);
+    cfg.blockDim = dim3(block_threads(variant_bn(v)), 1, 1);
+    cfg.dynamicSmemBytes = variant_smem(v);
+    cfg.stream = s;
+    cfg.attrs = nullptr;
+    cfg.numAttrs = 0;
+    if (variant_pair(v)) {
+        attr->id = cudaLaunchAttributeClusterDimension;
+        attr->val.clusterDim.x = 2;
+        attr->val.clusterDim.y = 1;
+        attr->val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+    }
+    return cfg;
+}
+
 struct DeviceInfo {
     std::once_flag once;
     int status = SFC_ERR_UNSUPPORTED;
     int num_sms = 0;
+    int chunk_slabs = kDefaultChunkSlabs;
+    int workers[kNumVariants] = {0, 0, 0, 0};  // co-resident workers (blocks or pairs) per variant
 };
 DeviceInfo g_devices[kMaxDevices];
 
@@ -43,19 +109,21 @@ int current_device(int* dev) {
     return SFC_OK;
 }
 
-template <int BN, int STAGES, typename OutT>
-cudaError_t set_smem_attr() {
-    return cudaFuncSetAttribute(sfc_gemm_kernel<BN, STAGES, OutT>,
-                                cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                SmemLayout<BN, STAGES>::kDynamicBytes);
+template <typename OutT>
+cudaError_t set_attrs() {
+    for (int v = 0; v < kNumVariants; ++v) {
+        cudaError_t e = cudaFuncSetAttribute(Kernels<OutT>::get(v), cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             variant_smem(v));
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
 }
 
-constexpr int kStages256 = 4;  // 4 x 48 KB ring
-constexpr int kStages128 = 6;  // 6 x 32 KB ring
-
 // One-time set-up of the current device: check it is an sm_103 part, read its
-// SM count, raise the shared-memory limit of every kernel instantiation.
-int device_setup(int* num_sms) {
+// SM count, raise the shared-memory limit of every kernel instantiation, and
+// find how many 2-SM pairs can be resident at once (clusters must fit in one
+// GPC, so this can be fewer than half the SMs).
+int device_setup(DeviceInfo** info) {
     int dev;
     int rc = current_device(&dev);
     if (rc != SFC_OK) return rc;
@@ -66,15 +134,29 @@ int device_setup(int* num_sms) {
         if (e != cudaSuccess) { d.status = cuda_fail(e); return; }
         if (prop.major != 10 || prop.minor != 3) { d.status = SFC_ERR_UNSUPPORTED; return; }
         d.num_sms = prop.multiProcessorCount;
-        cudaError_t errs[] = {
-            set_smem_attr<256, kStages256, float>(), set_smem_attr<256, kStages256, __nv_bfloat16>(),
-            set_smem_attr<128, kStages128, float>(), set_smem_attr<128, kStages128, __nv_bfloat16>(),
-        };
-        for (cudaError_t x : errs)
-            if (x != cudaSuccess) { d.status = cuda_fail(x); return; }
+        // experiment override of the accumulation chain length (slabs of 64 k; 0 = one chain per item)
+        if (const char* env = std::getenv("SFC_GEMM_CHUNK_SLABS")) {
+            const int v = std::atoi(env);
+            d.chunk_slabs = v > 0 ? v : (1 << 30);
+        }
+        e = set_attrs<float>();
+        if (e == cudaSuccess) e = set_attrs<__nv_bfloat16>();
+        if (e != cudaSuccess) { d.status = cuda_fail(e); return; }
+        for (int v = 0; v < kNumVariants; ++v) {
+            if (!variant_pair(v)) {
+                d.workers[v] = d.num_sms;
+                continue;
+            }
+            cudaLaunchAttribute attr;
+            cudaLaunchConfig_t cfg = launch_config(v, d.num_sms, nullptr, &attr);
+            int clusters = 0;
+            e = cudaOccupancyMaxActiveClusters(&clusters, Kernels<float>::get(v), &cfg);
+            if (e != cudaSuccess) { d.status = cuda_fail(e); return; }
+            d.workers[v] = clusters;
+        }
         d.status = SFC_OK;
     });
-    if (d.status == SFC_OK) *num_sms = d.num_sms;
+    if (d.status == SFC_OK) *info = &d;
     return d.status;
 }
 
@@ -119,21 +201,36 @@ int make_bf16_map(CUtensorMap* map, const void* ptr, int64_t rows, int64_t cols,
 
 // ------------------------------------------------------------------ planning
 
-struct Plan {
-    int64_t M, N, K;
-    int Mt, Nt, Kt, bn, ca_c, grid;
-    int64_t items;
-};
-
 int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
-int pick_bn(int64_t M, int64_t N, int ca_c, int num_sms, sfc_tile_t tile) {
-    if (tile == SFC_TILE_N128) return 128;
-    if (tile == SFC_TILE_N256) return 256;
-    // wide tiles halve the shared-memory traffic per flop; use them when they
-    // still give every SM at least one item
-    const int64_t items256 = ceil_div(M, kBM) * ceil_div(N, 256) * ca_c;
-    return items256 >= num_sms ? 256 : 128;
+// Tile shape for a call.  AUTO estimates each variant's time as
+// (waves of items) x (per-SM work of one item) / (its relative efficiency) and
+// takes the fastest; 2-SM pairs move half the B bytes per flop of one SM.
+int pick_variant(int64_t M, int64_t N, int ca_c, const DeviceInfo& d, sfc_tile_t tile) {
+    switch (tile) {
+        case SFC_TILE_N128: return kSingle128;
+        case SFC_TILE_N256: return kSingle256;
+        case SFC_TILE_PAIR_N128: return d.workers[kPair128] > 0 ? kPair128 : kSingle128;
+        case SFC_TILE_PAIR_N256: return d.workers[kPair256] > 0 ? kPair256 : kSingle256;
+        default: break;
+    }
+    // relative tensor-pipe efficiency measured on GB300 (256-wide tiles feed the
+    // tensor core with fewer shared-memory bytes per flop)
+    static const double eff[kNumVariants] = {0.50, 0.85, 0.55, 0.95};
+    int best = kSingle128;
+    double best_t = 0.0;
+    for (int v = 0; v < kNumVariants; ++v) {
+        if (d.workers[v] <= 0) continue;
+        const int bm = variant_pair(v) ? 256 : 128, bn = variant_bn(v);
+        const int64_t items = ((M + bm - 1) / bm) * ((N + bn - 1) / bn) * ca_c;
+        const int64_t waves = (items + d.workers[v] - 1) / d.workers[v];
+        const double t = static_cast<double>(waves) * 128.0 * bn / eff[v];
+        if (v == kSingle128 || t < best_t) {
+            best = v;
+            best_t = t;
+        }
+    }
+    return best;
 }
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
@@ -146,7 +243,9 @@ int validate(int64_t M, int64_t N, int64_t K, const void* A, const void* B, cons
     if (order != SFC_ORDER_SFC && order != SFC_ORDER_RASTER) return SFC_ERR_INVALID_ARG;
     if (assign != SFC_ASSIGN_SEGMENT && assign != SFC_ASSIGN_WAVE && assign != SFC_ASSIGN_AUTO)
         return SFC_ERR_INVALID_ARG;
-    if (tile != SFC_TILE_AUTO && tile != SFC_TILE_N128 && tile != SFC_TILE_N256) return SFC_ERR_INVALID_ARG;
+    if (tile != SFC_TILE_AUTO && tile != SFC_TILE_N128 && tile != SFC_TILE_N256 && tile != SFC_TILE_PAIR_N128 &&
+        tile != SFC_TILE_PAIR_N256)
+        return SFC_ERR_INVALID_ARG;
     // TMA coordinates and tile indices are 32-bit
     if (M > (int64_t(1) << 31) - kBM || N > (int64_t(1) << 31) - 256 || K > (int64_t(1) << 31) - kBK)
         return SFC_ERR_INVALID_ARG;
@@ -160,19 +259,13 @@ int validate(int64_t M, int64_t N, int64_t K, const void* A, const void* B, cons
 
 int64_t ws_ld(int64_t N) { return (N + 3) / 4 * 4; }
 
-template <int BN, int STAGES, typename OutT>
-cudaError_t launch_gemm(const CUtensorMap& ta, const CUtensorMap& tb, const GemmParams& p, int grid,
-                        cudaStream_t s) {
-    sfc_gemm_kernel<BN, STAGES, OutT>
-        <<<grid, kThreads, SmemLayout<BN, STAGES>::kDynamicBytes, s>>>(ta, tb, p);
-    return cudaGetLastError();
-}
-
 template <typename OutT>
-cudaError_t dispatch_bn(int bn, const CUtensorMap& ta, const CUtensorMap& tb, const GemmParams& p, int grid,
+cudaError_t launch_gemm(int v, const CUtensorMap& ta, const CUtensorMap& tb, const GemmParams& p, int grid,
                         cudaStream_t s) {
-    if (bn == 256) return launch_gemm<256, kStages256, OutT>(ta, tb, p, grid, s);
-    return launch_gemm<128, kStages128, OutT>(ta, tb, p, grid, s);
+    cudaLaunchAttribute attr;
+    cudaLaunchConfig_t cfg = launch_config(v, grid, s, &attr);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, Kernels<OutT>::get(v), ta, tb, p);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void* C, int64_t lda, int64_t ldb,
@@ -184,13 +277,15 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     if (workspace && workspace_bytes < ws_need) return SFC_ERR_WORKSPACE;
     if (workspace && !aligned16(workspace)) return SFC_ERR_UNALIGNED;
 
-    int num_sms = 0;
-    rc = device_setup(&num_sms);
+    DeviceInfo* dev = nullptr;
+    rc = device_setup(&dev);
     if (rc != SFC_OK) return rc;
 
-    const int bn = pick_bn(M, N, ca_c, num_sms, static_cast<sfc_tile_t>(tile));
+    const int v = pick_variant(M, N, ca_c, *dev, static_cast<sfc_tile_t>(tile));
+    const int bn = variant_bn(v);
+    const int bm = variant_pair(v) ? kPairBM : kBM;
     CUtensorMap ta, tb;
-    rc = make_bf16_map(&ta, A, M, K, lda, kBM, kBK);
+    rc = make_bf16_map(&ta, A, M, K, lda, kBM, kBK);  // each CTA loads 128 rows of A
     if (rc != SFC_OK) return rc;
     rc = make_bf16_map(&tb, B, K, N, ldb, kBK, kBBox);
     if (rc != SFC_OK) return rc;
@@ -198,16 +293,19 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     GemmParams p;
     p.M = M;
     p.N = N;
-    p.Mt = static_cast<int>(ceil_div(M, kBM));
+    p.Mt = static_cast<int>(ceil_div(M, bm));
     p.Nt = static_cast<int>(ceil_div(N, bn));
     p.Kt = static_cast<int>(ceil_div(K, kBK));
     p.ca_c = ca_c;
+    p.kc = dev->chunk_slabs;
     p.num_items = static_cast<int64_t>(p.Mt) * p.Nt * ca_c;
     p.order = order;
     p.assign = (assign == SFC_ASSIGN_SEGMENT) ? 0 : 1;
     p.debug_never = debug_never;
     p.timeout_ns = timeout_ns;
-    const int grid = static_cast<int>(p.num_items < num_sms ? p.num_items : num_sms);
+    const int64_t workers = dev->workers[v];
+    const int64_t used = p.num_items < workers ? p.num_items : workers;
+    const int grid = static_cast<int>(variant_pair(v) ? 2 * used : used);
 
     void* ws = workspace;
     bool pooled = false;
@@ -224,18 +322,18 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
         p.layer_stride = 0;
         const size_t esz = (c_dtype == SFC_F32) ? 4 : 2;
         p.vec_store = aligned16(C) && ((ldc * esz) % 16 == 0);
-        e = (c_dtype == SFC_F32) ? dispatch_bn<float>(bn, ta, tb, p, grid, stream)
-                                 : dispatch_bn<__nv_bfloat16>(bn, ta, tb, p, grid, stream);
+        e = (c_dtype == SFC_F32) ? launch_gemm<float>(v, ta, tb, p, grid, stream)
+                                 : launch_gemm<__nv_bfloat16>(v, ta, tb, p, grid, stream);
     } else {
         p.out = ws;
         p.ldo = ws_ld(N);
         p.layer_stride = M * p.ldo;
         p.vec_store = 1;
-        e = dispatch_bn<float>(bn, ta, tb, p, grid, stream);
+        e = launch_gemm<float>(v, ta, tb, p, grid, stream);
         if (e == cudaSuccess) {
             const int64_t work = M * ((N + 3) / 4);
             int64_t blocks = ceil_div(work, 256);
-            const int64_t cap = static_cast<int64_t>(num_sms) * 8;
+            const int64_t cap = static_cast<int64_t>(dev->num_sms) * 8;
             if (blocks > cap) blocks = cap;
             const int vec = (c_dtype == SFC_F32) ? (aligned16(C) && (ldc % 4) == 0)
                                                  : (((reinterpret_cast<uintptr_t>(C) & 7u) == 0) && (ldc % 4) == 0);
@@ -278,8 +376,8 @@ SFC_API int sfc_tile_order_device(int Mt, int Nt, int32_t* out_idx_dev, void* st
     if (Mt < 1 || Nt < 1 || !out_idx_dev) return SFC_ERR_INVALID_ARG;
     const int64_t n = static_cast<int64_t>(Mt) * Nt;
     if (n > INT32_MAX) return SFC_ERR_INVALID_ARG;
-    int num_sms = 0;
-    int rc = device_setup(&num_sms);
+    DeviceInfo* dev = nullptr;
+    int rc = device_setup(&dev);
     if (rc != SFC_OK) return rc;
     int64_t blocks = (n + 255) / 256;
     if (blocks > 65535) blocks = 65535;
@@ -325,9 +423,9 @@ SFC_API int sfc_get_device_status(void* stream) {
 SFC_API int sfc_last_cuda_error(void) { return t_last_cuda_error; }
 
 SFC_API int sfc_num_workers(void) {
-    int n = 0;
-    int rc = device_setup(&n);
-    return rc == SFC_OK ? n : rc;
+    DeviceInfo* dev = nullptr;
+    int rc = device_setup(&dev);
+    return rc == SFC_OK ? dev->num_sms : rc;
 }
 
 SFC_API int sfc_debug_force_timeout(const void* A, const void* B, void* C, int limit_ms, void* stream) {

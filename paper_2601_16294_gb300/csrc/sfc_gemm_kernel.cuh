@@ -1,25 +1,32 @@
-// sfc_gemm_kernel.cuh -- persistent SFC / SFC-CA GEMM kernel for sm_103a.
+// sfc_gemm_kernel.cuh -- persistent SFC / SFC-CA GEMM kernels for sm_103a.
 //
-// One thread block per SM walks its share of the task space of Listing 1
-// (Mt*Nt*K_layers items: item i -> K layer i / (Mt*Nt), curve position
-// i % (Mt*Nt) -> output tile).  For each item it contracts the layer's K range
-// of one 128 x BN output tile (the paper's batch-reduce GEMM over K blocks,
-// Sec. II-A; C is zeroed at the first K block, Listing 1) on the tcgen05
-// tensor cores:
+// A block (or a 2-SM pair of blocks) resident on each SM walks its share of
+// the task space of Listing 1: Mt*Nt*K_layers items, item i -> K layer
+// i / (Mt*Nt), curve position i % (Mt*Nt) -> output tile.  For each item it
+// contracts the layer's K range of one output tile (the paper's batch-reduce
+// GEMM over K blocks, Sec. II-A; C is zeroed at the first K block, Listing 1)
+// on the tcgen05 tensor cores:
 //
-//   warp 0      TMA producer: loads 128x64 A and 64xBN B slabs (bf16, 128-byte
-//               swizzle) into a STAGES-deep shared-memory ring, completion on
-//               the stage's "full" mbarrier;
-//   warp 1      MMA issuer: 4 x tcgen05.mma (128 x BN x 16) per slab into one
-//               of two tensor-memory accumulators; tcgen05.commit frees the
-//               ring stage and, after the last slab, publishes the accumulator;
-//   warps 2..5  epilogue: tcgen05.ld the accumulator (warp w reads TMEM lanes
-//               32*(w%4)...), convert, store the tile (masked at the M/N edges),
-//               then hand the accumulator back.  Two accumulators let the
-//               epilogue of one tile overlap the main loop of the next.
+//   warp 0        TMA producer: 64-wide K slabs of A and B (bf16, 128-byte
+//                 swizzle) into a STAGES-deep shared-memory ring;
+//   warp 1        MMA issuer: tcgen05.mma (K = 16 each) into one of two
+//                 tensor-memory accumulators; tcgen05.commit frees ring stages
+//                 and publishes finished accumulators;
+//   warps 2..     epilogue: tcgen05.ld the accumulator (warp w reads TMEM lanes
+//                 32*(w%4)..), add it into fp32 running sums held in registers,
+//                 and after the item's last chunk convert and store the tile
+//                 (masked at the M/N edges).
 //
-// With K_layers > 1 the epilogue writes the layer's fp32 partial tile to the
-// workspace copy of C for that layer; ca_reduce_kernel sums the copies.
+// Accumulation chains.  The tensor core's fp32 accumulation drops low-order
+// bits on every accumulate, so the error of one long chain grows linearly with
+// K.  Each item's K range is therefore cut into chunks of at most p.kc slabs;
+// every chunk restarts the tensor-memory accumulator and the epilogue adds the
+// chunk's result into its register running sum with round-to-nearest fp32
+// adds.  Two accumulators let chunk j+1 run on the tensor core while the
+// epilogue drains chunk j, and the last chunk of a tile overlap the next tile.
+//
+// With K_layers > 1 the epilogue writes the layer's fp32 partial tile to that
+// layer's workspace copy of C; ca_reduce_kernel sums the copies in layer order.
 //
 // Every mbarrier wait is bounded (globaltimer).  A wait that runs out sets the
 // device error word and a block-wide abort flag; all roles then leave their
@@ -35,11 +42,15 @@
 
 namespace sfc {
 
-constexpr int kBM = 128;            // output tile rows (UMMA M)
-constexpr int kBK = 64;             // K slab: 64 bf16 = one 128-byte swizzle row
-constexpr int kUmmaK = 16;          // K per tcgen05.mma for 16-bit inputs
-constexpr int kThreads = 192;       // 6 warps
-constexpr int kBBox = 64;           // B is loaded in 64-column boxes (128 bytes)
+constexpr int kBM = 128;          // output tile rows per CTA (UMMA M of one CTA)
+constexpr int kBK = 64;           // K slab: 64 bf16 = one 128-byte swizzle row
+constexpr int kUmmaK = 16;        // K per tcgen05.mma for 16-bit inputs
+constexpr int kBBox = 64;         // B is loaded in 64-column boxes (128 bytes)
+constexpr int kEpiCols = 128;     // accumulator columns each epilogue thread owns
+
+// Threads of a block: producer warp, MMA warp, BN/32 epilogue warps
+// (4 warps per 128 columns: one warp per TMEM lane quarter).
+__host__ __device__ constexpr int block_threads(int bn) { return 64 + 32 * (bn / 32); }
 
 // device error word: bit 0 = a bounded wait gave up; bits 8.. = which wait
 __device__ unsigned int g_sfc_status = 0;
@@ -55,8 +66,9 @@ enum WaitSite : unsigned int {
 
 struct GemmParams {
     int64_t M, N;
-    int Mt, Nt, Kt;
-    int ca_c;
+    int Mt, Nt, Kt;        // tile grid and number of 64-wide K slabs
+    int ca_c;              // K layers
+    int kc;                // max slabs per tensor-memory accumulation chain
     int64_t num_items;     // Mt * Nt * ca_c
     void* out;             // C when ca_c == 1, else the fp32 workspace
     int64_t ldo;           // row stride of `out` in elements
@@ -66,20 +78,6 @@ struct GemmParams {
     int vec_store;         // 1 if 16-byte vector stores are aligned
     int debug_never;       // test hook: MMA warp waits on a barrier nobody arrives at
     uint64_t timeout_ns;   // bound for every mbarrier wait
-};
-
-template <int BN, int STAGES>
-struct SmemLayout {
-    static constexpr int kABytes = kBM * kBK * 2;
-    static constexpr int kBBytes = BN * kBK * 2;
-    static constexpr int kStageBytes = kABytes + kBBytes;
-    static constexpr int kRingBytes = kStageBytes * STAGES;
-    static constexpr int kNumBars = 2 * STAGES + 6;  // full, empty, acc full x2, acc empty x2, drain, never
-    static constexpr int kBarOffset = kRingBytes;
-    static constexpr int kMiscOffset = kBarOffset + kNumBars * 8;
-    static constexpr int kBytes = kMiscOffset + 16;
-    static constexpr int kDynamicBytes = kBytes + 1024;  // slack to align the ring to 1024 B
-    static_assert(kABytes % 1024 == 0 && kBBytes % 1024 == 0, "swizzle atoms need 1 KB alignment");
 };
 
 struct WorkItem {
@@ -100,18 +98,26 @@ __device__ __forceinline__ WorkItem decode_item(int64_t i, const GemmParams& p) 
     return w;
 }
 
-// Items of this block: [first, end) with stride `step`.
-__device__ __forceinline__ void block_items(const GemmParams& p, int64_t& first, int64_t& end,
-                                            int64_t& step) {
-    const int64_t P = gridDim.x, b = blockIdx.x;
+// Chunks of an item's K range: n = ceil(len / kc), boundaries balanced.
+__device__ __forceinline__ int num_chunks(const WorkItem& w, int kc) {
+    const int len = w.k1 - w.k0;
+    return (len + kc - 1) / kc;
+}
+__device__ __forceinline__ int chunk_begin(const WorkItem& w, int j, int n) {
+    return w.k0 + static_cast<int>((static_cast<int64_t>(j) * (w.k1 - w.k0)) / n);
+}
+
+// Items of worker `worker` out of `workers`: [first, end) with stride `step`.
+__device__ __forceinline__ void worker_items(const GemmParams& p, int64_t worker, int64_t workers,
+                                             int64_t& first, int64_t& end, int64_t& step) {
     if (p.assign == 0) {
-        first = b * p.num_items / P;
-        end = (b + 1) * p.num_items / P;
+        first = worker * p.num_items / workers;
+        end = (worker + 1) * p.num_items / workers;
         step = 1;
     } else {
-        first = b;
+        first = worker;
         end = p.num_items;
-        step = P;
+        step = workers;
     }
 }
 
@@ -140,17 +146,14 @@ __device__ __forceinline__ float cvt_out<float>(float v) { return v; }
 template <>
 __device__ __forceinline__ __nv_bfloat16 cvt_out<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
 
-// Store 32 consecutive accumulator columns of one row.
+// Store 32 consecutive columns v[0..31] of one row, starting at column col0.
 template <typename OutT>
-__device__ __forceinline__ void store_chunk(OutT* row_ptr, int64_t col0, int64_t N, const uint32_t (&r)[32],
-                                            bool vec) {
+__device__ __forceinline__ void store_chunk(OutT* row_ptr, int64_t col0, int64_t N, const float* v, bool vec) {
     if (vec && col0 + 32 <= N) {
         if constexpr (sizeof(OutT) == 4) {
             float4* dst = reinterpret_cast<float4*>(row_ptr + col0);
 #pragma unroll
-            for (int j = 0; j < 8; ++j)
-                dst[j] = make_float4(__uint_as_float(r[4 * j]), __uint_as_float(r[4 * j + 1]),
-                                     __uint_as_float(r[4 * j + 2]), __uint_as_float(r[4 * j + 3]));
+            for (int j = 0; j < 8; ++j) dst[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
         } else {
             uint4* dst = reinterpret_cast<uint4*>(row_ptr + col0);
 #pragma unroll
@@ -158,9 +161,8 @@ __device__ __forceinline__ void store_chunk(OutT* row_ptr, int64_t col0, int64_t
                 uint32_t w[4];
 #pragma unroll
                 for (int h = 0; h < 4; ++h) {
-                    __nv_bfloat162 v = __floats2bfloat162_rn(__uint_as_float(r[8 * j + 2 * h]),
-                                                             __uint_as_float(r[8 * j + 2 * h + 1]));
-                    w[h] = *reinterpret_cast<uint32_t*>(&v);
+                    __nv_bfloat162 b = __floats2bfloat162_rn(v[8 * j + 2 * h], v[8 * j + 2 * h + 1]);
+                    w[h] = *reinterpret_cast<uint32_t*>(&b);
                 }
                 dst[j] = make_uint4(w[0], w[1], w[2], w[3]);
             }
@@ -168,49 +170,140 @@ __device__ __forceinline__ void store_chunk(OutT* row_ptr, int64_t col0, int64_t
     } else {
 #pragma unroll
         for (int j = 0; j < 32; ++j)
-            if (col0 + j < N) row_ptr[col0 + j] = cvt_out<OutT>(__uint_as_float(r[j]));
+            if (col0 + j < N) row_ptr[col0 + j] = cvt_out<OutT>(v[j]);
     }
 }
 
+// Per-block barrier set and smem layout shared by both kernels.
+struct Barriers {
+    uint32_t bars;
+    int stages;
+    __device__ __forceinline__ uint32_t full(int s) const { return bars + 8u * s; }
+    __device__ __forceinline__ uint32_t empty(int s) const { return bars + 8u * (stages + s); }
+    __device__ __forceinline__ uint32_t acc_full(int a) const { return bars + 8u * (2 * stages + a); }
+    __device__ __forceinline__ uint32_t acc_empty(int a) const { return bars + 8u * (2 * stages + 2 + a); }
+    __device__ __forceinline__ uint32_t drain() const { return bars + 8u * (2 * stages + 4); }
+    __device__ __forceinline__ uint32_t never() const { return bars + 8u * (2 * stages + 5); }
+};
+
+template <int STAGE_BYTES, int STAGES>
+struct RingLayout {
+    static constexpr int kRingBytes = STAGE_BYTES * STAGES;
+    static constexpr int kNumBars = 2 * STAGES + 6;
+    static constexpr int kBarOffset = kRingBytes;
+    static constexpr int kMiscOffset = kBarOffset + kNumBars * 8;
+    static constexpr int kBytes = kMiscOffset + 16;
+    static constexpr int kDynamicBytes = kBytes + 1024;  // slack to align the ring to 1024 B
+};
+
+// -------------------------------------------------------------------------
+// Epilogue of one block: drain chunks, promote, store.  `rows_base` is the
+// first output row this block's TMEM lanes map to for tile row tm.
+// -------------------------------------------------------------------------
+template <int BN, typename OutT, bool PAIR>
+__device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers& B, uint32_t tmem_base,
+                                             volatile int* abort_flag, int64_t first, int64_t end,
+                                             int64_t step, int tile_rows, int row_offset, int warp, int lane) {
+    const int ew = warp - 2;                 // epilogue warp index
+    const int quarter = warp & 3;            // TMEM lane quarter this warp may access
+    const int half = ew / 4;                 // which 128-column half of the tile
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    OutT* out = static_cast<OutT*>(p.out);
+    const uint32_t acce_target = PAIR ? ptx::map_to_cta(B.acc_empty(0), 0) : B.acc_empty(0);
+    float run[kEpiCols];
+    for (int64_t it = first; it < end; it += step) {
+        const WorkItem w = decode_item(it, p);
+        const int nch = num_chunks(w, p.kc);
+        bool ok = true;
+        for (int ck = 0; ck < nch; ++ck) {
+            int ready = 1;
+            if (lane == 0)
+                ready = wait_bounded(B.acc_full(acc), acc_phase, abort_flag, p.timeout_ns, kWaitEpiAccFull);
+            ready = __shfl_sync(0xffffffffu, ready, 0);
+            if (!ready) {
+                ok = false;
+                break;
+            }
+            ptx::tc_fence_after();
+            const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
+                                   static_cast<uint32_t>(acc * BN + half * kEpiCols);
+#pragma unroll
+            for (int g = 0; g < kEpiCols / 32; ++g) {
+                uint32_t r[32];
+                ptx::tmem_ld_32x32b_x32(taddr + g * 32, r);
+                ptx::tmem_ld_wait();
+                if (ck == 0) {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) run[g * 32 + j] = __uint_as_float(r[j]);
+                } else {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) run[g * 32 + j] = __fadd_rn(run[g * 32 + j], __uint_as_float(r[j]));
+                }
+            }
+            ptx::tc_fence_before();
+            __syncwarp();
+            if (lane == 0) {
+                // the accumulator-empty barriers are 8 bytes apart
+                if (PAIR) ptx::mbar_arrive_cluster(acce_target + 8u * acc);
+                else ptx::mbar_arrive(B.acc_empty(acc));
+            }
+            if (++acc == 2) {
+                acc = 0;
+                acc_phase ^= 1u;
+            }
+        }
+        if (!ok) break;
+        const int64_t row = static_cast<int64_t>(w.tm) * tile_rows + row_offset + quarter * 32 + lane;
+        if (row < p.M) {
+            OutT* row_ptr = out + static_cast<int64_t>(w.layer) * p.layer_stride + row * p.ldo;
+            const int64_t col_base = static_cast<int64_t>(w.tn) * BN + half * kEpiCols;
+#pragma unroll
+            for (int g = 0; g < kEpiCols / 32; ++g)
+                store_chunk<OutT>(row_ptr, col_base + g * 32, p.N, run + g * 32, p.vec_store != 0);
+        }
+    }
+}
+
+// -------------------------------------------------------------------------
+// Single-SM kernel: 128 x BN tiles, UMMA 128 x BN x 16.
+// -------------------------------------------------------------------------
 template <int BN, int STAGES, typename OutT>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(block_threads(BN), 1)
 sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_b,
                 const GemmParams p) {
-    using L = SmemLayout<BN, STAGES>;
-    static_assert(BN % kBBox == 0 && BN >= 64 && BN <= 256, "BN must be 64..256 in steps of 64");
-    static_assert(2 * BN <= 512, "two accumulators must fit in 512 TMEM columns");
+    static_assert(BN == 128 || BN == 256, "tiles are 128 x 128 or 128 x 256");
+    constexpr int kABytes = kBM * kBK * 2;
+    constexpr int kBBytes = BN * kBK * 2;
+    constexpr int kStageBytes = kABytes + kBBytes;
+    using L = RingLayout<kStageBytes, STAGES>;
     constexpr uint32_t kIdesc = ptx::idesc_bf16_f32(kBM, BN, /*A K-major*/ 0, /*B MN-major*/ 1);
     constexpr uint32_t kTmemCols = 2 * BN;
+    constexpr int kEpiWarps = BN / 32;
 
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = ptx::smem_addr(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
     uint8_t* smem = smem_raw + (base - raw);
     const uint32_t ring = base;
-    const uint32_t bars = base + L::kBarOffset;
-    const uint32_t drain_bar = bars + 8 * (2 * STAGES + 4);
-    const uint32_t never_bar = bars + 8 * (2 * STAGES + 5);
+    const Barriers B{base + L::kBarOffset, STAGES};
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::kMiscOffset);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::kMiscOffset + 4);
-    auto full_bar = [&](int s) { return bars + 8u * s; };
-    auto empty_bar = [&](int s) { return bars + 8u * (STAGES + s); };
-    auto accf_bar = [&](int a) { return bars + 8u * (2 * STAGES + a); };
-    auto acce_bar = [&](int a) { return bars + 8u * (2 * STAGES + 2 + a); };
 
     const int warp = threadIdx.x / 32;
     const int lane = threadIdx.x % 32;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
-            ptx::mbar_init(full_bar(s), 1);
-            ptx::mbar_init(empty_bar(s), 1);
+            ptx::mbar_init(B.full(s), 1);
+            ptx::mbar_init(B.empty(s), 1);
         }
         for (int a = 0; a < 2; ++a) {
-            ptx::mbar_init(accf_bar(a), 1);
-            ptx::mbar_init(acce_bar(a), 4);  // one arrive per epilogue warp
+            ptx::mbar_init(B.acc_full(a), 1);
+            ptx::mbar_init(B.acc_empty(a), kEpiWarps);  // one arrive per epilogue warp
         }
-        ptx::mbar_init(drain_bar, 1);
-        ptx::mbar_init(never_bar, 1);
+        ptx::mbar_init(B.drain(), 1);
+        ptx::mbar_init(B.never(), 1);
         *abort_flag = 0;
         ptx::fence_barrier_init();
     }
@@ -228,7 +321,7 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
     const uint32_t tmem_base = *tmem_slot;
 
     int64_t first, end, step;
-    block_items(p, first, end, step);
+    worker_items(p, blockIdx.x, gridDim.x, first, end, step);
 
     if (warp == 0) {
         // ------------------------------------------------------ TMA producer
@@ -240,19 +333,18 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
             for (int64_t it = first; ok && it < end; it += step) {
                 const WorkItem w = decode_item(it, p);
                 for (int kt = w.k0; kt < w.k1; ++kt) {
-                    if (!wait_bounded(empty_bar(stage), phase ^ 1u, abort_flag, p.timeout_ns,
-                                      kWaitProducerEmpty)) {
+                    if (!wait_bounded(B.empty(stage), phase ^ 1u, abort_flag, p.timeout_ns, kWaitProducerEmpty)) {
                         ok = false;
                         break;
                     }
-                    ptx::mbar_arrive_expect_tx(full_bar(stage), L::kStageBytes);
-                    const uint32_t sa = ring + stage * L::kStageBytes;
-                    const uint32_t sb = sa + L::kABytes;
-                    ptx::tma_load_2d(sa, &tmap_a, full_bar(stage), kt * kBK, w.tm * kBM);
+                    ptx::mbar_arrive_expect_tx(B.full(stage), kStageBytes);
+                    const uint32_t sa = ring + stage * kStageBytes;
+                    const uint32_t sb = sa + kABytes;
+                    ptx::tma_load_2d(sa, &tmap_a, B.full(stage), kt * kBK, w.tm * kBM);
 #pragma unroll
                     for (int j = 0; j < BN / kBBox; ++j)
-                        ptx::tma_load_2d(sb + j * (kBBox * kBK * 2), &tmap_b, full_bar(stage),
-                                         w.tn * BN + j * kBBox, kt * kBK);
+                        ptx::tma_load_2d(sb + j * (kBBox * kBK * 2), &tmap_b, B.full(stage), w.tn * BN + j * kBBox,
+                                         kt * kBK);
                     ++issued;
                     if (++stage == STAGES) {
                         stage = 0;
@@ -267,11 +359,9 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
             for (int64_t n = n0; n < issued; ++n) {
                 const int slot = static_cast<int>(n % STAGES);
                 const uint32_t par = static_cast<uint32_t>((n / STAGES) & 1);
-                if (ok)
-                    ok = wait_bounded(empty_bar(slot), par, abort_flag, p.timeout_ns, kWaitProducerEmpty);
+                if (ok) ok = wait_bounded(B.empty(slot), par, abort_flag, p.timeout_ns, kWaitProducerEmpty);
                 if (!ok)
-                    wait_bounded(full_bar(slot), par, abort_flag, p.timeout_ns, kWaitDrain,
-                                 /*honour_abort=*/false);
+                    wait_bounded(B.full(slot), par, abort_flag, p.timeout_ns, kWaitDrain, /*honour_abort=*/false);
             }
         }
     } else if (warp == 1) {
@@ -282,89 +372,57 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
             int acc = 0;
             uint32_t acc_phase = 0;
             bool ok = true;
-            if (p.debug_never)
-                ok = wait_bounded(never_bar, 0, abort_flag, p.timeout_ns, kWaitDebugNever);
+            if (p.debug_never) ok = wait_bounded(B.never(), 0, abort_flag, p.timeout_ns, kWaitDebugNever);
             for (int64_t it = first; ok && it < end; it += step) {
                 const WorkItem w = decode_item(it, p);
-                if (!wait_bounded(acce_bar(acc), acc_phase ^ 1u, abort_flag, p.timeout_ns,
-                                  kWaitMmaAccEmpty)) {
-                    ok = false;
-                    break;
-                }
-                ptx::tc_fence_after();
-                const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
-                for (int kt = w.k0; kt < w.k1; ++kt) {
-                    if (!wait_bounded(full_bar(stage), phase, abort_flag, p.timeout_ns, kWaitMmaFull)) {
+                const int nch = num_chunks(w, p.kc);
+                for (int ck = 0; ok && ck < nch; ++ck) {
+                    const int kb = chunk_begin(w, ck, nch), ke = chunk_begin(w, ck + 1, nch);
+                    if (!wait_bounded(B.acc_empty(acc), acc_phase ^ 1u, abort_flag, p.timeout_ns, kWaitMmaAccEmpty)) {
                         ok = false;
                         break;
                     }
                     ptx::tc_fence_after();
-                    const uint32_t sa = ring + stage * L::kStageBytes;
-                    const uint32_t sb = sa + L::kABytes;
+                    const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
+                    for (int kt = kb; kt < ke; ++kt) {
+                        if (!wait_bounded(B.full(stage), phase, abort_flag, p.timeout_ns, kWaitMmaFull)) {
+                            ok = false;
+                            break;
+                        }
+                        ptx::tc_fence_after();
+                        const uint32_t sa = ring + stage * kStageBytes;
+                        const uint32_t sb = sa + kABytes;
 #pragma unroll
-                    for (int kk = 0; kk < kBK / kUmmaK; ++kk) {
-                        // A: K-major, 128-byte rows, 8-row atoms 1024 B apart; step 32 B per K=16
-                        const uint64_t adesc = ptx::smem_desc_sw128(sa + kk * (kUmmaK * 2), 16, 1024);
-                        // B: MN-major, 64-column boxes 8 KB apart, 8-row atoms 1024 B apart;
-                        // step 16 rows (2 KB) per K=16
-                        const uint64_t bdesc =
-                            ptx::smem_desc_sw128(sb + kk * (kUmmaK * 128), kBBox * kBK * 2, 1024);
-                        ptx::tc_mma_f16(d_tmem, adesc, bdesc, kIdesc, (kt > w.k0 || kk > 0) ? 1u : 0u);
+                        for (int kk = 0; kk < kBK / kUmmaK; ++kk) {
+                            // A: K-major, 128-byte rows, 8-row atoms 1024 B apart; 32 B per K=16
+                            const uint64_t adesc = ptx::smem_desc_sw128(sa + kk * (kUmmaK * 2), 16, 1024);
+                            // B: MN-major, 64-column boxes 8 KB apart, 8-row atoms 1 KB apart; 2 KB per K=16
+                            const uint64_t bdesc =
+                                ptx::smem_desc_sw128(sb + kk * (kUmmaK * 128), kBBox * kBK * 2, 1024);
+                            ptx::tc_mma_f16(d_tmem, adesc, bdesc, kIdesc, (kt > kb || kk > 0) ? 1u : 0u);
+                        }
+                        ptx::tc_commit(B.empty(stage));  // frees the stage once these MMAs finish
+                        if (++stage == STAGES) {
+                            stage = 0;
+                            phase ^= 1u;
+                        }
                     }
-                    ptx::tc_commit(empty_bar(stage));  // frees the stage once these MMAs finish
-                    if (++stage == STAGES) {
-                        stage = 0;
-                        phase ^= 1u;
+                    if (!ok) break;
+                    ptx::tc_commit(B.acc_full(acc));  // chunk ready for the epilogue
+                    if (++acc == 2) {
+                        acc = 0;
+                        acc_phase ^= 1u;
                     }
-                }
-                if (!ok) break;
-                ptx::tc_commit(accf_bar(acc));  // accumulator ready for the epilogue
-                if (++acc == 2) {
-                    acc = 0;
-                    acc_phase ^= 1u;
                 }
             }
             if (!ok) {
                 // wait (bounded) until every MMA issued so far has finished
-                ptx::tc_commit(drain_bar);
-                wait_bounded(drain_bar, 0, abort_flag, p.timeout_ns, kWaitDrain, /*honour_abort=*/false);
+                ptx::tc_commit(B.drain());
+                wait_bounded(B.drain(), 0, abort_flag, p.timeout_ns, kWaitDrain, /*honour_abort=*/false);
             }
         }
     } else {
-        // ---------------------------------------------------------- epilogue
-        const int quarter = warp & 3;  // TMEM lanes 32*quarter .. +31
-        int acc = 0;
-        uint32_t acc_phase = 0;
-        OutT* out = static_cast<OutT*>(p.out);
-        for (int64_t it = first; it < end; it += step) {
-            const WorkItem w = decode_item(it, p);
-            // lane 0 waits, the warp follows its verdict (tcgen05.ld needs the whole warp)
-            int ready = 1;
-            if (lane == 0)
-                ready = wait_bounded(accf_bar(acc), acc_phase, abort_flag, p.timeout_ns, kWaitEpiAccFull);
-            ready = __shfl_sync(0xffffffffu, ready, 0);
-            if (!ready) break;
-            ptx::tc_fence_after();
-            const int64_t row = static_cast<int64_t>(w.tm) * kBM + quarter * 32 + lane;
-            OutT* row_ptr = out + static_cast<int64_t>(w.layer) * p.layer_stride + row * p.ldo;
-            const uint32_t taddr =
-                tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + static_cast<uint32_t>(acc * BN);
-            const int64_t col_base = static_cast<int64_t>(w.tn) * BN;
-#pragma unroll 1
-            for (int ch = 0; ch < BN / 32; ++ch) {
-                uint32_t r[32];
-                ptx::tmem_ld_32x32b_x32(taddr + ch * 32, r);
-                ptx::tmem_ld_wait();
-                if (row < p.M) store_chunk<OutT>(row_ptr, col_base + ch * 32, p.N, r, p.vec_store != 0);
-            }
-            ptx::tc_fence_before();
-            __syncwarp();
-            if (lane == 0) ptx::mbar_arrive(acce_bar(acc));
-            if (++acc == 2) {
-                acc = 0;
-                acc_phase ^= 1u;
-            }
-        }
+        run_epilogue<BN, OutT, false>(p, B, tmem_base, abort_flag, first, end, step, kBM, 0, warp, lane);
     }
 
     ptx::tc_fence_before();
@@ -413,7 +471,7 @@ ca_reduce_kernel(const float* __restrict__ ws, int64_t ldw, int64_t layer_stride
     }
 }
 
-// out[s] = tm * Nt + tn for every curve position s, with the kernel's decoder.
+// out[s] = tm * Nt + tn for every curve position s, with the kernels' decoder.
 __global__ void tile_order_kernel(int Mt, int Nt, int32_t* __restrict__ out) {
     const int64_t n = static_cast<int64_t>(Mt) * Nt;
     for (int64_t s = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; s < n;

@@ -1,0 +1,220 @@
+// sfc_gemm_pair_kernel.cuh -- the SFC / SFC-CA GEMM on 2-SM CTA pairs.
+//
+// Same task space, item order, accumulation chunks and epilogue as
+// sfc_gemm_kernel, but each worker is a cluster of two CTAs on two SMs that
+// computes a 256 x BN output tile with tcgen05.mma.cta_group::2 (UMMA M = 256):
+//
+//   - CTA r of the pair loads rows [128 r, 128 r + 128) of the A slab and
+//     columns [r BN/2, (r+1) BN/2) of the B slab into its own shared memory;
+//     both CTAs' TMA copies complete on the leader CTA's "full" barrier;
+//   - the leader's MMA warp issues the pair MMAs.  Each SM's tensor core uses
+//     its own A half and both B halves, so a 256 x BN tile costs each SM
+//     128 x 64 + 64 x BN/2 bf16 of shared-memory and L2 traffic per slab,
+//     against 128 x 64 + 64 x BN for a 128 x BN tile on one SM;
+//   - MMA completion (tcgen05.commit ... multicast) frees the ring stage in
+//     both CTAs and publishes the accumulator chunk to both epilogues;
+//   - CTA r's tensor memory holds rows [128 r, 128 r + 128) of the tile; its
+//     epilogue warps drain them and arrive on the leader's accumulator-empty
+//     barrier.
+//
+// Waits are bounded as in the single-SM kernel.  The pair meets at a cluster
+// barrier after set-up (barriers initialised before any remote signal) and
+// before exit (no CTA leaves while its peer may still signal it); then both
+// CTAs free their tensor memory.
+#pragma once
+
+#include "sfc_gemm_kernel.cuh"
+
+namespace sfc {
+
+constexpr int kPairBM = 256;  // output tile rows of a pair (128 per CTA)
+
+template <int BN>
+struct PairStage {
+    static constexpr int kHalfN = BN / 2;
+    static constexpr int kABytes = 128 * kBK * 2;
+    static constexpr int kBBytes = kHalfN * kBK * 2;
+    static constexpr int kBytes = kABytes + kBBytes;
+    static_assert(kABytes % 1024 == 0 && kBBytes % 1024 == 0, "swizzle atoms need 1 KB alignment");
+};
+
+template <int BN, int STAGES, typename OutT>
+__global__ void __launch_bounds__(block_threads(BN), 1)
+sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_b,
+                     const GemmParams p) {
+    static_assert(BN == 128 || BN == 256, "pair tiles are 256 x 128 or 256 x 256");
+    using S = PairStage<BN>;
+    using L = RingLayout<S::kBytes, STAGES>;
+    constexpr int kHalfN = S::kHalfN;
+    constexpr uint32_t kIdesc = ptx::idesc_bf16_f32(kPairBM, BN, /*A K-major*/ 0, /*B MN-major*/ 1);
+    constexpr uint32_t kTmemCols = 2 * BN;
+    constexpr int kEpiWarps = BN / 32;
+    constexpr uint16_t kBothCtas = 0x3;
+
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw = ptx::smem_addr(smem_raw);
+    const uint32_t base = (raw + 1023u) & ~1023u;
+    uint8_t* smem = smem_raw + (base - raw);
+    const uint32_t ring = base;
+    const Barriers B{base + L::kBarOffset, STAGES};
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + L::kMiscOffset);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::kMiscOffset + 4);
+
+    const int warp = threadIdx.x / 32;
+    const int lane = threadIdx.x % 32;
+    const uint32_t rank = ptx::cluster_ctarank();
+    const bool leader = (rank == 0);
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            ptx::mbar_init(B.full(s), 1);   // the leader's producer arrives once (+ both CTAs' bytes)
+            ptx::mbar_init(B.empty(s), 1);  // one multicast commit per use of the stage
+        }
+        for (int a = 0; a < 2; ++a) {
+            ptx::mbar_init(B.acc_full(a), 1);               // one multicast commit per chunk
+            ptx::mbar_init(B.acc_empty(a), 2 * kEpiWarps);  // epilogue warps of both CTAs (leader's copy used)
+        }
+        ptx::mbar_init(B.drain(), 1);
+        ptx::mbar_init(B.never(), 1);
+        *abort_flag = 0;
+        ptx::fence_barrier_init();
+    }
+    if (warp == 0 && lane == 0) {
+        ptx::tma_prefetch_desc(&tmap_a);
+        ptx::tma_prefetch_desc(&tmap_b);
+    }
+    if (warp == 1) {
+        ptx::tmem_alloc_pair(ptx::smem_addr(tmem_slot), kTmemCols);
+        ptx::tmem_relinquish_pair();
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::cluster_sync();  // the peer's barriers are initialised before anyone signals them
+    ptx::tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+
+    int64_t first, end, step;
+    worker_items(p, blockIdx.x / 2, gridDim.x / 2, first, end, step);
+
+    if (warp == 0) {
+        // ------------------------------------------------ TMA producer (both CTAs)
+        if (lane == 0) {
+            int stage = 0;
+            uint32_t phase = 0;
+            int64_t issued = 0;
+            bool ok = true;
+            for (int64_t it = first; ok && it < end; it += step) {
+                const WorkItem w = decode_item(it, p);
+                const int32_t a_row = w.tm * kPairBM + static_cast<int32_t>(rank) * 128;
+                const int32_t b_col = w.tn * BN + static_cast<int32_t>(rank) * kHalfN;
+                for (int kt = w.k0; kt < w.k1; ++kt) {
+                    if (!wait_bounded(B.empty(stage), phase ^ 1u, abort_flag, p.timeout_ns, kWaitProducerEmpty)) {
+                        ok = false;
+                        break;
+                    }
+                    if (leader) ptx::mbar_arrive_expect_tx(B.full(stage), 2 * S::kBytes);
+                    const uint32_t leader_full = ptx::map_to_cta(B.full(stage), 0);
+                    const uint32_t sa = ring + stage * S::kBytes;
+                    const uint32_t sb = sa + S::kABytes;
+                    ptx::tma_load_2d_pair(sa, &tmap_a, leader_full, kt * kBK, a_row);
+#pragma unroll
+                    for (int j = 0; j < kHalfN / kBBox; ++j)
+                        ptx::tma_load_2d_pair(sb + j * (kBBox * kBK * 2), &tmap_b, leader_full, b_col + j * kBBox,
+                                              kt * kBK);
+                    ++issued;
+                    if (++stage == STAGES) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+            }
+            // Tail: on success wait until the last STAGES issues are released
+            // (no commit may land after exit).  After a failure the leader waits
+            // (bounded) on its full barriers, which count both CTAs' bytes; the
+            // peer cannot observe the leader's barriers and waits a fixed 2 ms,
+            // far beyond the latency of a tile load.
+            const int64_t n0 = issued > STAGES ? issued - STAGES : 0;
+            for (int64_t n = n0; n < issued && ok; ++n)
+                ok = wait_bounded(B.empty(static_cast<int>(n % STAGES)), static_cast<uint32_t>((n / STAGES) & 1),
+                                  abort_flag, p.timeout_ns, kWaitProducerEmpty);
+            if (!ok) {
+                if (leader) {
+                    for (int64_t n = n0; n < issued; ++n)
+                        wait_bounded(B.full(static_cast<int>(n % STAGES)), static_cast<uint32_t>((n / STAGES) & 1),
+                                     abort_flag, p.timeout_ns, kWaitDrain, /*honour_abort=*/false);
+                } else {
+                    const uint64_t t0 = ptx::global_timer_ns();
+                    while (ptx::global_timer_ns() - t0 < 2000000ull) {
+                    }
+                }
+            }
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------ MMA issuer (leader CTA)
+        if (lane == 0 && leader) {
+            int stage = 0;
+            uint32_t phase = 0;
+            int acc = 0;
+            uint32_t acc_phase = 0;
+            bool ok = true;
+            if (p.debug_never) ok = wait_bounded(B.never(), 0, abort_flag, p.timeout_ns, kWaitDebugNever);
+            for (int64_t it = first; ok && it < end; it += step) {
+                const WorkItem w = decode_item(it, p);
+                const int nch = num_chunks(w, p.kc);
+                for (int ck = 0; ok && ck < nch; ++ck) {
+                    const int kb = chunk_begin(w, ck, nch), ke = chunk_begin(w, ck + 1, nch);
+                    if (!wait_bounded(B.acc_empty(acc), acc_phase ^ 1u, abort_flag, p.timeout_ns, kWaitMmaAccEmpty)) {
+                        ok = false;
+                        break;
+                    }
+                    ptx::tc_fence_after();
+                    const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
+                    for (int kt = kb; kt < ke; ++kt) {
+                        if (!wait_bounded(B.full(stage), phase, abort_flag, p.timeout_ns, kWaitMmaFull)) {
+                            ok = false;
+                            break;
+                        }
+                        ptx::tc_fence_after();
+                        const uint32_t sa = ring + stage * S::kBytes;
+                        const uint32_t sb = sa + S::kABytes;
+#pragma unroll
+                        for (int kk = 0; kk < kBK / kUmmaK; ++kk) {
+                            // A half: K-major, 128-byte rows, 8-row atoms 1 KB apart; 32 B per K=16
+                            const uint64_t adesc = ptx::smem_desc_sw128(sa + kk * (kUmmaK * 2), 16, 1024);
+                            // B half: MN-major, 64-column boxes 8 KB apart; 2 KB per K=16
+                            const uint64_t bdesc =
+                                ptx::smem_desc_sw128(sb + kk * (kUmmaK * 128), kBBox * kBK * 2, 1024);
+                            ptx::tc_mma_f16_pair(d_tmem, adesc, bdesc, kIdesc, (kt > kb || kk > 0) ? 1u : 0u);
+                        }
+                        ptx::tc_commit_pair_multicast(B.empty(stage), kBothCtas);
+                        if (++stage == STAGES) {
+                            stage = 0;
+                            phase ^= 1u;
+                        }
+                    }
+                    if (!ok) break;
+                    ptx::tc_commit_pair_multicast(B.acc_full(acc), kBothCtas);
+                    if (++acc == 2) {
+                        acc = 0;
+                        acc_phase ^= 1u;
+                    }
+                }
+            }
+            if (!ok) {
+                ptx::tc_commit_pair(B.drain());
+                wait_bounded(B.drain(), 0, abort_flag, p.timeout_ns, kWaitDrain, /*honour_abort=*/false);
+            }
+        }
+    } else {
+        run_epilogue<BN, OutT, true>(p, B, tmem_base, abort_flag, first, end, step, kPairBM,
+                                     static_cast<int>(rank) * 128, warp, lane);
+    }
+
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::cluster_sync();  // no CTA leaves while its peer may still signal it
+    ptx::tc_fence_after();
+    if (warp == 1) ptx::tmem_dealloc_pair(tmem_base, kTmemCols);
+}
+
+}  // namespace sfc

@@ -61,8 +61,11 @@ SHAPES = [
 ]
 
 
+TILES = [128, 256, "pair128", "pair256"]
+
+
 @pytest.mark.parametrize("M,N,K", SHAPES)
-@pytest.mark.parametrize("tile", [128, 256])
+@pytest.mark.parametrize("tile", TILES)
 def test_shapes_fp32_and_bf16(sfc, oracle, M, N, K, tile):
     lda, ldb = synth.pad8(K), synth.pad8(N)
     A, B = synth.gemm_inputs(M, N, K, "uniform", seed=M + N + K, lda=lda, ldb=ldb)
@@ -85,7 +88,7 @@ def test_integer_inputs_bit_exact_every_variant(sfc, oracle):
     for c in (1, 2, 4, 8):
         for order in ("sfc", "raster"):
             for assign in ("segment", "wave"):
-                for tile in (128, 256):
+                for tile in TILES:
                     C = sfc.gemm(Ad, Bd, ca_c=c, order=order, assign=assign, tile=tile)
                     assert np.array_equal(C.cpu().numpy().astype(np.float64), ref), (c, order, assign, tile)
                     Cb = sfc.gemm(Ad, Bd, ca_c=c, order=order, assign=assign, tile=tile,
@@ -101,19 +104,30 @@ def test_order_and_assignment_do_not_change_bits(sfc):
     A, B = synth.gemm_inputs(1000, 1200, 2500, "uniform", seed=5, lda=synth.pad8(2500))
     Ad, Bd = to_dev(A, B)
     for c in (1, 3):
-        outs = [sfc.gemm(Ad, Bd, ca_c=c, order=o, assign=a, tile=256)
-                for o in ("sfc", "raster") for a in ("segment", "wave")]
-        for other in outs[1:]:
-            assert torch.equal(outs[0], other)
-        again = sfc.gemm(Ad, Bd, ca_c=c, order="sfc", assign="segment", tile=256)
-        assert torch.equal(outs[0], again)                     # repeatable
+        for tile in TILES:
+            outs = [sfc.gemm(Ad, Bd, ca_c=c, order=o, assign=a, tile=tile)
+                    for o in ("sfc", "raster") for a in ("segment", "wave")]
+            for other in outs[1:]:
+                assert torch.equal(outs[0], other)
+            again = sfc.gemm(Ad, Bd, ca_c=c, order="sfc", assign="segment", tile=tile)
+            assert torch.equal(outs[0], again)                 # repeatable
 
 
 def test_k_layers_agree_within_tolerance(sfc, oracle):
     A, B = synth.gemm_inputs(256, 256, 8192, "uniform", seed=9)
     ref = oracle.gemm_f64(A, B)
     for c in (1, 2, 4, 8, 128):
-        check_fp32(run(sfc, A, B, ca_c=c), ref, 8192)
+        for tile in TILES:
+            check_fp32(run(sfc, A, B, ca_c=c, tile=tile), ref, 8192)
+
+
+@pytest.mark.parametrize("tile", TILES)
+def test_long_k_chains_stay_accurate(sfc, oracle, tile):
+    # K = 65536 in one layer: 16 accumulation chains of 4096 per tile, promoted
+    # with round-to-nearest fp32 adds; the fp32 tolerance must hold at c = 1.
+    A, B = synth.gemm_inputs(256, 384, 65536, "uniform", seed=12)
+    ref = oracle.gemm_f64(A, B)
+    check_fp32(run(sfc, A, B, ca_c=1, tile=tile), ref, 65536)
 
 
 def test_unaligned_ldc_uses_scalar_stores(sfc, oracle):
@@ -122,10 +136,10 @@ def test_unaligned_ldc_uses_scalar_stores(sfc, oracle):
     ref = oracle.gemm_f64(A, B.contiguous())
     Ad, Bd = to_dev(A, B)
     for dt in (torch.float32, torch.bfloat16):
-        for c in (1, 2):
+        for c, tile in ((1, 128), (2, 256), (1, "pair128"), (2, "pair256")):
             big = torch.full((M, N + 1), float("nan"), dtype=dt, device="cuda")
             C = big[:, :N]                                     # ldc = N + 1: not 16-byte rows
-            sfc.gemm(Ad, Bd, C, ca_c=c)
+            sfc.gemm(Ad, Bd, C, ca_c=c, tile=tile)
             torch.cuda.synchronize()
             got = C.float().cpu().numpy().astype(np.float64)
             if dt == torch.float32:
