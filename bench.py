@@ -92,6 +92,8 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--no-cublas", action="store_true",
+                    help="skip the comparison with torch.matmul (cuBLAS) in the same power window")
     return ap.parse_args()
 
 
@@ -344,6 +346,15 @@ def run_ours(args, rank, local, world):
                 "unit": "TFLOP/s", "frac": round(achieved / peaks["bf16_tflops"], 4), "traffic": traffic,
                 "kernel": "sfc_gemm_kernel", "peak_source": peaks["source"] + " dense bf16 (burst)",
                 "frac_of_sustained_peak": round(achieved / peaks["bf16_tflops_sustained"], 4)}
+    # burst peak for a short timed region, sustained (power-capped) peak for a long one
+    sustained = elapsed_ms > 500.0
+    peak = peaks["bf16_tflops_sustained"] if sustained else peaks["bf16_tflops"]
+    roofline["peak"] = peak
+    roofline["frac"] = round(achieved / peak, 4)
+    roofline["peak_source"] = "%s dense bf16 %s (timed region %.0f ms)" % (
+        peaks["source"], "sustained" if sustained else "burst", elapsed_ms)
+    roofline["frac_of_burst_peak"] = round(achieved / peaks["bf16_tflops"], 4)
+    del roofline["frac_of_sustained_peak"]
     launches = args.steps * sum(1 if m["c"] == 1 else 2 for m in mats)
     desc = WORKLOADS[args.workload]["desc"] if not args.sizes else "square sweep sizes %s" % args.sizes
     result = {
@@ -362,11 +373,50 @@ def run_ours(args, rank, local, world):
     }
     if clock_info is not None:
         result["clocks"] = clock_info
+    if not args.no_cublas and world == 1:
+        result["cublas_same_window"] = run_cublas_compare(args, mats, stream, call)
     if not args.no_e2e:
         result["e2e"] = run_e2e(args, mats, stream, world)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         result["cpu_baseline"] = run_cpu_baseline(mats)
     return result
+
+
+def run_cublas_compare(args, mats, stream, call):
+    """Comparison only: torch.matmul (cuBLAS) on the same shapes, alternating
+    step by step with this library so both see the same clocks and power."""
+    import torch
+
+    def cublas(m):
+        if m["C"].dtype == torch.bfloat16:
+            torch.matmul(m["Ad"], m["Bd"], out=m["C"])
+        else:
+            m["C"].copy_(torch.matmul(m["Ad"], m["Bd"]))
+
+    steps = max(3, min(args.steps, 50))
+    ours = cub = 0.0
+    for _ in range(2):
+        for m in mats:
+            cublas(m)
+    for k in range(steps):
+        for which in (0, 1):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for m in mats:
+                if which == 0:
+                    call(m, m["c"])
+                else:
+                    cublas(m)
+            e1.record(stream)
+            torch.cuda.synchronize()
+            if which == 0:
+                ours += e0.elapsed_time(e1)
+            else:
+                cub += e0.elapsed_time(e1)
+    flops = sum(2.0 * m["s"]["M"] * m["s"]["N"] * m["s"]["K"] for m in mats) * steps
+    return {"cublas_tflops": round(flops / (cub * 1e-3) / 1e12, 1),
+            "ours_tflops": round(flops / (ours * 1e-3) / 1e12, 1), "steps": steps,
+            "note": "alternating steps, same stream; cuBLAS output is bf16 (fp32 rows: bf16 GEMM then cast)"}
 
 
 def run_e2e(args, mats, stream, world):

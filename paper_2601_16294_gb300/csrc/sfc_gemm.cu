@@ -98,6 +98,7 @@ struct DeviceInfo {
     int status = SFC_ERR_UNSUPPORTED;
     int num_sms = 0;
     int chunk_slabs = kDefaultChunkSlabs;
+    int serpentine = 0;
     int workers[kNumVariants] = {0, 0, 0, 0};  // co-resident workers (blocks or pairs) per variant
 };
 DeviceInfo g_devices[kMaxDevices];
@@ -139,6 +140,7 @@ int device_setup(DeviceInfo** info) {
             const int v = std::atoi(env);
             d.chunk_slabs = v > 0 ? v : (1 << 30);
         }
+        if (const char* env = std::getenv("SFC_GEMM_SERPENTINE")) d.serpentine = std::atoi(env) != 0;
         e = set_attrs<float>();
         if (e == cudaSuccess) e = set_attrs<__nv_bfloat16>();
         if (e != cudaSuccess) { d.status = cuda_fail(e); return; }
@@ -298,6 +300,7 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     p.Kt = static_cast<int>(ceil_div(K, kBK));
     p.ca_c = ca_c;
     p.kc = dev->chunk_slabs;
+    p.serpentine = dev->serpentine;
     p.num_items = static_cast<int64_t>(p.Mt) * p.Nt * ca_c;
     p.order = order;
     p.assign = (assign == SFC_ASSIGN_SEGMENT) ? 0 : 1;

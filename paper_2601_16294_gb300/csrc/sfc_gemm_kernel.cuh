@@ -76,13 +76,18 @@ struct GemmParams {
     int order;             // 0 = generalized Hilbert, 1 = raster
     int assign;            // 0 = contiguous segments, 1 = strided waves
     int vec_store;         // 1 if 16-byte vector stores are aligned
+    int serpentine;        // 1: alternate the K direction between a worker's consecutive items
     int debug_never;       // test hook: MMA warp waits on a barrier nobody arrives at
     uint64_t timeout_ns;   // bound for every mbarrier wait
 };
 
 struct WorkItem {
     int tm, tn, k0, k1, layer;
+    int rev;  // 1: walk this item's K slabs from k1-1 down to k0
 };
+
+// Slab index of the q-th slab this item processes.
+__device__ __forceinline__ int slab_at(const WorkItem& w, int q) { return w.rev ? (w.k1 - 1 - q) : (w.k0 + q); }
 
 __device__ __forceinline__ WorkItem decode_item(int64_t i, const GemmParams& p) {
     const int64_t grid = static_cast<int64_t>(p.Mt) * p.Nt;
@@ -95,6 +100,16 @@ __device__ __forceinline__ WorkItem decode_item(int64_t i, const GemmParams& p) 
     w.layer = layer;
     w.k0 = static_cast<int>((static_cast<int64_t>(layer) * p.Kt) / p.ca_c);
     w.k1 = static_cast<int>((static_cast<int64_t>(layer + 1) * p.Kt) / p.ca_c);
+    w.rev = 0;
+    return w;
+}
+
+// The j-th item of a worker's sequence (it = first + j * step).  With
+// serpentine K order, odd j walk K backwards so that a worker starts each item
+// on the K slabs its previous, neighbouring tile touched last.
+__device__ __forceinline__ WorkItem item_at(int64_t it, int64_t first, int64_t step, const GemmParams& p) {
+    WorkItem w = decode_item(it, p);
+    w.rev = p.serpentine ? static_cast<int>(((it - first) / step) & 1) : 0;
     return w;
 }
 
@@ -103,8 +118,9 @@ __device__ __forceinline__ int num_chunks(const WorkItem& w, int kc) {
     const int len = w.k1 - w.k0;
     return (len + kc - 1) / kc;
 }
+// Position (0-based, in processing order) where chunk j of n starts.
 __device__ __forceinline__ int chunk_begin(const WorkItem& w, int j, int n) {
-    return w.k0 + static_cast<int>((static_cast<int64_t>(j) * (w.k1 - w.k0)) / n);
+    return static_cast<int>((static_cast<int64_t>(j) * (w.k1 - w.k0)) / n);
 }
 
 // Items of worker `worker` out of `workers`: [first, end) with stride `step`.
@@ -213,7 +229,7 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
     const uint32_t acce_target = PAIR ? ptx::map_to_cta(B.acc_empty(0), 0) : B.acc_empty(0);
     float run[kEpiCols];
     for (int64_t it = first; it < end; it += step) {
-        const WorkItem w = decode_item(it, p);
+        const WorkItem w = item_at(it, first, step, p);
         const int nch = num_chunks(w, p.kc);
         bool ok = true;
         for (int ck = 0; ck < nch; ++ck) {
@@ -331,8 +347,9 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
             int64_t issued = 0;
             bool ok = true;
             for (int64_t it = first; ok && it < end; it += step) {
-                const WorkItem w = decode_item(it, p);
-                for (int kt = w.k0; kt < w.k1; ++kt) {
+                const WorkItem w = item_at(it, first, step, p);
+                for (int q = 0; q < w.k1 - w.k0; ++q) {
+                    const int kt = slab_at(w, q);
                     if (!wait_bounded(B.empty(stage), phase ^ 1u, abort_flag, p.timeout_ns, kWaitProducerEmpty)) {
                         ok = false;
                         break;
@@ -374,7 +391,7 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
             bool ok = true;
             if (p.debug_never) ok = wait_bounded(B.never(), 0, abort_flag, p.timeout_ns, kWaitDebugNever);
             for (int64_t it = first; ok && it < end; it += step) {
-                const WorkItem w = decode_item(it, p);
+                const WorkItem w = item_at(it, first, step, p);
                 const int nch = num_chunks(w, p.kc);
                 for (int ck = 0; ok && ck < nch; ++ck) {
                     const int kb = chunk_begin(w, ck, nch), ke = chunk_begin(w, ck + 1, nch);
@@ -384,7 +401,7 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
                     }
                     ptx::tc_fence_after();
                     const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
-                    for (int kt = kb; kt < ke; ++kt) {
+                    for (int q = kb; q < ke; ++q) {
                         if (!wait_bounded(B.full(stage), phase, abort_flag, p.timeout_ns, kWaitMmaFull)) {
                             ok = false;
                             break;
@@ -399,7 +416,7 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
                             // B: MN-major, 64-column boxes 8 KB apart, 8-row atoms 1 KB apart; 2 KB per K=16
                             const uint64_t bdesc =
                                 ptx::smem_desc_sw128(sb + kk * (kUmmaK * 128), kBBox * kBK * 2, 1024);
-                            ptx::tc_mma_f16(d_tmem, adesc, bdesc, kIdesc, (kt > kb || kk > 0) ? 1u : 0u);
+                            ptx::tc_mma_f16(d_tmem, adesc, bdesc, kIdesc, (q > kb || kk > 0) ? 1u : 0u);
                         }
                         ptx::tc_commit(B.empty(stage));  // frees the stage once these MMAs finish
                         if (++stage == STAGES) {

@@ -104,10 +104,11 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
             int64_t issued = 0;
             bool ok = true;
             for (int64_t it = first; ok && it < end; it += step) {
-                const WorkItem w = decode_item(it, p);
+                const WorkItem w = item_at(it, first, step, p);
                 const int32_t a_row = w.tm * kPairBM + static_cast<int32_t>(rank) * 128;
                 const int32_t b_col = w.tn * BN + static_cast<int32_t>(rank) * kHalfN;
-                for (int kt = w.k0; kt < w.k1; ++kt) {
+                for (int q = 0; q < w.k1 - w.k0; ++q) {
+                    const int kt = slab_at(w, q);
                     if (!wait_bounded(B.empty(stage), phase ^ 1u, abort_flag, p.timeout_ns, kWaitProducerEmpty)) {
                         ok = false;
                         break;
@@ -159,7 +160,7 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
             bool ok = true;
             if (p.debug_never) ok = wait_bounded(B.never(), 0, abort_flag, p.timeout_ns, kWaitDebugNever);
             for (int64_t it = first; ok && it < end; it += step) {
-                const WorkItem w = decode_item(it, p);
+                const WorkItem w = item_at(it, first, step, p);
                 const int nch = num_chunks(w, p.kc);
                 for (int ck = 0; ok && ck < nch; ++ck) {
                     const int kb = chunk_begin(w, ck, nch), ke = chunk_begin(w, ck + 1, nch);
@@ -169,7 +170,7 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
                     }
                     ptx::tc_fence_after();
                     const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * BN);
-                    for (int kt = kb; kt < ke; ++kt) {
+                    for (int q = kb; q < ke; ++q) {
                         if (!wait_bounded(B.full(stage), phase, abort_flag, p.timeout_ns, kWaitMmaFull)) {
                             ok = false;
                             break;
@@ -184,7 +185,7 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
                             // B half: MN-major, 64-column boxes 8 KB apart; 2 KB per K=16
                             const uint64_t bdesc =
                                 ptx::smem_desc_sw128(sb + kk * (kUmmaK * 128), kBBox * kBK * 2, 1024);
-                            ptx::tc_mma_f16_pair(d_tmem, adesc, bdesc, kIdesc, (kt > kb || kk > 0) ? 1u : 0u);
+                            ptx::tc_mma_f16_pair(d_tmem, adesc, bdesc, kIdesc, (q > kb || kk > 0) ? 1u : 0u);
                         }
                         ptx::tc_commit_pair_multicast(B.empty(stage), kBothCtas);
                         if (++stage == STAGES) {
