@@ -394,28 +394,30 @@ def run_cublas_compare(args, mats, stream, call):
             m["C"].copy_(torch.matmul(m["Ad"], m["Bd"]))
 
     steps = max(3, min(args.steps, 50))
-    ours = cub = 0.0
+    t = [[0.0, 0.0] for _ in mats]
     for _ in range(2):
         for m in mats:
             cublas(m)
     for k in range(steps):
         for which in (0, 1):
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-            for m in mats:
+            ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in mats]
+            for i, m in enumerate(mats):
+                ev[i][0].record(stream)
                 if which == 0:
                     call(m, m["c"])
                 else:
                     cublas(m)
-            e1.record(stream)
+                ev[i][1].record(stream)
             torch.cuda.synchronize()
-            if which == 0:
-                ours += e0.elapsed_time(e1)
-            else:
-                cub += e0.elapsed_time(e1)
-    flops = sum(2.0 * m["s"]["M"] * m["s"]["N"] * m["s"]["K"] for m in mats) * steps
-    return {"cublas_tflops": round(flops / (cub * 1e-3) / 1e12, 1),
-            "ours_tflops": round(flops / (ours * 1e-3) / 1e12, 1), "steps": steps,
+            for i in range(len(mats)):
+                t[i][which] += ev[i][0].elapsed_time(ev[i][1])
+    fl = [2.0 * m["s"]["M"] * m["s"]["N"] * m["s"]["K"] * steps for m in mats]
+    ours, cub = sum(x[0] for x in t), sum(x[1] for x in t)
+    return {"cublas_tflops": round(sum(fl) / (cub * 1e-3) / 1e12, 1),
+            "ours_tflops": round(sum(fl) / (ours * 1e-3) / 1e12, 1), "steps": steps,
+            "per_shape": [{"M": m["s"]["M"], "N": m["s"]["N"], "K": m["s"]["K"],
+                           "ours": round(f / (x[0] * 1e-3) / 1e12, 1), "cublas": round(f / (x[1] * 1e-3) / 1e12, 1)}
+                          for m, f, x in zip(mats, fl, t)],
             "note": "alternating steps, same stream; cuBLAS output is bf16 (fp32 rows: bf16 GEMM then cast)"}
 
 

@@ -112,7 +112,7 @@ size_t sfc_gemm_workspace_size(int64_t M, int64_t N, int64_t K, int ca_c);
  * curve order, automatic assignment and tile width.
  *   A: bf16, M x K, row stride lda.   B: bf16, K x N, row stride ldb.
  *   C: fp32, M x N, row stride ldc.   Written, never read (beta = 0).
- *   ca_c: number of K layers, 1 <= ca_c <= ceil(K/64).  Layer l contracts K
+ *   ca_c: number of K layers, 1 <= ca_c <= min(ceil(K/64), 4096).  Layer l contracts K
  *         tiles [floor(l*Kt/ca_c), floor((l+1)*Kt/ca_c)) of the Kt = ceil(K/64)
  *         64-wide K tiles.  For ca_c > 1 the library takes its fp32 workspace
  *         from a stream-ordered pool (cudaMallocAsync / cudaFreeAsync on

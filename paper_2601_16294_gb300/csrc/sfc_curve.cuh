@@ -31,7 +31,9 @@ struct TileCoord {
 __host__ __device__ __forceinline__ int sgn_i(int v) { return (v > 0) - (v < 0); }
 __host__ __device__ __forceinline__ int abs_i(int v) { return v < 0 ? -v : v; }
 
-__host__ __device__ inline TileCoord curve_decode(int64_t s, int Mt, int Nt) {
+// s in [0, Mt*Nt), Mt*Nt < 2^31: every count below fits in 32 bits, which
+// keeps this single-thread dependent chain short on the GPU.
+__host__ __device__ inline TileCoord curve_decode(int s, int Mt, int Nt) {
     // current region: origin (x, y), major vector (ax, ay), minor vector (bx, by)
     int x = 0, y = 0, ax, ay, bx, by;
     bool major_is_x = Nt >= Mt;
@@ -41,13 +43,13 @@ __host__ __device__ inline TileCoord curve_decode(int64_t s, int Mt, int Nt) {
     if (major_is_x) { ax = Nt; ay = 0; bx = 0; by = Mt; }
     else            { ax = 0;  ay = Mt; bx = Nt; by = 0; }
 
-    int64_t r = s;  // rank of the wanted cell inside the current region
+    int r = s;  // rank of the wanted cell inside the current region
     for (;;) {
         const int w = abs_i(ax + ay), h = abs_i(bx + by);
         const int ux = sgn_i(ax), uy = sgn_i(ay);  // unit step along the major axis
         const int vx = sgn_i(bx), vy = sgn_i(by);  // unit step along the minor axis
-        if (h == 1) { x += static_cast<int>(r) * ux; y += static_cast<int>(r) * uy; break; }
-        if (w == 1) { x += static_cast<int>(r) * vx; y += static_cast<int>(r) * vy; break; }
+        if (h == 1) { x += r * ux; y += r * uy; break; }
+        if (w == 1) { x += r * vx; y += r * vy; break; }
 
         int hax = ax / 2, hay = ay / 2;  // first part of the major axis
         int hbx = bx / 2, hby = by / 2;  // first part of the minor axis
@@ -56,15 +58,15 @@ __host__ __device__ inline TileCoord curve_decode(int64_t s, int Mt, int Nt) {
         if (2 * w > 3 * h) {
             // two pieces along the major axis, first one even when possible
             if ((hw & 1) && w > 2) { hax += ux; hay += uy; ++hw; }
-            const int64_t first = static_cast<int64_t>(hw) * h;
+            const int first = hw * h;
             if (r < first) { ax = hax; ay = hay; }
             else { r -= first; x += hax; y += hay; ax -= hax; ay -= hay; }
             continue;
         }
 
         if ((hh & 1) && h > 2) { hbx += vx; hby += vy; ++hh; }
-        const int64_t corner = static_cast<int64_t>(hh) * hw;      // first corner block
-        const int64_t strip = static_cast<int64_t>(w) * (h - hh);  // strip across
+        const int corner = hh * hw;       // first corner block
+        const int strip = w * (h - hh);   // strip across
         if (r < corner) {
             // axes exchanged: major = first part of b, minor = first half of a
             const int nax = hbx, nay = hby;
@@ -85,8 +87,9 @@ __host__ __device__ inline TileCoord curve_decode(int64_t s, int Mt, int Nt) {
     return TileCoord{y, x};
 }
 
-__host__ __device__ __forceinline__ TileCoord raster_decode(int64_t s, int Nt) {
-    return TileCoord{static_cast<int>(s / Nt), static_cast<int>(s % Nt)};
+__host__ __device__ __forceinline__ TileCoord raster_decode(int s, int Nt) {
+    const int tm = s / Nt;
+    return TileCoord{tm, s - tm * Nt};
 }
 
 }  // namespace sfc

@@ -20,6 +20,7 @@ namespace sfc {
 namespace {
 
 constexpr int kMaxDevices = 64;
+constexpr int kMaxLayers = 4096;  // keeps the kernels' layer arithmetic in 32 bits
 constexpr uint64_t kDefaultTimeoutNs = 2000000000ull;  // 2 s per wait
 
 thread_local int t_last_cuda_error = 0;
@@ -43,21 +44,21 @@ constexpr int variant_bn(int v) { return (v == kSingle128 || v == kPair128) ? 12
 constexpr bool variant_pair(int v) { return v == kPair128 || v == kPair256; }
 
 template <int BN, int STAGES>
-constexpr int single_smem() { return RingLayout<(kBM + BN) * kBK * 2, STAGES>::kDynamicBytes; }
+constexpr int single_smem() { return RingLayout<(kBM + BN) * kBK * 2, STAGES, BN / 32>::kDynamicBytes; }
 template <int BN, int STAGES>
-constexpr int pair_smem() { return RingLayout<PairStage<BN>::kBytes, STAGES>::kDynamicBytes; }
+constexpr int pair_smem() { return RingLayout<PairStage<BN>::kBytes, STAGES, BN / 32>::kDynamicBytes; }
 
 template <typename OutT>
 struct Kernels {
-    static constexpr void (*single128)(CUtensorMap, CUtensorMap, GemmParams) =
+    static constexpr void (*single128)(CUtensorMap, CUtensorMap, CUtensorMap, GemmParams) =
         sfc_gemm_kernel<128, kStagesSingle128, OutT>;
-    static constexpr void (*single256)(CUtensorMap, CUtensorMap, GemmParams) =
+    static constexpr void (*single256)(CUtensorMap, CUtensorMap, CUtensorMap, GemmParams) =
         sfc_gemm_kernel<256, kStagesSingle256, OutT>;
-    static constexpr void (*pair128)(CUtensorMap, CUtensorMap, GemmParams) =
+    static constexpr void (*pair128)(CUtensorMap, CUtensorMap, CUtensorMap, GemmParams) =
         sfc_gemm_pair_kernel<128, kStagesPair128, OutT>;
-    static constexpr void (*pair256)(CUtensorMap, CUtensorMap, GemmParams) =
+    static constexpr void (*pair256)(CUtensorMap, CUtensorMap, CUtensorMap, GemmParams) =
         sfc_gemm_pair_kernel<256, kStagesPair256, OutT>;
-    static void (*get(int v))(CUtensorMap, CUtensorMap, GemmParams) {
+    static void (*get(int v))(CUtensorMap, CUtensorMap, CUtensorMap, GemmParams) {
         switch (v) {
             case kSingle128: return single128;
             case kSingle256: return single256;
@@ -201,6 +202,33 @@ int make_bf16_map(CUtensorMap* map, const void* ptr, int64_t rows, int64_t cols,
     return SFC_OK;
 }
 
+// Output map for the staged TMA-store epilogue: 32 x 32 element boxes, swizzled
+// to match the staging layout (64-byte rows for bf16, 128-byte rows for fp32).
+// layers > 1: a 3-D map (columns, rows, layer) over the workspace copies, so a
+// box at the M edge of one layer is clipped instead of spilling into the next.
+int make_out_map(CUtensorMap* map, const void* ptr, int64_t rows, int64_t cols, int64_t ld, int elem_bytes,
+                 int layers) {
+    PFN_cuTensorMapEncodeTiled_v12000 encode;
+    int rc = get_encoder(&encode);
+    if (rc != SFC_OK) return rc;
+    cuuint64_t dims[3] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows),
+                          static_cast<cuuint64_t>(layers)};
+    cuuint64_t strides[2] = {static_cast<cuuint64_t>(ld) * elem_bytes,
+                             static_cast<cuuint64_t>(ld) * elem_bytes * static_cast<cuuint64_t>(rows)};
+    cuuint32_t box[3] = {32, 32, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    const CUtensorMapDataType dt = elem_bytes == 4 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+    const CUtensorMapSwizzle sw = elem_bytes == 4 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
+    CUresult r = encode(map, dt, layers > 1 ? 3 : 2, const_cast<void*>(ptr), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+        t_last_cuda_error = static_cast<int>(r);
+        return SFC_ERR_CUDA;
+    }
+    return SFC_OK;
+}
+
 // ------------------------------------------------------------------ planning
 
 int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
@@ -252,7 +280,7 @@ int validate(int64_t M, int64_t N, int64_t K, const void* A, const void* B, cons
     if (M > (int64_t(1) << 31) - kBM || N > (int64_t(1) << 31) - 256 || K > (int64_t(1) << 31) - kBK)
         return SFC_ERR_INVALID_ARG;
     const int64_t Kt = ceil_div(K, kBK);
-    if (ca_c < 1 || ca_c > Kt) return SFC_ERR_INVALID_ARG;
+    if (ca_c < 1 || ca_c > Kt || ca_c > kMaxLayers) return SFC_ERR_INVALID_ARG;
     if (ceil_div(M, kBM) * ceil_div(N, 128) * ca_c > (int64_t(1) << 31) - 1) return SFC_ERR_INVALID_ARG;
     if (!aligned16(A) || !aligned16(B) || (lda % 8) != 0 || (ldb % 8) != 0) return SFC_ERR_UNALIGNED;
     if (lda >= (int64_t(1) << 39) || ldb >= (int64_t(1) << 39)) return SFC_ERR_INVALID_ARG;
@@ -262,11 +290,11 @@ int validate(int64_t M, int64_t N, int64_t K, const void* A, const void* B, cons
 int64_t ws_ld(int64_t N) { return (N + 3) / 4 * 4; }
 
 template <typename OutT>
-cudaError_t launch_gemm(int v, const CUtensorMap& ta, const CUtensorMap& tb, const GemmParams& p, int grid,
-                        cudaStream_t s) {
+cudaError_t launch_gemm(int v, const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc,
+                        const GemmParams& p, int grid, cudaStream_t s) {
     cudaLaunchAttribute attr;
     cudaLaunchConfig_t cfg = launch_config(v, grid, s, &attr);
-    cudaError_t e = cudaLaunchKernelEx(&cfg, Kernels<OutT>::get(v), ta, tb, p);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, Kernels<OutT>::get(v), ta, tb, tc, p);
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
@@ -299,6 +327,9 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     p.Nt = static_cast<int>(ceil_div(N, bn));
     p.Kt = static_cast<int>(ceil_div(K, kBK));
     p.ca_c = ca_c;
+    p.grid_tiles = p.Mt * p.Nt;
+    p.kq = p.Kt / ca_c;
+    p.kr = p.Kt % ca_c;
     p.kc = dev->chunk_slabs;
     p.serpentine = dev->serpentine;
     p.num_items = static_cast<int64_t>(p.Mt) * p.Nt * ca_c;
@@ -319,20 +350,24 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     }
 
     cudaError_t e;
+    CUtensorMap tc;
+    std::memset(&tc, 0, sizeof(tc));
     if (ca_c == 1) {
         p.out = C;
         p.ldo = ldc;
         p.layer_stride = 0;
-        const size_t esz = (c_dtype == SFC_F32) ? 4 : 2;
+        const int esz = (c_dtype == SFC_F32) ? 4 : 2;
         p.vec_store = aligned16(C) && ((ldc * esz) % 16 == 0);
-        e = (c_dtype == SFC_F32) ? launch_gemm<float>(v, ta, tb, p, grid, stream)
-                                 : launch_gemm<__nv_bfloat16>(v, ta, tb, p, grid, stream);
+        p.tma_store = p.vec_store && make_out_map(&tc, C, M, N, ldc, esz, 1) == SFC_OK;
+        e = (c_dtype == SFC_F32) ? launch_gemm<float>(v, ta, tb, tc, p, grid, stream)
+                                 : launch_gemm<__nv_bfloat16>(v, ta, tb, tc, p, grid, stream);
     } else {
         p.out = ws;
         p.ldo = ws_ld(N);
         p.layer_stride = M * p.ldo;
         p.vec_store = 1;
-        e = launch_gemm<float>(v, ta, tb, p, grid, stream);
+        p.tma_store = make_out_map(&tc, ws, M, N, p.ldo, 4, ca_c) == SFC_OK;
+        e = launch_gemm<float>(v, ta, tb, tc, p, grid, stream);
         if (e == cudaSuccess) {
             const int64_t work = M * ((N + 3) / 4);
             int64_t blocks = ceil_div(work, 256);
@@ -369,7 +404,7 @@ SFC_API int sfc_tile_order(int Mt, int Nt, int32_t* out_idx) {
     const int64_t n = static_cast<int64_t>(Mt) * Nt;
     if (n > INT32_MAX) return SFC_ERR_INVALID_ARG;
     for (int64_t s = 0; s < n; ++s) {
-        const TileCoord t = curve_decode(s, Mt, Nt);
+        const TileCoord t = curve_decode(static_cast<int>(s), Mt, Nt);
         out_idx[s] = t.tm * Nt + t.tn;
     }
     return SFC_OK;

@@ -68,6 +68,8 @@ struct GemmParams {
     int64_t M, N;
     int Mt, Nt, Kt;        // tile grid and number of 64-wide K slabs
     int ca_c;              // K layers
+    int grid_tiles;        // Mt * Nt
+    int kq, kr;            // Kt / ca_c and Kt % ca_c (layer l starts at l*kq + l*kr/ca_c)
     int kc;                // max slabs per tensor-memory accumulation chain
     int64_t num_items;     // Mt * Nt * ca_c
     void* out;             // C when ca_c == 1, else the fp32 workspace
@@ -76,6 +78,7 @@ struct GemmParams {
     int order;             // 0 = generalized Hilbert, 1 = raster
     int assign;            // 0 = contiguous segments, 1 = strided waves
     int vec_store;         // 1 if 16-byte vector stores are aligned
+    int tma_store;         // 1: stores go through smem staging and the output tensor map
     int serpentine;        // 1: alternate the K direction between a worker's consecutive items
     int debug_never;       // test hook: MMA warp waits on a barrier nobody arrives at
     uint64_t timeout_ns;   // bound for every mbarrier wait
@@ -89,17 +92,22 @@ struct WorkItem {
 // Slab index of the q-th slab this item processes.
 __device__ __forceinline__ int slab_at(const WorkItem& w, int q) { return w.rev ? (w.k1 - 1 - q) : (w.k0 + q); }
 
-__device__ __forceinline__ WorkItem decode_item(int64_t i, const GemmParams& p) {
-    const int64_t grid = static_cast<int64_t>(p.Mt) * p.Nt;
-    const int layer = static_cast<int>(i / grid);
-    const int64_t s = i - static_cast<int64_t>(layer) * grid;
+// First K slab of layer l: floor(l * Kt / c) = l * (Kt / c) + floor(l * (Kt % c) / c),
+// in 32-bit arithmetic (c <= 4096 keeps l * (Kt % c) below 2^24).
+__device__ __forceinline__ int layer_k0(int l, const GemmParams& p) { return l * p.kq + (l * p.kr) / p.ca_c; }
+
+// Item index i < 2^31 (validated on the host) -> tile, K layer and K range.
+__device__ __forceinline__ WorkItem decode_item(int64_t i64, const GemmParams& p) {
+    const int i = static_cast<int>(i64);
+    const int layer = (p.ca_c == 1) ? 0 : i / p.grid_tiles;
+    const int s = i - layer * p.grid_tiles;
     const TileCoord t = (p.order == 0) ? curve_decode(s, p.Mt, p.Nt) : raster_decode(s, p.Nt);
     WorkItem w;
     w.tm = t.tm;
     w.tn = t.tn;
     w.layer = layer;
-    w.k0 = static_cast<int>((static_cast<int64_t>(layer) * p.Kt) / p.ca_c);
-    w.k1 = static_cast<int>((static_cast<int64_t>(layer + 1) * p.Kt) / p.ca_c);
+    w.k0 = layer_k0(layer, p);
+    w.k1 = layer_k0(layer + 1, p);
     w.rev = 0;
     return w;
 }
@@ -202,15 +210,50 @@ struct Barriers {
     __device__ __forceinline__ uint32_t never() const { return bars + 8u * (2 * stages + 5); }
 };
 
-template <int STAGE_BYTES, int STAGES>
+// Epilogue staging: one 4 KB buffer per epilogue warp (32 rows x 32 columns
+// of fp32, or of bf16 in its first half), swizzled like the output tensor map.
+constexpr int kStageBufBytes = 4096;
+
+template <int STAGE_BYTES, int STAGES, int EPI_WARPS>
 struct RingLayout {
     static constexpr int kRingBytes = STAGE_BYTES * STAGES;
+    static constexpr int kStagingOffset = kRingBytes;
+    static constexpr int kStagingBytes = EPI_WARPS * kStageBufBytes;
     static constexpr int kNumBars = 2 * STAGES + 6;
-    static constexpr int kBarOffset = kRingBytes;
+    static constexpr int kBarOffset = kRingBytes + kStagingBytes;
     static constexpr int kMiscOffset = kBarOffset + kNumBars * 8;
     static constexpr int kBytes = kMiscOffset + 16;
     static constexpr int kDynamicBytes = kBytes + 1024;  // slack to align the ring to 1024 B
 };
+
+// Write 32 columns of this lane's row into the warp's staging buffer (32 rows
+// x 32 columns), in the layout of a 64-byte (bf16) or 128-byte (fp32)
+// swizzled TMA box: 16-byte unit j of row r sits at unit j ^ (swizzle of r).
+// Distinct rows of 8 consecutive lanes land in distinct bank groups.
+template <typename OutT>
+__device__ __forceinline__ void stage_row(uint8_t* buf, int lane, const float* v) {
+    if constexpr (sizeof(OutT) == 4) {
+        uint8_t* row = buf + lane * 128;
+        const int sw = lane & 7;
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+            *reinterpret_cast<float4*>(row + ((j ^ sw) * 16)) =
+                make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+    } else {
+        uint8_t* row = buf + lane * 64;
+        const int sw = (lane >> 1) & 3;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            uint32_t w[4];
+#pragma unroll
+            for (int h = 0; h < 4; ++h) {
+                __nv_bfloat162 b = __floats2bfloat162_rn(v[8 * j + 2 * h], v[8 * j + 2 * h + 1]);
+                w[h] = *reinterpret_cast<uint32_t*>(&b);
+            }
+            *reinterpret_cast<uint4*>(row + ((j ^ sw) * 16)) = make_uint4(w[0], w[1], w[2], w[3]);
+        }
+    }
+}
 
 // -------------------------------------------------------------------------
 // Epilogue of one block: drain chunks, promote, store.  `rows_base` is the
@@ -219,7 +262,8 @@ struct RingLayout {
 template <int BN, typename OutT, bool PAIR>
 __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers& B, uint32_t tmem_base,
                                              volatile int* abort_flag, int64_t first, int64_t end,
-                                             int64_t step, int tile_rows, int row_offset, int warp, int lane) {
+                                             int64_t step, int tile_rows, int row_offset, int warp, int lane,
+                                             const CUtensorMap* tmap_c, uint8_t* staging) {
     const int ew = warp - 2;                 // epilogue warp index
     const int quarter = warp & 3;            // TMEM lane quarter this warp may access
     const int half = ew / 4;                 // which 128-column half of the tile
@@ -270,15 +314,41 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
             }
         }
         if (!ok) break;
-        const int64_t row = static_cast<int64_t>(w.tm) * tile_rows + row_offset + quarter * 32 + lane;
-        if (row < p.M) {
-            OutT* row_ptr = out + static_cast<int64_t>(w.layer) * p.layer_stride + row * p.ldo;
-            const int64_t col_base = static_cast<int64_t>(w.tn) * BN + half * kEpiCols;
+        const int64_t warp_row = static_cast<int64_t>(w.tm) * tile_rows + row_offset + quarter * 32;
+        const int64_t col_base = static_cast<int64_t>(w.tn) * BN + half * kEpiCols;
+        if (p.tma_store) {
+            // stage 32 x 32 blocks and let the TMA write them (edges clipped by the map)
+            uint8_t* buf = staging + ew * kStageBufBytes;
+            const uint32_t buf_addr = ptx::smem_addr(buf);
 #pragma unroll
-            for (int g = 0; g < kEpiCols / 32; ++g)
-                store_chunk<OutT>(row_ptr, col_base + g * 32, p.N, run + g * 32, p.vec_store != 0);
+            for (int g = 0; g < kEpiCols / 32; ++g) {
+                if (col_base + g * 32 >= p.N) break;  // warp-uniform
+                stage_row<OutT>(buf, lane, run + g * 32);
+                ptx::fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) {
+                    if (p.ca_c > 1)
+                        ptx::tma_store_3d(tmap_c, buf_addr, static_cast<int32_t>(col_base + g * 32),
+                                          static_cast<int32_t>(warp_row), w.layer);
+                    else
+                        ptx::tma_store_2d(tmap_c, buf_addr, static_cast<int32_t>(col_base + g * 32),
+                                          static_cast<int32_t>(warp_row));
+                    ptx::bulk_commit();
+                    ptx::bulk_wait_read_all();  // buffer free again
+                }
+                __syncwarp();
+            }
+        } else {
+            const int64_t row = warp_row + lane;
+            if (row < p.M) {
+                OutT* row_ptr = out + static_cast<int64_t>(w.layer) * p.layer_stride + row * p.ldo;
+#pragma unroll
+                for (int g = 0; g < kEpiCols / 32; ++g)
+                    store_chunk<OutT>(row_ptr, col_base + g * 32, p.N, run + g * 32, p.vec_store != 0);
+            }
         }
     }
+    if (p.tma_store && lane == 0) ptx::bulk_wait_all();
 }
 
 // -------------------------------------------------------------------------
@@ -287,15 +357,15 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
 template <int BN, int STAGES, typename OutT>
 __global__ void __launch_bounds__(block_threads(BN), 1)
 sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_b,
-                const GemmParams p) {
+                const __grid_constant__ CUtensorMap tmap_c, const GemmParams p) {
     static_assert(BN == 128 || BN == 256, "tiles are 128 x 128 or 128 x 256");
     constexpr int kABytes = kBM * kBK * 2;
     constexpr int kBBytes = BN * kBK * 2;
     constexpr int kStageBytes = kABytes + kBBytes;
-    using L = RingLayout<kStageBytes, STAGES>;
+    constexpr int kEpiWarps = BN / 32;
+    using L = RingLayout<kStageBytes, STAGES, kEpiWarps>;
     constexpr uint32_t kIdesc = ptx::idesc_bf16_f32(kBM, BN, /*A K-major*/ 0, /*B MN-major*/ 1);
     constexpr uint32_t kTmemCols = 2 * BN;
-    constexpr int kEpiWarps = BN / 32;
 
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = ptx::smem_addr(smem_raw);
@@ -326,6 +396,7 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
     if (warp == 0 && lane == 0) {
         ptx::tma_prefetch_desc(&tmap_a);
         ptx::tma_prefetch_desc(&tmap_b);
+        if (p.tma_store) ptx::tma_prefetch_desc(&tmap_c);
     }
     if (warp == 1) {
         ptx::tmem_alloc(ptx::smem_addr(tmem_slot), kTmemCols);
@@ -439,7 +510,8 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
             }
         }
     } else {
-        run_epilogue<BN, OutT, false>(p, B, tmem_base, abort_flag, first, end, step, kBM, 0, warp, lane);
+        run_epilogue<BN, OutT, false>(p, B, tmem_base, abort_flag, first, end, step, kBM, 0, warp, lane, &tmap_c,
+                                      smem + L::kStagingOffset);
     }
 
     ptx::tc_fence_before();
@@ -493,7 +565,7 @@ __global__ void tile_order_kernel(int Mt, int Nt, int32_t* __restrict__ out) {
     const int64_t n = static_cast<int64_t>(Mt) * Nt;
     for (int64_t s = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; s < n;
          s += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-        const TileCoord t = curve_decode(s, Mt, Nt);
+        const TileCoord t = curve_decode(static_cast<int>(s), Mt, Nt);
         out[s] = t.tm * Nt + t.tn;
     }
 }

@@ -41,14 +41,14 @@ struct PairStage {
 template <int BN, int STAGES, typename OutT>
 __global__ void __launch_bounds__(block_threads(BN), 1)
 sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_b,
-                     const GemmParams p) {
+                     const __grid_constant__ CUtensorMap tmap_c, const GemmParams p) {
     static_assert(BN == 128 || BN == 256, "pair tiles are 256 x 128 or 256 x 256");
     using S = PairStage<BN>;
-    using L = RingLayout<S::kBytes, STAGES>;
+    constexpr int kEpiWarps = BN / 32;
+    using L = RingLayout<S::kBytes, STAGES, kEpiWarps>;
     constexpr int kHalfN = S::kHalfN;
     constexpr uint32_t kIdesc = ptx::idesc_bf16_f32(kPairBM, BN, /*A K-major*/ 0, /*B MN-major*/ 1);
     constexpr uint32_t kTmemCols = 2 * BN;
-    constexpr int kEpiWarps = BN / 32;
     constexpr uint16_t kBothCtas = 0x3;
 
     extern __shared__ uint8_t smem_raw[];
@@ -82,6 +82,7 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
     if (warp == 0 && lane == 0) {
         ptx::tma_prefetch_desc(&tmap_a);
         ptx::tma_prefetch_desc(&tmap_b);
+        if (p.tma_store) ptx::tma_prefetch_desc(&tmap_c);
     }
     if (warp == 1) {
         ptx::tmem_alloc_pair(ptx::smem_addr(tmem_slot), kTmemCols);
@@ -208,7 +209,7 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
         }
     } else {
         run_epilogue<BN, OutT, true>(p, B, tmem_base, abort_flag, first, end, step, kPairBM,
-                                     static_cast<int>(rank) * 128, warp, lane);
+                                     static_cast<int>(rank) * 128, warp, lane, &tmap_c, smem + L::kStagingOffset);
     }
 
     ptx::tc_fence_before();
