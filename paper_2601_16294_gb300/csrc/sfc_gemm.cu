@@ -75,21 +75,28 @@ constexpr int variant_smem(int v) {
                              : pair_smem<256, kStagesPair256>();
 }
 
-cudaLaunchConfig_t launch_config(int v, int grid, cudaStream_t s, cudaLaunchAttribute* attr) {
+// attr must hold two entries.  With `pdl` the kernel may begin launching
+// while the previous kernel in the stream finishes (programmatic dependent
+// launch); the kernels wait for it before touching global memory.
+cudaLaunchConfig_t launch_config(int v, int grid, cudaStream_t s, cudaLaunchAttribute* attr, bool pdl) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid, 1, 1);
     cfg.blockDim = dim3(block_threads(variant_bn(v)), 1, 1);
     cfg.dynamicSmemBytes = variant_smem(v);
     cfg.stream = s;
-    cfg.attrs = nullptr;
+    cfg.attrs = attr;
     cfg.numAttrs = 0;
     if (variant_pair(v)) {
-        attr->id = cudaLaunchAttributeClusterDimension;
-        attr->val.clusterDim.x = 2;
-        attr->val.clusterDim.y = 1;
-        attr->val.clusterDim.z = 1;
-        cfg.attrs = attr;
-        cfg.numAttrs = 1;
+        attr[cfg.numAttrs].id = cudaLaunchAttributeClusterDimension;
+        attr[cfg.numAttrs].val.clusterDim.x = 2;
+        attr[cfg.numAttrs].val.clusterDim.y = 1;
+        attr[cfg.numAttrs].val.clusterDim.z = 1;
+        ++cfg.numAttrs;
+    }
+    if (pdl) {
+        attr[cfg.numAttrs].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[cfg.numAttrs].val.programmaticStreamSerializationAllowed = 1;
+        ++cfg.numAttrs;
     }
     return cfg;
 }
@@ -150,8 +157,8 @@ int device_setup(DeviceInfo** info) {
                 d.workers[v] = d.num_sms;
                 continue;
             }
-            cudaLaunchAttribute attr;
-            cudaLaunchConfig_t cfg = launch_config(v, d.num_sms, nullptr, &attr);
+            cudaLaunchAttribute attr[2];
+            cudaLaunchConfig_t cfg = launch_config(v, d.num_sms, nullptr, attr, false);
             int clusters = 0;
             e = cudaOccupancyMaxActiveClusters(&clusters, Kernels<float>::get(v), &cfg);
             if (e != cudaSuccess) { d.status = cuda_fail(e); return; }
@@ -292,8 +299,8 @@ int64_t ws_ld(int64_t N) { return (N + 3) / 4 * 4; }
 template <typename OutT>
 cudaError_t launch_gemm(int v, const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc,
                         const GemmParams& p, int grid, cudaStream_t s) {
-    cudaLaunchAttribute attr;
-    cudaLaunchConfig_t cfg = launch_config(v, grid, s, &attr);
+    cudaLaunchAttribute attr[2];
+    cudaLaunchConfig_t cfg = launch_config(v, grid, s, attr, true);
     cudaError_t e = cudaLaunchKernelEx(&cfg, Kernels<OutT>::get(v), ta, tb, tc, p);
     return e != cudaSuccess ? e : cudaGetLastError();
 }
@@ -375,15 +382,23 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
             if (blocks > cap) blocks = cap;
             const int vec = (c_dtype == SFC_F32) ? (aligned16(C) && (ldc % 4) == 0)
                                                  : (((reinterpret_cast<uintptr_t>(C) & 7u) == 0) && (ldc % 4) == 0);
+            cudaLaunchConfig_t cfg = {};
+            cudaLaunchAttribute attr;
+            attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+            attr.val.programmaticStreamSerializationAllowed = 1;
+            cfg.gridDim = dim3(static_cast<unsigned>(blocks), 1, 1);
+            cfg.blockDim = dim3(256, 1, 1);
+            cfg.stream = stream;
+            cfg.attrs = &attr;
+            cfg.numAttrs = 1;
+            const float* wsf = static_cast<const float*>(ws);
             if (c_dtype == SFC_F32)
-                ca_reduce_kernel<float><<<static_cast<int>(blocks), 256, 0, stream>>>(
-                    static_cast<const float*>(ws), p.ldo, p.layer_stride, ca_c, M, N, static_cast<float*>(C),
-                    ldc, vec);
+                e = cudaLaunchKernelEx(&cfg, ca_reduce_kernel<float>, wsf, p.ldo, p.layer_stride, ca_c, M, N,
+                                       static_cast<float*>(C), ldc, vec);
             else
-                ca_reduce_kernel<__nv_bfloat16><<<static_cast<int>(blocks), 256, 0, stream>>>(
-                    static_cast<const float*>(ws), p.ldo, p.layer_stride, ca_c, M, N,
-                    static_cast<__nv_bfloat16*>(C), ldc, vec);
-            e = cudaGetLastError();
+                e = cudaLaunchKernelEx(&cfg, ca_reduce_kernel<__nv_bfloat16>, wsf, p.ldo, p.layer_stride, ca_c, M,
+                                       N, static_cast<__nv_bfloat16*>(C), ldc, vec);
+            if (e == cudaSuccess) e = cudaGetLastError();
         }
     }
     if (pooled) {

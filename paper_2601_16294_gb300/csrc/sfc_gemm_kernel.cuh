@@ -289,16 +289,16 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
             const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
                                    static_cast<uint32_t>(acc * BN + half * kEpiCols);
 #pragma unroll
-            for (int g = 0; g < kEpiCols / 32; ++g) {
-                uint32_t r[32];
-                ptx::tmem_ld_32x32b_x32(taddr + g * 32, r);
+            for (int g = 0; g < kEpiCols / 16; ++g) {
+                uint32_t r[16];
+                ptx::tmem_ld_32x32b_x16(taddr + g * 16, r);
                 ptx::tmem_ld_wait();
                 if (ck == 0) {
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) run[g * 32 + j] = __uint_as_float(r[j]);
+                    for (int j = 0; j < 16; ++j) run[g * 16 + j] = __uint_as_float(r[j]);
                 } else {
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) run[g * 32 + j] = __fadd_rn(run[g * 32 + j], __uint_as_float(r[j]));
+                    for (int j = 0; j < 16; ++j) run[g * 16 + j] = __fadd_rn(run[g * 16 + j], __uint_as_float(r[j]));
                 }
             }
             ptx::tc_fence_before();
@@ -380,6 +380,7 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
     const int lane = threadIdx.x % 32;
 
     if (threadIdx.x == 0) {
+        ptx::pdl_launch_dependents();
         for (int s = 0; s < STAGES; ++s) {
             ptx::mbar_init(B.full(s), 1);
             ptx::mbar_init(B.empty(s), 1);
@@ -406,6 +407,7 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
+    ptx::pdl_wait();  // on-chip set-up above overlaps the previous kernel; global memory only after it
 
     int64_t first, end, step;
     worker_items(p, blockIdx.x, gridDim.x, first, end, step);
@@ -526,6 +528,8 @@ template <typename OutT>
 __global__ void __launch_bounds__(256)
 ca_reduce_kernel(const float* __restrict__ ws, int64_t ldw, int64_t layer_stride, int c, int64_t M,
                  int64_t N, OutT* __restrict__ C, int64_t ldc, int vec_store) {
+    ptx::pdl_launch_dependents();
+    ptx::pdl_wait();  // the partials come from the GEMM kernel just before
     const int64_t n4 = (N + 3) / 4;
     const int64_t total = M * n4;
     for (int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; idx < total;

@@ -66,6 +66,7 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
     const bool leader = (rank == 0);
 
     if (threadIdx.x == 0) {
+        ptx::pdl_launch_dependents();
         for (int s = 0; s < STAGES; ++s) {
             ptx::mbar_init(B.full(s), 1);   // the leader's producer arrives once (+ both CTAs' bytes)
             ptx::mbar_init(B.empty(s), 1);  // one multicast commit per use of the stage
@@ -93,6 +94,7 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
     ptx::cluster_sync();  // the peer's barriers are initialised before anyone signals them
     ptx::tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
+    ptx::pdl_wait();  // on-chip set-up above overlaps the previous kernel; global memory only after it
 
     int64_t first, end, step;
     worker_items(p, blockIdx.x / 2, gridDim.x / 2, first, end, step);

@@ -92,6 +92,7 @@ def test_gemm_validation_codes(lib):
     assert call_ex(lib, ldc=100) == E.SFC_ERR_INVALID_ARG          # ldc < N
     assert call_ex(lib, ca_c=0) == E.SFC_ERR_INVALID_ARG
     assert call_ex(lib, K=256, ca_c=5) == E.SFC_ERR_INVALID_ARG    # Kt = 4 < ca_c
+    assert call_ex(lib, K=64 * 5000, ca_c=4097) == E.SFC_ERR_INVALID_ARG  # more than 4096 layers
     assert call_ex(lib, dtype=7) == E.SFC_ERR_INVALID_ARG
     assert call_ex(lib, order=3) == E.SFC_ERR_INVALID_ARG
     assert call_ex(lib, assign=9) == E.SFC_ERR_INVALID_ARG
