@@ -60,13 +60,22 @@ typedef enum { SFC_F32 = 0, SFC_BF16 = 1 } sfc_dtype_t;
 typedef enum { SFC_ORDER_SFC = 0, SFC_ORDER_RASTER = 1 } sfc_order_t;
 
 /* How items are dealt to the P persistent workers.
- * SEGMENT: worker p takes the contiguous block [p*W/P, (p+1)*W/P) of the W
- *          items, the static block partition of Listing 1's parallel loop.
- * WAVE:    worker p takes items p, p+P, p+2P, ...: consecutive curve positions
- *          run at the same time on different SMs, so each wave of P tiles is a
- *          compact patch of the grid and A/B panels are shared through L2.
- * AUTO:    the library picks (currently WAVE). */
-typedef enum { SFC_ASSIGN_SEGMENT = 0, SFC_ASSIGN_WAVE = 1, SFC_ASSIGN_AUTO = 2 } sfc_assign_t;
+ * SEGMENT:     worker p takes the contiguous block [p*W/P, (p+1)*W/P) of the W
+ *              items, the static block partition of Listing 1's parallel loop.
+ * WAVE:        each worker, when free, takes the next curve position from a
+ *              counter shared by the launch, so the tiles running at any time
+ *              are consecutive curve positions -- a compact patch of the grid
+ *              whose A/B panels are shared through L2 -- however the workers'
+ *              speeds drift.
+ * WAVE_STATIC: worker p takes items p, p+P, p+2P, ... (the same deal decided
+ *              up front; kept for comparison).
+ * AUTO:        the library picks (currently WAVE). */
+typedef enum {
+    SFC_ASSIGN_SEGMENT = 0,
+    SFC_ASSIGN_WAVE = 1,
+    SFC_ASSIGN_AUTO = 2,
+    SFC_ASSIGN_WAVE_STATIC = 3
+} sfc_assign_t;
 
 /* Output tile shape and the hardware that computes it.
  * N128 / N256:           128 x 128 / 128 x 256 tiles, one SM each.

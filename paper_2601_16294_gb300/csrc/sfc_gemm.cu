@@ -24,6 +24,7 @@ constexpr int kMaxLayers = 4096;  // keeps the kernels' layer arithmetic in 32 b
 constexpr uint64_t kDefaultTimeoutNs = 2000000000ull;  // 2 s per wait
 
 thread_local int t_last_cuda_error = 0;
+std::atomic<uint64_t> g_launch_seq{0};  // picks each launch's scheduler counter slot
 
 int cuda_fail(cudaError_t e) {
     t_last_cuda_error = static_cast<int>(e);
@@ -107,6 +108,7 @@ struct DeviceInfo {
     int num_sms = 0;
     int chunk_slabs = kDefaultChunkSlabs;
     int serpentine = 0;
+    int one_item_per_worker = 0;
     int workers[kNumVariants] = {0, 0, 0, 0};  // co-resident workers (blocks or pairs) per variant
 };
 DeviceInfo g_devices[kMaxDevices];
@@ -149,6 +151,9 @@ int device_setup(DeviceInfo** info) {
             d.chunk_slabs = v > 0 ? v : (1 << 30);
         }
         if (const char* env = std::getenv("SFC_GEMM_SERPENTINE")) d.serpentine = std::atoi(env) != 0;
+        // experiment override: launch one block (pair) per item instead of one per SM, so the
+        // hardware dispatches the items in curve order as SMs free up
+        if (const char* env = std::getenv("SFC_GEMM_ONE_ITEM_PER_WORKER")) d.one_item_per_worker = std::atoi(env) != 0;
         e = set_attrs<float>();
         if (e == cudaSuccess) e = set_attrs<__nv_bfloat16>();
         if (e != cudaSuccess) { d.status = cuda_fail(e); return; }
@@ -278,7 +283,8 @@ int validate(int64_t M, int64_t N, int64_t K, const void* A, const void* B, cons
     if (lda < K || ldb < N || ldc < N) return SFC_ERR_INVALID_ARG;
     if (c_dtype != SFC_F32 && c_dtype != SFC_BF16) return SFC_ERR_INVALID_ARG;
     if (order != SFC_ORDER_SFC && order != SFC_ORDER_RASTER) return SFC_ERR_INVALID_ARG;
-    if (assign != SFC_ASSIGN_SEGMENT && assign != SFC_ASSIGN_WAVE && assign != SFC_ASSIGN_AUTO)
+    if (assign != SFC_ASSIGN_SEGMENT && assign != SFC_ASSIGN_WAVE && assign != SFC_ASSIGN_AUTO &&
+        assign != SFC_ASSIGN_WAVE_STATIC)
         return SFC_ERR_INVALID_ARG;
     if (tile != SFC_TILE_AUTO && tile != SFC_TILE_N128 && tile != SFC_TILE_N256 && tile != SFC_TILE_PAIR_N128 &&
         tile != SFC_TILE_PAIR_N256)
@@ -342,9 +348,12 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     p.num_items = static_cast<int64_t>(p.Mt) * p.Nt * ca_c;
     p.order = order;
     p.assign = (assign == SFC_ASSIGN_SEGMENT) ? 0 : 1;
+    // dynamic dealing of curve positions for WAVE / AUTO; the static deals stay for comparison
+    p.dynamic = (assign == SFC_ASSIGN_WAVE || assign == SFC_ASSIGN_AUTO) ? 1 : 0;
+    p.sched_slot = static_cast<int>(g_launch_seq.fetch_add(1, std::memory_order_relaxed) % kSchedSlots);
     p.debug_never = debug_never;
     p.timeout_ns = timeout_ns;
-    const int64_t workers = dev->workers[v];
+    const int64_t workers = dev->one_item_per_worker ? p.num_items : dev->workers[v];
     const int64_t used = p.num_items < workers ? p.num_items : workers;
     const int grid = static_cast<int>(variant_pair(v) ? 2 * used : used);
 
@@ -469,6 +478,11 @@ SFC_API int sfc_get_device_status(void* stream) {
     if (word == 0) return SFC_OK;
     const unsigned int zero = 0;
     e = cudaMemcpyToSymbol(g_sfc_status, &zero, sizeof(zero));
+    if (e != cudaSuccess) return cuda_fail(e);
+    // a launch that gave up still returns its scheduler slot, but make sure
+    static const unsigned int zeros[kSchedSlots] = {};
+    e = cudaMemcpyToSymbol(g_sched_next, zeros, sizeof(zeros));
+    if (e == cudaSuccess) e = cudaMemcpyToSymbol(g_sched_done, zeros, sizeof(zeros));
     if (e != cudaSuccess) return cuda_fail(e);
     return SFC_ERR_TIMEOUT;
 }

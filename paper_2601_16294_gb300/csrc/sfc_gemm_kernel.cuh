@@ -62,7 +62,17 @@ enum WaitSite : unsigned int {
     kWaitEpiAccFull = 1u << 11,
     kWaitDebugNever = 1u << 12,
     kWaitDrain = 1u << 13,
+    kWaitQueueFull = 1u << 14,
+    kWaitQueueEmpty = 1u << 15,
 };
+
+// Dynamic item scheduler: per-launch counters (a ring of slots, reset by the
+// last block of the launch to finish) and a small per-worker queue through
+// which the fetching thread hands item indices to the other roles.
+constexpr int kSchedSlots = 1024;
+constexpr int kQueue = 4;
+__device__ unsigned int g_sched_next[kSchedSlots];
+__device__ unsigned int g_sched_done[kSchedSlots];
 
 struct GemmParams {
     int64_t M, N;
@@ -76,7 +86,9 @@ struct GemmParams {
     int64_t ldo;           // row stride of `out` in elements
     int64_t layer_stride;  // elements between K-layer copies in `out`
     int order;             // 0 = generalized Hilbert, 1 = raster
-    int assign;            // 0 = contiguous segments, 1 = strided waves
+    int assign;            // static deal: 0 = contiguous segments, 1 = strided waves
+    int dynamic;           // 1: workers take the next curve position from a shared counter
+    int sched_slot;        // counter slot of this launch (dynamic)
     int vec_store;         // 1 if 16-byte vector stores are aligned
     int tma_store;         // 1: stores go through smem staging and the output tensor map
     int serpentine;        // 1: alternate the K direction between a worker's consecutive items
@@ -112,12 +124,12 @@ __device__ __forceinline__ WorkItem decode_item(int64_t i64, const GemmParams& p
     return w;
 }
 
-// The j-th item of a worker's sequence (it = first + j * step).  With
-// serpentine K order, odd j walk K backwards so that a worker starts each item
-// on the K slabs its previous, neighbouring tile touched last.
-__device__ __forceinline__ WorkItem item_at(int64_t it, int64_t first, int64_t step, const GemmParams& p) {
+// Item `it`, the j-th of its worker.  With serpentine K order, odd j walk K
+// backwards so that a worker starts each item on the K slabs its previous,
+// neighbouring tile touched last.
+__device__ __forceinline__ WorkItem item_at(int64_t it, int j, const GemmParams& p) {
     WorkItem w = decode_item(it, p);
-    w.rev = p.serpentine ? static_cast<int>(((it - first) / step) & 1) : 0;
+    w.rev = p.serpentine ? (j & 1) : 0;
     return w;
 }
 
@@ -208,6 +220,8 @@ struct Barriers {
     __device__ __forceinline__ uint32_t acc_empty(int a) const { return bars + 8u * (2 * stages + 2 + a); }
     __device__ __forceinline__ uint32_t drain() const { return bars + 8u * (2 * stages + 4); }
     __device__ __forceinline__ uint32_t never() const { return bars + 8u * (2 * stages + 5); }
+    __device__ __forceinline__ uint32_t q_full(int q) const { return bars + 8u * (2 * stages + 6 + q); }
+    __device__ __forceinline__ uint32_t q_empty(int q) const { return bars + 8u * (2 * stages + 6 + kQueue + q); }
 };
 
 // Epilogue staging: one 4 KB buffer per epilogue warp (32 rows x 32 columns
@@ -219,12 +233,72 @@ struct RingLayout {
     static constexpr int kRingBytes = STAGE_BYTES * STAGES;
     static constexpr int kStagingOffset = kRingBytes;
     static constexpr int kStagingBytes = EPI_WARPS * kStageBufBytes;
-    static constexpr int kNumBars = 2 * STAGES + 6;
+    static constexpr int kNumBars = 2 * STAGES + 6 + 2 * kQueue;
     static constexpr int kBarOffset = kRingBytes + kStagingBytes;
     static constexpr int kMiscOffset = kBarOffset + kNumBars * 8;
-    static constexpr int kBytes = kMiscOffset + 16;
+    static constexpr int kQueueOffset = kMiscOffset + 16;  // kQueue item indices
+    static constexpr int kBytes = kQueueOffset + 4 * kQueue;
     static constexpr int kDynamicBytes = kBytes + 1024;  // slack to align the ring to 1024 B
 };
+
+// Where a role gets its items: the static deal (first + j * step < end), or
+// the dynamic queue filled by the worker's fetching thread.
+struct ItemSource {
+    int64_t first, end, step;
+    int dynamic;
+    uint32_t q_full0;          // this CTA's q_full[0]
+    uint32_t q_empty0;         // the fetcher CTA's q_empty[0] (cluster address)
+    volatile int* q_item;      // this CTA's queue
+};
+
+// Item j for a consuming role: index >= 0, -1 when there are no more, -2 when
+// a bounded wait gave up.
+__device__ __forceinline__ int64_t src_get(const ItemSource& S, int j, volatile int* abort_flag, uint64_t tmo) {
+    if (!S.dynamic) {
+        const int64_t it = S.first + j * S.step;
+        return it < S.end ? it : -1;
+    }
+    const int q = j % kQueue;
+    if (!wait_bounded(S.q_full0 + 8u * q, static_cast<uint32_t>((j / kQueue) & 1), abort_flag, tmo, kWaitQueueFull))
+        return -2;
+    const int item = S.q_item[q];
+    ptx::mbar_arrive_cluster(S.q_empty0 + 8u * q);  // slot free once every consumer has read it
+    return item;
+}
+
+// Item j for the fetching thread: takes the next curve position from the
+// launch's counter and publishes it to this CTA's queue and, for a pair, to
+// the peer CTA's queue.
+__device__ __forceinline__ int64_t src_fetch(const ItemSource& S, int j, const GemmParams& p, volatile int* abort_flag,
+                                             bool to_peer, uint32_t peer_q_item0, uint32_t peer_q_full0) {
+    if (!S.dynamic) return src_get(S, j, abort_flag, p.timeout_ns);
+    const int q = j % kQueue;
+    if (!wait_bounded(S.q_empty0 + 8u * q, static_cast<uint32_t>(((j / kQueue) & 1) ^ 1), abort_flag, p.timeout_ns,
+                      kWaitQueueEmpty))
+        return -2;
+    const unsigned int v = atomicAdd(&g_sched_next[p.sched_slot], 1u);
+    const int item = (static_cast<int64_t>(v) < p.num_items) ? static_cast<int>(v) : -1;
+    S.q_item[q] = item;
+    ptx::mbar_arrive(S.q_full0 + 8u * q);
+    if (to_peer) {
+        ptx::st_shared_cluster(peer_q_item0 + 4u * q, item);
+        ptx::mbar_arrive_cluster(peer_q_full0 + 8u * q);
+    }
+    return item;
+}
+
+// Called once per block after all roles are done: the last block of the
+// launch returns the counter slot to zero for its next user.
+__device__ __forceinline__ void sched_release(const GemmParams& p) {
+    if (!p.dynamic) return;
+    __threadfence();
+    const unsigned int before = atomicAdd(&g_sched_done[p.sched_slot], 1u);
+    if (before == gridDim.x - 1) {
+        g_sched_next[p.sched_slot] = 0;
+        g_sched_done[p.sched_slot] = 0;
+        __threadfence();
+    }
+}
 
 // Write 32 columns of this lane's row into the warp's staging buffer (32 rows
 // x 32 columns), in the layout of a 64-byte (bf16) or 128-byte (fp32)
@@ -261,8 +335,8 @@ __device__ __forceinline__ void stage_row(uint8_t* buf, int lane, const float* v
 // -------------------------------------------------------------------------
 template <int BN, typename OutT, bool PAIR>
 __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers& B, uint32_t tmem_base,
-                                             volatile int* abort_flag, int64_t first, int64_t end,
-                                             int64_t step, int tile_rows, int row_offset, int warp, int lane,
+                                             volatile int* abort_flag, const ItemSource& src,
+                                             int tile_rows, int row_offset, int warp, int lane,
                                              const CUtensorMap* tmap_c, uint8_t* staging) {
     const int ew = warp - 2;                 // epilogue warp index
     const int quarter = warp & 3;            // TMEM lane quarter this warp may access
@@ -272,8 +346,13 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
     OutT* out = static_cast<OutT*>(p.out);
     const uint32_t acce_target = PAIR ? ptx::map_to_cta(B.acc_empty(0), 0) : B.acc_empty(0);
     float run[kEpiCols];
-    for (int64_t it = first; it < end; it += step) {
-        const WorkItem w = item_at(it, first, step, p);
+    for (int j = 0;; ++j) {
+        // lane 0 takes the item, the warp follows (tcgen05.ld needs the whole warp)
+        int64_t it = 0;
+        if (lane == 0) it = src_get(src, j, abort_flag, p.timeout_ns);
+        it = __shfl_sync(0xffffffffu, it, 0);
+        if (it < 0) break;
+        const WorkItem w = item_at(it, j, p);
         const int nch = num_chunks(w, p.kc);
         bool ok = true;
         for (int ck = 0; ck < nch; ++ck) {
@@ -391,6 +470,10 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
         }
         ptx::mbar_init(B.drain(), 1);
         ptx::mbar_init(B.never(), 1);
+        for (int q = 0; q < kQueue; ++q) {
+            ptx::mbar_init(B.q_full(q), 1);              // the fetching producer publishes
+            ptx::mbar_init(B.q_empty(q), 1 + kEpiWarps);  // MMA warp + epilogue warps have read
+        }
         *abort_flag = 0;
         ptx::fence_barrier_init();
     }
@@ -409,8 +492,12 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
     const uint32_t tmem_base = *tmem_slot;
     ptx::pdl_wait();  // on-chip set-up above overlaps the previous kernel; global memory only after it
 
-    int64_t first, end, step;
-    worker_items(p, blockIdx.x, gridDim.x, first, end, step);
+    ItemSource src;
+    worker_items(p, blockIdx.x, gridDim.x, src.first, src.end, src.step);
+    src.dynamic = p.dynamic;
+    src.q_full0 = B.q_full(0);
+    src.q_empty0 = B.q_empty(0);
+    src.q_item = reinterpret_cast<volatile int*>(smem + L::kQueueOffset);
 
     if (warp == 0) {
         // ------------------------------------------------------ TMA producer
@@ -419,8 +506,13 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
             uint32_t phase = 0;
             int64_t issued = 0;
             bool ok = true;
-            for (int64_t it = first; ok && it < end; it += step) {
-                const WorkItem w = item_at(it, first, step, p);
+            for (int j = 0; ok; ++j) {
+                const int64_t it = src_fetch(src, j, p, abort_flag, false, 0, 0);
+                if (it < 0) {
+                    ok = (it == -1);
+                    break;
+                }
+                const WorkItem w = item_at(it, j, p);
                 for (int q = 0; q < w.k1 - w.k0; ++q) {
                     const int kt = slab_at(w, q);
                     if (!wait_bounded(B.empty(stage), phase ^ 1u, abort_flag, p.timeout_ns, kWaitProducerEmpty)) {
@@ -463,8 +555,13 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
             uint32_t acc_phase = 0;
             bool ok = true;
             if (p.debug_never) ok = wait_bounded(B.never(), 0, abort_flag, p.timeout_ns, kWaitDebugNever);
-            for (int64_t it = first; ok && it < end; it += step) {
-                const WorkItem w = item_at(it, first, step, p);
+            for (int j = 0; ok; ++j) {
+                const int64_t it = src_get(src, j, abort_flag, p.timeout_ns);
+                if (it < 0) {
+                    ok = (it == -1);
+                    break;
+                }
+                const WorkItem w = item_at(it, j, p);
                 const int nch = num_chunks(w, p.kc);
                 for (int ck = 0; ok && ck < nch; ++ck) {
                     const int kb = chunk_begin(w, ck, nch), ke = chunk_begin(w, ck + 1, nch);
@@ -512,7 +609,7 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
             }
         }
     } else {
-        run_epilogue<BN, OutT, false>(p, B, tmem_base, abort_flag, first, end, step, kBM, 0, warp, lane, &tmap_c,
+        run_epilogue<BN, OutT, false>(p, B, tmem_base, abort_flag, src, kBM, 0, warp, lane, &tmap_c,
                                       smem + L::kStagingOffset);
     }
 
@@ -520,6 +617,7 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
     __syncthreads();
     ptx::tc_fence_after();
     if (warp == 1) ptx::tmem_dealloc(tmem_base, kTmemCols);
+    if (threadIdx.x == 0) sched_release(p);
 }
 
 // C = cvt(sum_{l=0}^{c-1} P_l), summed in layer order, 4 columns per thread.

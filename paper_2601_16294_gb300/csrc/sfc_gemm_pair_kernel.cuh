@@ -77,6 +77,11 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
         }
         ptx::mbar_init(B.drain(), 1);
         ptx::mbar_init(B.never(), 1);
+        for (int q = 0; q < kQueue; ++q) {
+            ptx::mbar_init(B.q_full(q), 1);  // the leader's producer publishes
+            // (leader's copy) leader MMA warp + peer producer + both CTAs' epilogue warps have read
+            ptx::mbar_init(B.q_empty(q), 2 + 2 * kEpiWarps);
+        }
         *abort_flag = 0;
         ptx::fence_barrier_init();
     }
@@ -96,8 +101,12 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
     const uint32_t tmem_base = *tmem_slot;
     ptx::pdl_wait();  // on-chip set-up above overlaps the previous kernel; global memory only after it
 
-    int64_t first, end, step;
-    worker_items(p, blockIdx.x / 2, gridDim.x / 2, first, end, step);
+    ItemSource src;
+    worker_items(p, blockIdx.x / 2, gridDim.x / 2, src.first, src.end, src.step);
+    src.dynamic = p.dynamic;
+    src.q_full0 = B.q_full(0);
+    src.q_empty0 = ptx::map_to_cta(B.q_empty(0), 0);
+    src.q_item = reinterpret_cast<volatile int*>(smem + L::kQueueOffset);
 
     if (warp == 0) {
         // ------------------------------------------------ TMA producer (both CTAs)
@@ -106,8 +115,17 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
             uint32_t phase = 0;
             int64_t issued = 0;
             bool ok = true;
-            for (int64_t it = first; ok && it < end; it += step) {
-                const WorkItem w = item_at(it, first, step, p);
+            const uint32_t peer_q_item0 = ptx::map_to_cta(ptx::smem_addr(smem + L::kQueueOffset), 1);
+            const uint32_t peer_q_full0 = ptx::map_to_cta(B.q_full(0), 1);
+            for (int j = 0; ok; ++j) {
+                // the leader takes the next item and hands it to both CTAs; the peer reads its queue
+                const int64_t it = leader ? src_fetch(src, j, p, abort_flag, true, peer_q_item0, peer_q_full0)
+                                          : src_get(src, j, abort_flag, p.timeout_ns);
+                if (it < 0) {
+                    ok = (it == -1);
+                    break;
+                }
+                const WorkItem w = item_at(it, j, p);
                 const int32_t a_row = w.tm * kPairBM + static_cast<int32_t>(rank) * 128;
                 const int32_t b_col = w.tn * BN + static_cast<int32_t>(rank) * kHalfN;
                 for (int q = 0; q < w.k1 - w.k0; ++q) {
@@ -162,8 +180,13 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
             uint32_t acc_phase = 0;
             bool ok = true;
             if (p.debug_never) ok = wait_bounded(B.never(), 0, abort_flag, p.timeout_ns, kWaitDebugNever);
-            for (int64_t it = first; ok && it < end; it += step) {
-                const WorkItem w = item_at(it, first, step, p);
+            for (int j = 0; ok; ++j) {
+                const int64_t it = src_get(src, j, abort_flag, p.timeout_ns);
+                if (it < 0) {
+                    ok = (it == -1);
+                    break;
+                }
+                const WorkItem w = item_at(it, j, p);
                 const int nch = num_chunks(w, p.kc);
                 for (int ck = 0; ok && ck < nch; ++ck) {
                     const int kb = chunk_begin(w, ck, nch), ke = chunk_begin(w, ck + 1, nch);
@@ -210,7 +233,7 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
             }
         }
     } else {
-        run_epilogue<BN, OutT, true>(p, B, tmem_base, abort_flag, first, end, step, kPairBM,
+        run_epilogue<BN, OutT, true>(p, B, tmem_base, abort_flag, src, kPairBM,
                                      static_cast<int>(rank) * 128, warp, lane, &tmap_c, smem + L::kStagingOffset);
     }
 
@@ -219,6 +242,7 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
     ptx::cluster_sync();  // no CTA leaves while its peer may still signal it
     ptx::tc_fence_after();
     if (warp == 1) ptx::tmem_dealloc_pair(tmem_base, kTmemCols);
+    if (threadIdx.x == 0) sched_release(p);
 }
 
 }  // namespace sfc
