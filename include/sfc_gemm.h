@@ -81,13 +81,16 @@ typedef enum {
  * N128 / N256:           128 x 128 / 128 x 256 tiles, one SM each.
  * PAIR_N128 / PAIR_N256: 256 x 128 / 256 x 256 tiles computed by a pair of SMs
  *                        (a 2-CTA cluster; each SM loads half of A and half of B).
+ * QUAD_N256:             512 x 256 tiles computed by two such pairs (a 4-CTA
+ *                        cluster) that share the B slab by TMA multicast.
  * AUTO picks per shape from the tile count and the number of workers. */
 typedef enum {
     SFC_TILE_AUTO = 0,
     SFC_TILE_N128 = 128,
     SFC_TILE_N256 = 256,
     SFC_TILE_PAIR_N128 = 1128,
-    SFC_TILE_PAIR_N256 = 1256
+    SFC_TILE_PAIR_N256 = 1256,
+    SFC_TILE_QUAD_N256 = 2256
 } sfc_tile_t;
 
 /*

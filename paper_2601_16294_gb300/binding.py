@@ -27,7 +27,7 @@ _NAMES = {0: "SFC_OK", -1: "SFC_ERR_INVALID_ARG", -2: "SFC_ERR_UNALIGNED", -3: "
 SFC_F32, SFC_BF16 = 0, 1
 ORDERS = {"sfc": 0, "raster": 1}
 ASSIGNS = {"segment": 0, "wave": 1, "auto": 2, "wave_static": 3}
-TILES = {0: 0, "auto": 0, 128: 128, 256: 256, "pair128": 1128, "pair256": 1256}
+TILES = {0: 0, "auto": 0, 128: 128, 256: 256, "pair128": 1128, "pair256": 1256, "quad256": 2256}
 
 EXPORTS = ("sfc_tile_order", "sfc_tile_order_device", "sfc_gemm_workspace_size", "sfc_gemm", "sfc_gemm_ex",
            "sfc_get_device_status", "sfc_last_cuda_error", "sfc_num_workers", "sfc_debug_force_timeout",

@@ -34,7 +34,7 @@ int cuda_fail(cudaError_t e) {
 // ---------------------------------------------------------- per-device state
 
 // Kernel variants.  Stage counts fill ~192 KB of shared memory per block.
-enum Variant { kSingle128 = 0, kSingle256 = 1, kPair128 = 2, kPair256 = 3, kNumVariants = 4 };
+enum Variant { kSingle128 = 0, kSingle256 = 1, kPair128 = 2, kPair256 = 3, kQuad256 = 4, kNumVariants = 5 };
 constexpr int kStagesSingle256 = 4;  // 48 KB stages
 constexpr int kStagesSingle128 = 6;  // 32 KB stages
 constexpr int kStagesPair256 = 6;    // 32 KB stages per CTA
@@ -42,7 +42,9 @@ constexpr int kStagesPair128 = 8;    // 24 KB stages per CTA
 constexpr int kDefaultChunkSlabs = 64;  // 4096 values of k per tensor-memory accumulation chain
 
 constexpr int variant_bn(int v) { return (v == kSingle128 || v == kPair128) ? 128 : 256; }
-constexpr bool variant_pair(int v) { return v == kPair128 || v == kPair256; }
+constexpr bool variant_pair(int v) { return v == kPair128 || v == kPair256 || v == kQuad256; }
+constexpr int variant_cluster(int v) { return v == kQuad256 ? 4 : (variant_pair(v) ? 2 : 1); }
+constexpr int variant_bm(int v) { return v == kQuad256 ? 512 : (variant_pair(v) ? 256 : 128); }
 
 template <int BN, int STAGES>
 constexpr int single_smem() { return RingLayout<(kBM + BN) * kBK * 2, STAGES, BN / 32>::kDynamicBytes; }
@@ -56,15 +58,18 @@ struct Kernels {
     static constexpr void (*single256)(CUtensorMap, CUtensorMap, CUtensorMap, GemmParams) =
         sfc_gemm_kernel<256, kStagesSingle256, OutT>;
     static constexpr void (*pair128)(CUtensorMap, CUtensorMap, CUtensorMap, GemmParams) =
-        sfc_gemm_pair_kernel<128, kStagesPair128, OutT>;
+        sfc_gemm_pair_kernel<128, kStagesPair128, OutT, false>;
     static constexpr void (*pair256)(CUtensorMap, CUtensorMap, CUtensorMap, GemmParams) =
-        sfc_gemm_pair_kernel<256, kStagesPair256, OutT>;
+        sfc_gemm_pair_kernel<256, kStagesPair256, OutT, false>;
+    static constexpr void (*quad256)(CUtensorMap, CUtensorMap, CUtensorMap, GemmParams) =
+        sfc_gemm_pair_kernel<256, kStagesPair256, OutT, true>;
     static void (*get(int v))(CUtensorMap, CUtensorMap, CUtensorMap, GemmParams) {
         switch (v) {
             case kSingle128: return single128;
             case kSingle256: return single256;
             case kPair128: return pair128;
-            default: return pair256;
+            case kPair256: return pair256;
+            default: return quad256;
         }
     }
 };
@@ -73,7 +78,7 @@ constexpr int variant_smem(int v) {
     return v == kSingle128   ? single_smem<128, kStagesSingle128>()
            : v == kSingle256 ? single_smem<256, kStagesSingle256>()
            : v == kPair128   ? pair_smem<128, kStagesPair128>()
-                             : pair_smem<256, kStagesPair256>();
+                             : pair_smem<256, kStagesPair256>();  // pair256 and quad256
 }
 
 // attr must hold two entries.  With `pdl` the kernel may begin launching
@@ -87,9 +92,9 @@ cudaLaunchConfig_t launch_config(int v, int grid, cudaStream_t s, cudaLaunchAttr
     cfg.stream = s;
     cfg.attrs = attr;
     cfg.numAttrs = 0;
-    if (variant_pair(v)) {
+    if (variant_cluster(v) > 1) {
         attr[cfg.numAttrs].id = cudaLaunchAttributeClusterDimension;
-        attr[cfg.numAttrs].val.clusterDim.x = 2;
+        attr[cfg.numAttrs].val.clusterDim.x = variant_cluster(v);
         attr[cfg.numAttrs].val.clusterDim.y = 1;
         attr[cfg.numAttrs].val.clusterDim.z = 1;
         ++cfg.numAttrs;
@@ -109,7 +114,7 @@ struct DeviceInfo {
     int chunk_slabs = kDefaultChunkSlabs;
     int serpentine = 0;
     int one_item_per_worker = 0;
-    int workers[kNumVariants] = {0, 0, 0, 0};  // co-resident workers (blocks or pairs) per variant
+    int workers[kNumVariants] = {0, 0, 0, 0, 0};  // co-resident workers (blocks or clusters) per variant
 };
 DeviceInfo g_devices[kMaxDevices];
 
@@ -227,10 +232,11 @@ int make_out_map(CUtensorMap* map, const void* ptr, int64_t rows, int64_t cols, 
                           static_cast<cuuint64_t>(layers)};
     cuuint64_t strides[2] = {static_cast<cuuint64_t>(ld) * elem_bytes,
                              static_cast<cuuint64_t>(ld) * elem_bytes * static_cast<cuuint64_t>(rows)};
-    cuuint32_t box[3] = {32, 32, 1};
+    // boxes of 32 rows x 64 bytes (32 bf16 or 16 fp32 columns), 64-byte swizzle
+    cuuint32_t box[3] = {static_cast<cuuint32_t>(64 / elem_bytes), 32, 1};
     cuuint32_t estr[3] = {1, 1, 1};
     const CUtensorMapDataType dt = elem_bytes == 4 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
-    const CUtensorMapSwizzle sw = elem_bytes == 4 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B;
+    const CUtensorMapSwizzle sw = CU_TENSOR_MAP_SWIZZLE_64B;
     CUresult r = encode(map, dt, layers > 1 ? 3 : 2, const_cast<void*>(ptr), dims, strides, box, estr,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, sw, CU_TENSOR_MAP_L2_PROMOTION_NONE,
                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
@@ -254,18 +260,20 @@ int pick_variant(int64_t M, int64_t N, int ca_c, const DeviceInfo& d, sfc_tile_t
         case SFC_TILE_N256: return kSingle256;
         case SFC_TILE_PAIR_N128: return d.workers[kPair128] > 0 ? kPair128 : kSingle128;
         case SFC_TILE_PAIR_N256: return d.workers[kPair256] > 0 ? kPair256 : kSingle256;
+        case SFC_TILE_QUAD_N256: return d.workers[kQuad256] > 0 ? kQuad256 : kSingle256;
         default: break;
     }
     // relative tensor-pipe efficiency measured on GB300 (256-wide tiles feed the
     // tensor core with fewer shared-memory bytes per flop)
-    static const double eff[kNumVariants] = {0.50, 0.85, 0.55, 0.95};
+    static const double eff[kNumVariants] = {0.50, 0.85, 0.55, 0.95, 0.90};
     int best = kSingle128;
     double best_t = 0.0;
     for (int v = 0; v < kNumVariants; ++v) {
         if (d.workers[v] <= 0) continue;
-        const int bm = variant_pair(v) ? 256 : 128, bn = variant_bn(v);
+        const int bm = variant_bm(v), bn = variant_bn(v);
         const int64_t items = ((M + bm - 1) / bm) * ((N + bn - 1) / bn) * ca_c;
         const int64_t waves = (items + d.workers[v] - 1) / d.workers[v];
+        // per-SM work of one item is 128 x bn for every variant
         const double t = static_cast<double>(waves) * 128.0 * bn / eff[v];
         if (v == kSingle128 || t < best_t) {
             best = v;
@@ -287,7 +295,7 @@ int validate(int64_t M, int64_t N, int64_t K, const void* A, const void* B, cons
         assign != SFC_ASSIGN_WAVE_STATIC)
         return SFC_ERR_INVALID_ARG;
     if (tile != SFC_TILE_AUTO && tile != SFC_TILE_N128 && tile != SFC_TILE_N256 && tile != SFC_TILE_PAIR_N128 &&
-        tile != SFC_TILE_PAIR_N256)
+        tile != SFC_TILE_PAIR_N256 && tile != SFC_TILE_QUAD_N256)
         return SFC_ERR_INVALID_ARG;
     // TMA coordinates and tile indices are 32-bit
     if (M > (int64_t(1) << 31) - kBM || N > (int64_t(1) << 31) - 256 || K > (int64_t(1) << 31) - kBK)
@@ -326,11 +334,12 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
 
     const int v = pick_variant(M, N, ca_c, *dev, static_cast<sfc_tile_t>(tile));
     const int bn = variant_bn(v);
-    const int bm = variant_pair(v) ? kPairBM : kBM;
+    const int bm = variant_bm(v);
     CUtensorMap ta, tb;
     rc = make_bf16_map(&ta, A, M, K, lda, kBM, kBK);  // each CTA loads 128 rows of A
     if (rc != SFC_OK) return rc;
-    rc = make_bf16_map(&tb, B, K, N, ldb, kBK, kBBox);
+    // B boxes: 64 K rows x 64 columns; with two pairs sharing B each CTA loads 32 K rows
+    rc = make_bf16_map(&tb, B, K, N, ldb, v == kQuad256 ? kBK / 2 : kBK, kBBox);
     if (rc != SFC_OK) return rc;
 
     GemmParams p;
@@ -355,7 +364,7 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     p.timeout_ns = timeout_ns;
     const int64_t workers = dev->one_item_per_worker ? p.num_items : dev->workers[v];
     const int64_t used = p.num_items < workers ? p.num_items : workers;
-    const int grid = static_cast<int>(variant_pair(v) ? 2 * used : used);
+    const int grid = static_cast<int>(variant_cluster(v) * used);
 
     void* ws = workspace;
     bool pooled = false;

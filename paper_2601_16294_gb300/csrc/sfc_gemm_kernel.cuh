@@ -15,7 +15,9 @@
 //   warps 2..     epilogue: tcgen05.ld the accumulator (warp w reads TMEM lanes
 //                 32*(w%4)..), add it into fp32 running sums held in registers,
 //                 and after the item's last chunk convert and store the tile
-//                 (masked at the M/N edges).
+//                 (masked at the M/N edges);
+//   last warp     scheduler: deals the worker's items (curve positions) and
+//                 decodes each into its tile before any other role needs it.
 //
 // Accumulation chains.  The tensor core's fp32 accumulation drops low-order
 // bits on every accumulate, so the error of one long chain grows linearly with
@@ -49,8 +51,9 @@ constexpr int kBBox = 64;         // B is loaded in 64-column boxes (128 bytes)
 constexpr int kEpiCols = 128;     // accumulator columns each epilogue thread owns
 
 // Threads of a block: producer warp, MMA warp, BN/32 epilogue warps
-// (4 warps per 128 columns: one warp per TMEM lane quarter).
-__host__ __device__ constexpr int block_threads(int bn) { return 64 + 32 * (bn / 32); }
+// (4 warps per 128 columns: one warp per TMEM lane quarter), scheduler warp.
+__host__ __device__ constexpr int block_threads(int bn) { return 96 + 32 * (bn / 32); }
+__host__ __device__ constexpr int scheduler_warp(int bn) { return 2 + bn / 32; }
 
 // device error word: bit 0 = a bounded wait gave up; bits 8.. = which wait
 __device__ unsigned int g_sfc_status = 0;
@@ -66,9 +69,14 @@ enum WaitSite : unsigned int {
     kWaitQueueEmpty = 1u << 15,
 };
 
-// Dynamic item scheduler: per-launch counters (a ring of slots, reset by the
-// last block of the launch to finish) and a small per-worker queue through
-// which the fetching thread hands item indices to the other roles.
+// Item dealing.  One scheduler thread per worker decodes the worker's items
+// (curve position -> tile, K layer) and hands them to every role of every CTA
+// of the worker through a small queue in shared memory.  Static dealing gives
+// worker w the items first + j * step; dynamic dealing gives it item w first
+// (so no block waits on a counter to start) and then workers + the next value
+// of a per-launch counter, i.e. curve positions are taken in order as workers
+// free up.  The counters form a ring of slots, one per launch, each reset by
+// the last scheduler of its launch to finish.
 constexpr int kSchedSlots = 1024;
 constexpr int kQueue = 4;
 __device__ unsigned int g_sched_next[kSchedSlots];
@@ -121,15 +129,6 @@ __device__ __forceinline__ WorkItem decode_item(int64_t i64, const GemmParams& p
     w.k0 = layer_k0(layer, p);
     w.k1 = layer_k0(layer + 1, p);
     w.rev = 0;
-    return w;
-}
-
-// Item `it`, the j-th of its worker.  With serpentine K order, odd j walk K
-// backwards so that a worker starts each item on the K slabs its previous,
-// neighbouring tile touched last.
-__device__ __forceinline__ WorkItem item_at(int64_t it, int j, const GemmParams& p) {
-    WorkItem w = decode_item(it, p);
-    w.rev = p.serpentine ? (j & 1) : 0;
     return w;
 }
 
@@ -222,10 +221,10 @@ struct Barriers {
     __device__ __forceinline__ uint32_t never() const { return bars + 8u * (2 * stages + 5); }
     __device__ __forceinline__ uint32_t q_full(int q) const { return bars + 8u * (2 * stages + 6 + q); }
     __device__ __forceinline__ uint32_t q_empty(int q) const { return bars + 8u * (2 * stages + 6 + kQueue + q); }
+    __device__ __forceinline__ uint32_t q_taken() const { return bars + 8u * (2 * stages + 6 + 2 * kQueue); }
 };
 
-// Epilogue staging: one 4 KB buffer per epilogue warp (32 rows x 32 columns
-// of fp32, or of bf16 in its first half), swizzled like the output tensor map.
+// Epilogue staging: one 4 KB buffer per epilogue warp (two output boxes).
 constexpr int kStageBufBytes = 4096;
 
 template <int STAGE_BYTES, int STAGES, int EPI_WARPS>
@@ -233,99 +232,172 @@ struct RingLayout {
     static constexpr int kRingBytes = STAGE_BYTES * STAGES;
     static constexpr int kStagingOffset = kRingBytes;
     static constexpr int kStagingBytes = EPI_WARPS * kStageBufBytes;
-    static constexpr int kNumBars = 2 * STAGES + 6 + 2 * kQueue;
-    static constexpr int kBarOffset = kRingBytes + kStagingBytes;
+    static constexpr int kQueueOffset = kRingBytes + kStagingBytes;  // kQueue entries of 16 bytes
+    static constexpr int kNumBars = 2 * STAGES + 7 + 2 * kQueue;
+    static constexpr int kBarOffset = kQueueOffset + 16 * kQueue;
     static constexpr int kMiscOffset = kBarOffset + kNumBars * 8;
-    static constexpr int kQueueOffset = kMiscOffset + 16;  // kQueue item indices
-    static constexpr int kBytes = kQueueOffset + 4 * kQueue;
+    static constexpr int kBytes = kMiscOffset + 16;
     static constexpr int kDynamicBytes = kBytes + 1024;  // slack to align the ring to 1024 B
 };
 
-// Where a role gets its items: the static deal (first + j * step < end), or
-// the dynamic queue filled by the worker's fetching thread.
+// A worker's item source: the scheduler's deal parameters and the queue.
+// Queue entry q (16 bytes): item index (-1: no more items), tm, tn, K layer.
 struct ItemSource {
-    int64_t first, end, step;
+    int64_t first, end, step;  // static deal: first + j * step while < end
+    int64_t worker, workers;   // this worker and the launch's worker count
     int dynamic;
     uint32_t q_full0;          // this CTA's q_full[0]
-    uint32_t q_empty0;         // the fetcher CTA's q_empty[0] (cluster address)
-    volatile int* q_item;      // this CTA's queue
+    uint32_t q_empty0;         // the scheduler CTA's q_empty[0] (cluster address)
+    volatile int* q_entry;     // this CTA's queue
 };
 
-// Item j for a consuming role: index >= 0, -1 when there are no more, -2 when
-// a bounded wait gave up.
-__device__ __forceinline__ int64_t src_get(const ItemSource& S, int j, volatile int* abort_flag, uint64_t tmo) {
-    if (!S.dynamic) {
-        const int64_t it = S.first + j * S.step;
-        return it < S.end ? it : -1;
-    }
+// Item j of a consuming role: fills w (tile, K layer and range; K order from
+// j) and returns the item index >= 0, or -1 when there are no more, -2 when a
+// bounded wait gave up.
+__device__ __forceinline__ int64_t src_take(const ItemSource& S, int j, const GemmParams& p, volatile int* abort_flag,
+                                            WorkItem& w) {
     const int q = j % kQueue;
-    if (!wait_bounded(S.q_full0 + 8u * q, static_cast<uint32_t>((j / kQueue) & 1), abort_flag, tmo, kWaitQueueFull))
+    if (!wait_bounded(S.q_full0 + 8u * q, static_cast<uint32_t>((j / kQueue) & 1), abort_flag, p.timeout_ns,
+                      kWaitQueueFull))
         return -2;
-    const int item = S.q_item[q];
+    const int item = S.q_entry[4 * q];
+    w.tm = S.q_entry[4 * q + 1];
+    w.tn = S.q_entry[4 * q + 2];
+    w.layer = S.q_entry[4 * q + 3];
     ptx::mbar_arrive_cluster(S.q_empty0 + 8u * q);  // slot free once every consumer has read it
+    w.k0 = layer_k0(w.layer, p);
+    w.k1 = layer_k0(w.layer + 1, p);
+    w.rev = p.serpentine ? (j & 1) : 0;
     return item;
 }
 
-// Item j for the fetching thread: takes the next curve position from the
-// launch's counter and publishes it to this CTA's queue and, for a pair, to
-// the peer CTA's queue.
-__device__ __forceinline__ int64_t src_fetch(const ItemSource& S, int j, const GemmParams& p, volatile int* abort_flag,
-                                             bool to_peer, uint32_t peer_q_item0, uint32_t peer_q_full0) {
-    if (!S.dynamic) return src_get(S, j, abort_flag, p.timeout_ns);
+// Scheduler: decode item j and publish it to slot j % kQueue of this CTA's
+// queue and of the other n_ctas - 1 CTAs of the cluster (the slot is free).
+__device__ __forceinline__ void sched_publish(const ItemSource& S, int j, int item, const GemmParams& p, int n_ctas) {
     const int q = j % kQueue;
-    if (!wait_bounded(S.q_empty0 + 8u * q, static_cast<uint32_t>(((j / kQueue) & 1) ^ 1), abort_flag, p.timeout_ns,
-                      kWaitQueueEmpty))
-        return -2;
-    const unsigned int v = atomicAdd(&g_sched_next[p.sched_slot], 1u);
-    const int item = (static_cast<int64_t>(v) < p.num_items) ? static_cast<int>(v) : -1;
-    S.q_item[q] = item;
+    int e[4] = {item, 0, 0, 0};
+    if (item >= 0) {
+        const WorkItem w = decode_item(item, p);
+        e[1] = w.tm;
+        e[2] = w.tn;
+        e[3] = w.layer;
+    }
+#pragma unroll
+    for (int k = 0; k < 4; ++k) S.q_entry[4 * q + k] = e[k];
     ptx::mbar_arrive(S.q_full0 + 8u * q);
-    if (to_peer) {
-        ptx::st_shared_cluster(peer_q_item0 + 4u * q, item);
-        ptx::mbar_arrive_cluster(peer_q_full0 + 8u * q);
+    const uint32_t mine = ptx::smem_addr(const_cast<int*>(S.q_entry) + 4 * q);
+    for (int r = 1; r < n_ctas; ++r) {
+        const uint32_t dst = ptx::map_to_cta(mine, r);
+#pragma unroll
+        for (int k = 0; k < 4; ++k) ptx::st_shared_cluster(dst + 4u * k, e[k]);
+        ptx::mbar_arrive_cluster(ptx::map_to_cta(S.q_full0 + 8u * q, r));
     }
-    return item;
 }
 
-// Called once per block after all roles are done: the last block of the
-// launch returns the counter slot to zero for its next user.
-__device__ __forceinline__ void sched_release(const GemmParams& p) {
-    if (!p.dynamic) return;
-    __threadfence();
-    const unsigned int before = atomicAdd(&g_sched_done[p.sched_slot], 1u);
-    if (before == gridDim.x - 1) {
-        g_sched_next[p.sched_slot] = 0;
-        g_sched_done[p.sched_slot] = 0;
+// Item j of the worker's deal (j >= 1 for dynamic dealing takes a ticket).
+__device__ __forceinline__ int sched_next(const ItemSource& S, int j, const GemmParams& p) {
+    int64_t pos;
+    if (S.dynamic)
+        pos = (j == 0) ? S.worker : S.workers + static_cast<int64_t>(atomicAdd(&g_sched_next[p.sched_slot], 1u));
+    else
+        pos = S.first + j * S.step;
+    const int64_t end = S.dynamic ? p.num_items : S.end;
+    return pos < end ? static_cast<int>(pos) : -1;
+}
+
+// Scheduler loop, items 1.. (item 0 is published during set-up).  Item j is
+// published once the worker's producer has taken item j - 1, so tickets are
+// taken one item ahead of need: late enough that dynamic dealing still
+// balances the last wave, early enough that the counter's round trip and the
+// decode are off every other role's path.  Returns false when a bounded wait
+// gave up.
+__device__ __forceinline__ bool run_scheduler(const ItemSource& S, int item0, const GemmParams& p, const Barriers& B,
+                                              volatile int* abort_flag, int n_ctas) {
+    bool ok = true;
+    for (int j = 1; ok && item0 >= 0; ++j) {
+        if (!wait_bounded(B.q_taken(), static_cast<uint32_t>((j - 1) & 1), abort_flag, p.timeout_ns,
+                          kWaitQueueEmpty) ||
+            !wait_bounded(S.q_empty0 + 8u * (j % kQueue), static_cast<uint32_t>(((j / kQueue) & 1) ^ 1), abort_flag,
+                          p.timeout_ns, kWaitQueueEmpty)) {
+            ok = false;
+            break;
+        }
+        const int item = sched_next(S, j, p);
+        sched_publish(S, j, item, p, n_ctas);
+        if (item < 0) break;
+    }
+    if (S.dynamic) {
+        // the last scheduler of the launch returns the counter slot to zero
         __threadfence();
+        const unsigned int before = atomicAdd(&g_sched_done[p.sched_slot], 1u);
+        if (static_cast<int64_t>(before) == S.workers - 1) {
+            g_sched_next[p.sched_slot] = 0;
+            g_sched_done[p.sched_slot] = 0;
+            __threadfence();
+        }
+    }
+    return ok;
+}
+
+// Producer loop shared by the kernels: takes the worker's items from the
+// queue and, for each K slab, waits for a free ring stage and calls
+// issue(w, kt, stage).  `signal_taken`: this is the producer the scheduler
+// paces itself on.  Returns false when a bounded wait gave up; `issued`
+// counts the stages filled.
+template <int STAGES, typename IssueFn>
+__device__ __forceinline__ bool produce(const ItemSource& src, const GemmParams& p, const Barriers& B,
+                                        volatile int* abort_flag, bool signal_taken, int64_t& issued,
+                                        IssueFn&& issue) {
+    int stage = 0;
+    uint32_t phase = 0;
+    for (int j = 0;; ++j) {
+        WorkItem w;
+        const int64_t it = src_take(src, j, p, abort_flag, w);
+        if (it < 0) return it == -1;
+        if (signal_taken) ptx::mbar_arrive(B.q_taken());
+        const int nq = w.k1 - w.k0;
+        for (int q = 0; q < nq; ++q) {
+            if (!wait_bounded(B.empty(stage), phase ^ 1u, abort_flag, p.timeout_ns, kWaitProducerEmpty))
+                return false;
+            issue(w, slab_at(w, q), stage);
+            ++issued;
+            if (++stage == STAGES) {
+                stage = 0;
+                phase ^= 1u;
+            }
+        }
     }
 }
 
-// Write 32 columns of this lane's row into the warp's staging buffer (32 rows
-// x 32 columns), in the layout of a 64-byte (bf16) or 128-byte (fp32)
-// swizzled TMA box: 16-byte unit j of row r sits at unit j ^ (swizzle of r).
-// Distinct rows of 8 consecutive lanes land in distinct bank groups.
+// Output staging boxes are 32 rows x 64 bytes: 32 bf16 or 16 fp32 columns,
+// in the layout of a 64-byte swizzled TMA box (16-byte unit j of row r sits at
+// unit j ^ ((r >> 1) & 3)).  Each epilogue warp owns a 4 KB buffer holding two
+// boxes, so one box is filled while the TMA still reads the other.
+constexpr int kBoxBytes = 2048;
 template <typename OutT>
-__device__ __forceinline__ void stage_row(uint8_t* buf, int lane, const float* v) {
-    if constexpr (sizeof(OutT) == 4) {
-        uint8_t* row = buf + lane * 128;
-        const int sw = lane & 7;
+__host__ __device__ constexpr int box_cols() { return 64 / static_cast<int>(sizeof(OutT)); }
+
+// Write this lane's row of one box (box_cols<OutT>() values from v).
+template <typename OutT>
+__device__ __forceinline__ void stage_row(uint8_t* box, int lane, const float* v) {
+    uint8_t* row = box + lane * 64;
+    const int sw = (lane >> 1) & 3;
 #pragma unroll
-        for (int j = 0; j < 8; ++j)
-            *reinterpret_cast<float4*>(row + ((j ^ sw) * 16)) =
-                make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
-    } else {
-        uint8_t* row = buf + lane * 64;
-        const int sw = (lane >> 1) & 3;
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
+    for (int j = 0; j < 4; ++j) {
+        uint4 u;
+        if constexpr (sizeof(OutT) == 4) {
+            u = make_uint4(__float_as_uint(v[4 * j]), __float_as_uint(v[4 * j + 1]), __float_as_uint(v[4 * j + 2]),
+                           __float_as_uint(v[4 * j + 3]));
+        } else {
             uint32_t w[4];
 #pragma unroll
             for (int h = 0; h < 4; ++h) {
                 __nv_bfloat162 b = __floats2bfloat162_rn(v[8 * j + 2 * h], v[8 * j + 2 * h + 1]);
                 w[h] = *reinterpret_cast<uint32_t*>(&b);
             }
-            *reinterpret_cast<uint4*>(row + ((j ^ sw) * 16)) = make_uint4(w[0], w[1], w[2], w[3]);
+            u = make_uint4(w[0], w[1], w[2], w[3]);
         }
+        *reinterpret_cast<uint4*>(row + ((j ^ sw) * 16)) = u;
     }
 }
 
@@ -337,22 +409,28 @@ template <int BN, typename OutT, bool PAIR>
 __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers& B, uint32_t tmem_base,
                                              volatile int* abort_flag, const ItemSource& src,
                                              int tile_rows, int row_offset, int warp, int lane,
-                                             const CUtensorMap* tmap_c, uint8_t* staging) {
+                                             const CUtensorMap* tmap_c, uint8_t* staging, uint32_t pair_leader = 0) {
     const int ew = warp - 2;                 // epilogue warp index
     const int quarter = warp & 3;            // TMEM lane quarter this warp may access
     const int half = ew / 4;                 // which 128-column half of the tile
     int acc = 0;
     uint32_t acc_phase = 0;
     OutT* out = static_cast<OutT*>(p.out);
-    const uint32_t acce_target = PAIR ? ptx::map_to_cta(B.acc_empty(0), 0) : B.acc_empty(0);
+    const uint32_t acce_target = PAIR ? ptx::map_to_cta(B.acc_empty(0), pair_leader) : B.acc_empty(0);
     float run[kEpiCols];
+    int nbox = 0;  // boxes this warp has stored (selects the staging half)
     for (int j = 0;; ++j) {
         // lane 0 takes the item, the warp follows (tcgen05.ld needs the whole warp)
         int64_t it = 0;
-        if (lane == 0) it = src_get(src, j, abort_flag, p.timeout_ns);
+        WorkItem w{};
+        if (lane == 0) it = src_take(src, j, p, abort_flag, w);
         it = __shfl_sync(0xffffffffu, it, 0);
         if (it < 0) break;
-        const WorkItem w = item_at(it, j, p);
+        w.tm = __shfl_sync(0xffffffffu, w.tm, 0);
+        w.tn = __shfl_sync(0xffffffffu, w.tn, 0);
+        w.layer = __shfl_sync(0xffffffffu, w.layer, 0);
+        w.k0 = __shfl_sync(0xffffffffu, w.k0, 0);
+        w.k1 = __shfl_sync(0xffffffffu, w.k1, 0);
         const int nch = num_chunks(w, p.kc);
         bool ok = true;
         for (int ck = 0; ck < nch; ++ck) {
@@ -368,17 +446,13 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
             const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
                                    static_cast<uint32_t>(acc * BN + half * kEpiCols);
 #pragma unroll
-            for (int g = 0; g < kEpiCols / 16; ++g) {
-                uint32_t r[16];
-                ptx::tmem_ld_32x32b_x16(taddr + g * 16, r);
+            for (int g = 0; g < kEpiCols / 32; ++g) {
+                uint32_t r[32];
+                ptx::tmem_ld_32x32b_x32(taddr + g * 32, r);
                 ptx::tmem_ld_wait();
-                if (ck == 0) {
 #pragma unroll
-                    for (int j = 0; j < 16; ++j) run[g * 16 + j] = __uint_as_float(r[j]);
-                } else {
-#pragma unroll
-                    for (int j = 0; j < 16; ++j) run[g * 16 + j] = __fadd_rn(run[g * 16 + j], __uint_as_float(r[j]));
-                }
+                for (int j = 0; j < 32; ++j)
+                    run[g * 32 + j] = (ck == 0) ? __uint_as_float(r[j]) : __fadd_rn(run[g * 32 + j], __uint_as_float(r[j]));
             }
             ptx::tc_fence_before();
             __syncwarp();
@@ -396,26 +470,29 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
         const int64_t warp_row = static_cast<int64_t>(w.tm) * tile_rows + row_offset + quarter * 32;
         const int64_t col_base = static_cast<int64_t>(w.tn) * BN + half * kEpiCols;
         if (p.tma_store) {
-            // stage 32 x 32 blocks and let the TMA write them (edges clipped by the map)
-            uint8_t* buf = staging + ew * kStageBufBytes;
-            const uint32_t buf_addr = ptx::smem_addr(buf);
+            // stage 32-row boxes and let the TMA write them (edges clipped by the map);
+            // the two boxes of the buffer alternate
+            constexpr int kCols = box_cols<OutT>();
 #pragma unroll
-            for (int g = 0; g < kEpiCols / 32; ++g) {
-                if (col_base + g * 32 >= p.N) break;  // warp-uniform
-                stage_row<OutT>(buf, lane, run + g * 32);
+            for (int g = 0; g < kEpiCols / kCols; ++g) {
+                if (col_base + g * kCols >= p.N) break;  // warp-uniform
+                uint8_t* box = staging + ew * kStageBufBytes + (nbox & 1) * kBoxBytes;
+                if (lane == 0) ptx::bulk_wait_read_1();  // the store that last used this box has read it
+                __syncwarp();
+                stage_row<OutT>(box, lane, run + g * kCols);
                 ptx::fence_proxy_async_smem();
                 __syncwarp();
                 if (lane == 0) {
+                    const uint32_t box_addr = ptx::smem_addr(box);
                     if (p.ca_c > 1)
-                        ptx::tma_store_3d(tmap_c, buf_addr, static_cast<int32_t>(col_base + g * 32),
+                        ptx::tma_store_3d(tmap_c, box_addr, static_cast<int32_t>(col_base + g * kCols),
                                           static_cast<int32_t>(warp_row), w.layer);
                     else
-                        ptx::tma_store_2d(tmap_c, buf_addr, static_cast<int32_t>(col_base + g * 32),
+                        ptx::tma_store_2d(tmap_c, box_addr, static_cast<int32_t>(col_base + g * kCols),
                                           static_cast<int32_t>(warp_row));
                     ptx::bulk_commit();
-                    ptx::bulk_wait_read_all();  // buffer free again
                 }
-                __syncwarp();
+                ++nbox;
             }
         } else {
             const int64_t row = warp_row + lane;
@@ -427,7 +504,8 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
             }
         }
     }
-    if (p.tma_store && lane == 0) ptx::bulk_wait_all();
+    // the staging buffer must not be released while the TMA still reads it
+    if (p.tma_store && lane == 0) ptx::bulk_wait_read_all();
 }
 
 // -------------------------------------------------------------------------
@@ -471,9 +549,10 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
         ptx::mbar_init(B.drain(), 1);
         ptx::mbar_init(B.never(), 1);
         for (int q = 0; q < kQueue; ++q) {
-            ptx::mbar_init(B.q_full(q), 1);              // the fetching producer publishes
-            ptx::mbar_init(B.q_empty(q), 1 + kEpiWarps);  // MMA warp + epilogue warps have read
+            ptx::mbar_init(B.q_full(q), 1);               // the scheduler publishes
+            ptx::mbar_init(B.q_empty(q), 2 + kEpiWarps);  // producer, MMA warp and epilogue warps have read
         }
+        ptx::mbar_init(B.q_taken(), 1);  // the producer took an item
         *abort_flag = 0;
         ptx::fence_barrier_init();
     }
@@ -490,50 +569,39 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
-    ptx::pdl_wait();  // on-chip set-up above overlaps the previous kernel; global memory only after it
 
     ItemSource src;
     worker_items(p, blockIdx.x, gridDim.x, src.first, src.end, src.step);
+    src.worker = blockIdx.x;
+    src.workers = gridDim.x;
     src.dynamic = p.dynamic;
     src.q_full0 = B.q_full(0);
     src.q_empty0 = B.q_empty(0);
-    src.q_item = reinterpret_cast<volatile int*>(smem + L::kQueueOffset);
+    src.q_entry = reinterpret_cast<volatile int*>(smem + L::kQueueOffset);
+    // the first item needs no global memory: decode and publish it before the wait below
+    const bool sched_thread = (warp == scheduler_warp(BN) && lane == 0);
+    int item0 = -1;
+    if (sched_thread) {
+        item0 = sched_next(src, 0, p);
+        sched_publish(src, 0, item0, p, 1);
+    }
+    ptx::pdl_wait();  // on-chip set-up above overlaps the previous kernel; global memory only after it
 
     if (warp == 0) {
         // ------------------------------------------------------ TMA producer
         if (lane == 0) {
-            int stage = 0;
-            uint32_t phase = 0;
             int64_t issued = 0;
-            bool ok = true;
-            for (int j = 0; ok; ++j) {
-                const int64_t it = src_fetch(src, j, p, abort_flag, false, 0, 0);
-                if (it < 0) {
-                    ok = (it == -1);
-                    break;
-                }
-                const WorkItem w = item_at(it, j, p);
-                for (int q = 0; q < w.k1 - w.k0; ++q) {
-                    const int kt = slab_at(w, q);
-                    if (!wait_bounded(B.empty(stage), phase ^ 1u, abort_flag, p.timeout_ns, kWaitProducerEmpty)) {
-                        ok = false;
-                        break;
-                    }
-                    ptx::mbar_arrive_expect_tx(B.full(stage), kStageBytes);
-                    const uint32_t sa = ring + stage * kStageBytes;
-                    const uint32_t sb = sa + kABytes;
-                    ptx::tma_load_2d(sa, &tmap_a, B.full(stage), kt * kBK, w.tm * kBM);
+            bool ok = produce<STAGES>(src, p, B, abort_flag, /*signal_taken=*/true, issued,
+                                      [&](const WorkItem& w, int kt, int stage) {
+                ptx::mbar_arrive_expect_tx(B.full(stage), kStageBytes);
+                const uint32_t sa = ring + stage * kStageBytes;
+                const uint32_t sb = sa + kABytes;
+                ptx::tma_load_2d(sa, &tmap_a, B.full(stage), kt * kBK, w.tm * kBM);
 #pragma unroll
-                    for (int j = 0; j < BN / kBBox; ++j)
-                        ptx::tma_load_2d(sb + j * (kBBox * kBK * 2), &tmap_b, B.full(stage), w.tn * BN + j * kBBox,
-                                         kt * kBK);
-                    ++issued;
-                    if (++stage == STAGES) {
-                        stage = 0;
-                        phase ^= 1u;
-                    }
-                }
-            }
+                for (int jb = 0; jb < BN / kBBox; ++jb)
+                    ptx::tma_load_2d(sb + jb * (kBBox * kBK * 2), &tmap_b, B.full(stage), w.tn * BN + jb * kBBox,
+                                     kt * kBK);
+            });
             // Tail: the last STAGES issues.  On success wait until the MMA warp's
             // commits have released them (no arrive may land after exit); after a
             // failure wait (bounded) for the copies still in flight into the ring.
@@ -556,12 +624,12 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
             bool ok = true;
             if (p.debug_never) ok = wait_bounded(B.never(), 0, abort_flag, p.timeout_ns, kWaitDebugNever);
             for (int j = 0; ok; ++j) {
-                const int64_t it = src_get(src, j, abort_flag, p.timeout_ns);
+                WorkItem w;
+                const int64_t it = src_take(src, j, p, abort_flag, w);
                 if (it < 0) {
                     ok = (it == -1);
                     break;
                 }
-                const WorkItem w = item_at(it, j, p);
                 const int nch = num_chunks(w, p.kc);
                 for (int ck = 0; ok && ck < nch; ++ck) {
                     const int kb = chunk_begin(w, ck, nch), ke = chunk_begin(w, ck + 1, nch);
@@ -608,16 +676,18 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
                 wait_bounded(B.drain(), 0, abort_flag, p.timeout_ns, kWaitDrain, /*honour_abort=*/false);
             }
         }
-    } else {
+    } else if (warp < scheduler_warp(BN)) {
         run_epilogue<BN, OutT, false>(p, B, tmem_base, abort_flag, src, kBM, 0, warp, lane, &tmap_c,
                                       smem + L::kStagingOffset);
+    } else if (sched_thread) {
+        // -------------------------------------------------------- scheduler
+        run_scheduler(src, item0, p, B, abort_flag, 1);
     }
 
     ptx::tc_fence_before();
     __syncthreads();
     ptx::tc_fence_after();
     if (warp == 1) ptx::tmem_dealloc(tmem_base, kTmemCols);
-    if (threadIdx.x == 0) sched_release(p);
 }
 
 // C = cvt(sum_{l=0}^{c-1} P_l), summed in layer order, 4 columns per thread.

@@ -1,4 +1,5 @@
-// sfc_gemm_pair_kernel.cuh -- the SFC / SFC-CA GEMM on 2-SM CTA pairs.
+// sfc_gemm_pair_kernel.cuh -- the SFC / SFC-CA GEMM on 2-SM CTA pairs (and on
+// clusters of two pairs that share the B slab).
 //
 // Same task space, item order, accumulation chunks and epilogue as
 // sfc_gemm_kernel, but each worker is a cluster of two CTAs on two SMs that
@@ -16,6 +17,13 @@
 //   - CTA r's tensor memory holds rows [128 r, 128 r + 128) of the tile; its
 //     epilogue warps drain them and arrive on the leader's accumulator-empty
 //     barrier.
+//
+// QUAD variant: a 4-CTA cluster holds two pairs stacked in M, so an item is a
+// 512 x BN tile.  Both pairs need the same B slab: CTA r of each pair loads 32 of
+// the 64 K rows of its B half and multicasts them to itself and its counterpart
+// in the other pair, which halves the B bytes each SM requests from L2.  A stage
+// of a CTA is then written by two producers, so it is free only after both
+// pairs' MMAs have committed it (empty barriers count two arrivals).
 //
 // Waits are bounded as in the single-SM kernel.  The pair meets at a cluster
 // barrier after set-up (barriers initialised before any remote signal) and
@@ -38,7 +46,7 @@ struct PairStage {
     static_assert(kABytes % 1024 == 0 && kBBytes % 1024 == 0, "swizzle atoms need 1 KB alignment");
 };
 
-template <int BN, int STAGES, typename OutT>
+template <int BN, int STAGES, typename OutT, bool QUAD>
 __global__ void __launch_bounds__(block_threads(BN), 1)
 sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_b,
                      const __grid_constant__ CUtensorMap tmap_c, const GemmParams p) {
@@ -49,7 +57,9 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
     constexpr int kHalfN = S::kHalfN;
     constexpr uint32_t kIdesc = ptx::idesc_bf16_f32(kPairBM, BN, /*A K-major*/ 0, /*B MN-major*/ 1);
     constexpr uint32_t kTmemCols = 2 * BN;
-    constexpr uint16_t kBothCtas = 0x3;
+    // QUAD: a cluster of two pairs stacked in M (a 512 x BN item) sharing the B slab
+    constexpr int kCtas = QUAD ? 4 : 2;
+    constexpr int kItemRows = QUAD ? 2 * kPairBM : kPairBM;
 
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = ptx::smem_addr(smem_raw);
@@ -63,25 +73,32 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
     const int warp = threadIdx.x / 32;
     const int lane = threadIdx.x % 32;
     const uint32_t rank = ptx::cluster_ctarank();
-    const bool leader = (rank == 0);
+    const uint32_t r = rank & 1u;               // position in the pair
+    const uint32_t pair_idx = rank >> 1;        // which pair of the cluster
+    const uint32_t pair_leader = rank & ~1u;    // the pair's MMA-issuing CTA
+    const bool leader = (r == 0);
+    const uint16_t pair_mask = static_cast<uint16_t>(0x3u << (2 * pair_idx));
+    const uint16_t stage_mask = QUAD ? 0xF : 0x3;  // CTAs whose smem a stage's loads write
 
     if (threadIdx.x == 0) {
         ptx::pdl_launch_dependents();
         for (int s = 0; s < STAGES; ++s) {
-            ptx::mbar_init(B.full(s), 1);   // the leader's producer arrives once (+ both CTAs' bytes)
-            ptx::mbar_init(B.empty(s), 1);  // one multicast commit per use of the stage
+            ptx::mbar_init(B.full(s), 1);           // the pair leader's producer arrives once (+ tx bytes)
+            ptx::mbar_init(B.empty(s), QUAD ? 2 : 1);  // a commit from each pair whose loads share the stage
         }
         for (int a = 0; a < 2; ++a) {
             ptx::mbar_init(B.acc_full(a), 1);               // one multicast commit per chunk
-            ptx::mbar_init(B.acc_empty(a), 2 * kEpiWarps);  // epilogue warps of both CTAs (leader's copy used)
+            ptx::mbar_init(B.acc_empty(a), 2 * kEpiWarps);  // epilogue warps of the pair (leader's copy used)
         }
         ptx::mbar_init(B.drain(), 1);
         ptx::mbar_init(B.never(), 1);
         for (int q = 0; q < kQueue; ++q) {
-            ptx::mbar_init(B.q_full(q), 1);  // the leader's producer publishes
-            // (leader's copy) leader MMA warp + peer producer + both CTAs' epilogue warps have read
-            ptx::mbar_init(B.q_empty(q), 2 + 2 * kEpiWarps);
+            ptx::mbar_init(B.q_full(q), 1);  // the cluster's scheduler (in CTA 0) publishes
+            // (CTA 0's copy is used) every consuming role of the cluster has read: all producers,
+            // the pair leaders' MMA warps and all epilogue warps
+            ptx::mbar_init(B.q_empty(q), kCtas + kCtas / 2 + kCtas * kEpiWarps);
         }
+        ptx::mbar_init(B.q_taken(), 1);  // CTA 0's producer took an item (CTA 0's copy is used)
         *abort_flag = 0;
         ptx::fence_barrier_init();
     }
@@ -96,65 +113,62 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
     }
     ptx::tc_fence_before();
     __syncthreads();
-    ptx::cluster_sync();  // the peer's barriers are initialised before anyone signals them
+    ptx::cluster_sync();  // every CTA's barriers are initialised before anyone signals them
     ptx::tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
-    ptx::pdl_wait();  // on-chip set-up above overlaps the previous kernel; global memory only after it
 
     ItemSource src;
-    worker_items(p, blockIdx.x / 2, gridDim.x / 2, src.first, src.end, src.step);
+    worker_items(p, blockIdx.x / kCtas, gridDim.x / kCtas, src.first, src.end, src.step);
+    src.worker = blockIdx.x / kCtas;
+    src.workers = gridDim.x / kCtas;
     src.dynamic = p.dynamic;
     src.q_full0 = B.q_full(0);
     src.q_empty0 = ptx::map_to_cta(B.q_empty(0), 0);
-    src.q_item = reinterpret_cast<volatile int*>(smem + L::kQueueOffset);
+    src.q_entry = reinterpret_cast<volatile int*>(smem + L::kQueueOffset);
+    // CTA 0's scheduler deals the cluster's items; the first needs no global
+    // memory, so it is decoded and published before the wait below
+    const bool sched_thread = (rank == 0 && warp == scheduler_warp(BN) && lane == 0);
+    int item0 = -1;
+    if (sched_thread) {
+        item0 = sched_next(src, 0, p);
+        sched_publish(src, 0, item0, p, kCtas);
+    }
+    ptx::pdl_wait();  // on-chip set-up above overlaps the previous kernel; global memory only after it
 
     if (warp == 0) {
-        // ------------------------------------------------ TMA producer (both CTAs)
+        // ----------------------------------------------- TMA producer (every CTA)
         if (lane == 0) {
-            int stage = 0;
-            uint32_t phase = 0;
             int64_t issued = 0;
-            bool ok = true;
-            const uint32_t peer_q_item0 = ptx::map_to_cta(ptx::smem_addr(smem + L::kQueueOffset), 1);
-            const uint32_t peer_q_full0 = ptx::map_to_cta(B.q_full(0), 1);
-            for (int j = 0; ok; ++j) {
-                // the leader takes the next item and hands it to both CTAs; the peer reads its queue
-                const int64_t it = leader ? src_fetch(src, j, p, abort_flag, true, peer_q_item0, peer_q_full0)
-                                          : src_get(src, j, abort_flag, p.timeout_ns);
-                if (it < 0) {
-                    ok = (it == -1);
-                    break;
-                }
-                const WorkItem w = item_at(it, j, p);
-                const int32_t a_row = w.tm * kPairBM + static_cast<int32_t>(rank) * 128;
-                const int32_t b_col = w.tn * BN + static_cast<int32_t>(rank) * kHalfN;
-                for (int q = 0; q < w.k1 - w.k0; ++q) {
-                    const int kt = slab_at(w, q);
-                    if (!wait_bounded(B.empty(stage), phase ^ 1u, abort_flag, p.timeout_ns, kWaitProducerEmpty)) {
-                        ok = false;
-                        break;
-                    }
-                    if (leader) ptx::mbar_arrive_expect_tx(B.full(stage), 2 * S::kBytes);
-                    const uint32_t leader_full = ptx::map_to_cta(B.full(stage), 0);
-                    const uint32_t sa = ring + stage * S::kBytes;
-                    const uint32_t sb = sa + S::kABytes;
-                    ptx::tma_load_2d_pair(sa, &tmap_a, leader_full, kt * kBK, a_row);
+            bool ok = produce<STAGES>(src, p, B, abort_flag, /*signal_taken=*/rank == 0, issued,
+                                      [&](const WorkItem& w, int kt, int stage) {
+                const int32_t a_row = w.tm * kItemRows + static_cast<int32_t>(pair_idx * kPairBM + r * 128);
+                const int32_t b_col = w.tn * BN + static_cast<int32_t>(r) * kHalfN;
+                if (leader) ptx::mbar_arrive_expect_tx(B.full(stage), 2 * S::kBytes);
+                const uint32_t leader_full = ptx::map_to_cta(B.full(stage), pair_leader);
+                const uint32_t sa = ring + stage * S::kBytes;
+                const uint32_t sb = sa + S::kABytes;
+                ptx::tma_load_2d_pair(sa, &tmap_a, leader_full, kt * kBK, a_row);
+                if constexpr (QUAD) {
+                    // the same B half-slab goes to this CTA and its counterpart in the
+                    // other pair: each loads 32 of the 64 K rows for both
+                    const uint16_t mask = static_cast<uint16_t>((1u << r) | (1u << (r + 2)));
 #pragma unroll
-                    for (int j = 0; j < kHalfN / kBBox; ++j)
-                        ptx::tma_load_2d_pair(sb + j * (kBBox * kBK * 2), &tmap_b, leader_full, b_col + j * kBBox,
+                    for (int jb = 0; jb < kHalfN / kBBox; ++jb)
+                        ptx::tma_load_2d_pair_multicast(sb + jb * (kBBox * kBK * 2) + pair_idx * (32 * 128),
+                                                        &tmap_b, leader_full, b_col + jb * kBBox,
+                                                        kt * kBK + static_cast<int32_t>(pair_idx) * 32, mask);
+                } else {
+#pragma unroll
+                    for (int jb = 0; jb < kHalfN / kBBox; ++jb)
+                        ptx::tma_load_2d_pair(sb + jb * (kBBox * kBK * 2), &tmap_b, leader_full, b_col + jb * kBBox,
                                               kt * kBK);
-                    ++issued;
-                    if (++stage == STAGES) {
-                        stage = 0;
-                        phase ^= 1u;
-                    }
                 }
-            }
+            });
             // Tail: on success wait until the last STAGES issues are released
-            // (no commit may land after exit).  After a failure the leader waits
-            // (bounded) on its full barriers, which count both CTAs' bytes; the
-            // peer cannot observe the leader's barriers and waits a fixed 2 ms,
-            // far beyond the latency of a tile load.
+            // (no commit may land after exit).  After a failure a pair leader waits
+            // (bounded) on its full barriers, which count all its pair's bytes;
+            // the other CTA cannot observe them and waits a fixed 2 ms, far beyond
+            // the latency of a tile load.
             const int64_t n0 = issued > STAGES ? issued - STAGES : 0;
             for (int64_t n = n0; n < issued && ok; ++n)
                 ok = wait_bounded(B.empty(static_cast<int>(n % STAGES)), static_cast<uint32_t>((n / STAGES) & 1),
@@ -172,7 +186,7 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
             }
         }
     } else if (warp == 1) {
-        // ------------------------------------------------ MMA issuer (leader CTA)
+        // ------------------------------------------ MMA issuer (each pair's leader)
         if (lane == 0 && leader) {
             int stage = 0;
             uint32_t phase = 0;
@@ -181,12 +195,12 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
             bool ok = true;
             if (p.debug_never) ok = wait_bounded(B.never(), 0, abort_flag, p.timeout_ns, kWaitDebugNever);
             for (int j = 0; ok; ++j) {
-                const int64_t it = src_get(src, j, abort_flag, p.timeout_ns);
+                WorkItem w;
+                const int64_t it = src_take(src, j, p, abort_flag, w);
                 if (it < 0) {
                     ok = (it == -1);
                     break;
                 }
-                const WorkItem w = item_at(it, j, p);
                 const int nch = num_chunks(w, p.kc);
                 for (int ck = 0; ok && ck < nch; ++ck) {
                     const int kb = chunk_begin(w, ck, nch), ke = chunk_begin(w, ck + 1, nch);
@@ -213,14 +227,16 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
                                 ptx::smem_desc_sw128(sb + kk * (kUmmaK * 128), kBBox * kBK * 2, 1024);
                             ptx::tc_mma_f16_pair(d_tmem, adesc, bdesc, kIdesc, (q > kb || kk > 0) ? 1u : 0u);
                         }
-                        ptx::tc_commit_pair_multicast(B.empty(stage), kBothCtas);
+                        // the stage is free in every CTA whose smem this pair read (and, with
+                        // QUAD, whose producer also wrote into this pair's smem)
+                        ptx::tc_commit_pair_multicast(B.empty(stage), stage_mask);
                         if (++stage == STAGES) {
                             stage = 0;
                             phase ^= 1u;
                         }
                     }
                     if (!ok) break;
-                    ptx::tc_commit_pair_multicast(B.acc_full(acc), kBothCtas);
+                    ptx::tc_commit_pair_multicast(B.acc_full(acc), pair_mask);
                     if (++acc == 2) {
                         acc = 0;
                         acc_phase ^= 1u;
@@ -232,17 +248,20 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
                 wait_bounded(B.drain(), 0, abort_flag, p.timeout_ns, kWaitDrain, /*honour_abort=*/false);
             }
         }
-    } else {
-        run_epilogue<BN, OutT, true>(p, B, tmem_base, abort_flag, src, kPairBM,
-                                     static_cast<int>(rank) * 128, warp, lane, &tmap_c, smem + L::kStagingOffset);
+    } else if (warp < scheduler_warp(BN)) {
+        run_epilogue<BN, OutT, true>(p, B, tmem_base, abort_flag, src, kItemRows,
+                                     static_cast<int>(pair_idx * kPairBM + r * 128), warp, lane, &tmap_c,
+                                     smem + L::kStagingOffset, pair_leader);
+    } else if (sched_thread) {
+        // -------------------------------------------------------- scheduler
+        run_scheduler(src, item0, p, B, abort_flag, kCtas);
     }
 
     ptx::tc_fence_before();
     __syncthreads();
-    ptx::cluster_sync();  // no CTA leaves while its peer may still signal it
+    ptx::cluster_sync();  // no CTA leaves while another CTA of the cluster may still signal it
     ptx::tc_fence_after();
     if (warp == 1) ptx::tmem_dealloc_pair(tmem_base, kTmemCols);
-    if (threadIdx.x == 0) sched_release(p);
 }
 
 }  // namespace sfc
