@@ -203,9 +203,35 @@ __device__ __forceinline__ void st_shared_cluster(uint32_t cluster_addr, int v) 
     asm volatile("st.shared::cluster.s32 [%0], %1;" ::"r"(cluster_addr), "r"(v) : "memory");
 }
 
-// Arrive on an mbarrier that may live in another CTA of the cluster.
+// Arrive on an mbarrier that may live in another CTA of the cluster, releasing
+// this thread's earlier writes at cluster scope: for publishing data that the
+// waiting side reads (e.g. after st.shared::cluster into the peer's memory).
 __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
     asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
+// Send 16 bytes into a peer CTA's shared memory; the peer's mbarrier counts
+// the bytes on arrival (complete_tx), which also makes them visible to threads
+// that observe the barrier's phase.  Pair with mbar_expect_tx_remote.
+__device__ __forceinline__ void st_async_v4(uint32_t cluster_dst, const int (&v)[4], uint32_t cluster_bar) {
+    asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.s32 [%0], {%1, %2, %3, %4}, [%5];"
+                 ::"r"(cluster_dst), "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(cluster_bar)
+                 : "memory");
+}
+
+// Arrive on a (possibly remote) mbarrier announcing `bytes` of st.async data.
+__device__ __forceinline__ void mbar_expect_tx_remote(uint32_t cluster_bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.relaxed.cluster.shared::cluster.b64 _, [%0], %1;" ::"r"(cluster_bar),
+                 "r"(bytes)
+                 : "memory");
+}
+
+// Arrive on an mbarrier that may live in another CTA of the cluster with the
+// default (CTA-scope) release: for a consumer handing a buffer back after its
+// reads have completed (queue slots, tensor-memory accumulators).  The
+// cluster-scope release above costs several hundred nanoseconds on each call.
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
+    asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
 
 __device__ __forceinline__ void cluster_sync() {

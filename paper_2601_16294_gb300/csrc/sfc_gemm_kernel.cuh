@@ -174,6 +174,25 @@ __device__ __forceinline__ bool wait_bounded(uint32_t bar, uint32_t parity, vola
     }
 }
 
+// wait_bounded for roles that wait long and can answer late (the epilogue,
+// the scheduler): sleeps between polls, so that idle warps neither take issue
+// slots from the producer and MMA warps nor burn power spinning.
+__device__ __forceinline__ bool wait_bounded_idle(uint32_t bar, uint32_t parity, volatile int* abort_flag,
+                                                  uint64_t limit_ns, unsigned int site, unsigned int sleep_ns) {
+    if (ptx::mbar_try_wait(bar, parity)) return true;
+    const uint64_t t0 = ptx::global_timer_ns();
+    for (;;) {
+        __nanosleep(sleep_ns);
+        if (ptx::mbar_try_wait(bar, parity)) return true;
+        if (*abort_flag) return false;
+        if (ptx::global_timer_ns() - t0 > limit_ns) {
+            *abort_flag = 1;
+            atomicOr(&g_sfc_status, 1u | site);
+            return false;
+        }
+    }
+}
+
 template <typename OutT>
 __device__ __forceinline__ OutT cvt_out(float v);
 template <>
@@ -264,7 +283,7 @@ __device__ __forceinline__ int64_t src_take(const ItemSource& S, int j, const Ge
     w.tm = S.q_entry[4 * q + 1];
     w.tn = S.q_entry[4 * q + 2];
     w.layer = S.q_entry[4 * q + 3];
-    ptx::mbar_arrive_cluster(S.q_empty0 + 8u * q);  // slot free once every consumer has read it
+    ptx::mbar_arrive_remote(S.q_empty0 + 8u * q);  // slot free once every consumer has read it
     w.k0 = layer_k0(w.layer, p);
     w.k1 = layer_k0(w.layer + 1, p);
     w.rev = p.serpentine ? (j & 1) : 0;
@@ -285,12 +304,12 @@ __device__ __forceinline__ void sched_publish(const ItemSource& S, int j, int it
 #pragma unroll
     for (int k = 0; k < 4; ++k) S.q_entry[4 * q + k] = e[k];
     ptx::mbar_arrive(S.q_full0 + 8u * q);
+    // the peers get the entry by st.async, counted as 16 bytes by their q_full
     const uint32_t mine = ptx::smem_addr(const_cast<int*>(S.q_entry) + 4 * q);
     for (int r = 1; r < n_ctas; ++r) {
-        const uint32_t dst = ptx::map_to_cta(mine, r);
-#pragma unroll
-        for (int k = 0; k < 4; ++k) ptx::st_shared_cluster(dst + 4u * k, e[k]);
-        ptx::mbar_arrive_cluster(ptx::map_to_cta(S.q_full0 + 8u * q, r));
+        const uint32_t rbar = ptx::map_to_cta(S.q_full0 + 8u * q, r);
+        ptx::mbar_expect_tx_remote(rbar, 16);
+        ptx::st_async_v4(ptx::map_to_cta(mine, r), e, rbar);
     }
 }
 
@@ -315,10 +334,10 @@ __device__ __forceinline__ bool run_scheduler(const ItemSource& S, int item0, co
                                               volatile int* abort_flag, int n_ctas) {
     bool ok = true;
     for (int j = 1; ok && item0 >= 0; ++j) {
-        if (!wait_bounded(B.q_taken(), static_cast<uint32_t>((j - 1) & 1), abort_flag, p.timeout_ns,
-                          kWaitQueueEmpty) ||
-            !wait_bounded(S.q_empty0 + 8u * (j % kQueue), static_cast<uint32_t>(((j / kQueue) & 1) ^ 1), abort_flag,
-                          p.timeout_ns, kWaitQueueEmpty)) {
+        if (!wait_bounded_idle(B.q_taken(), static_cast<uint32_t>((j - 1) & 1), abort_flag, p.timeout_ns,
+                               kWaitQueueEmpty, 256) ||
+            !wait_bounded_idle(S.q_empty0 + 8u * (j % kQueue), static_cast<uint32_t>(((j / kQueue) & 1) ^ 1),
+                               abort_flag, p.timeout_ns, kWaitQueueEmpty, 256)) {
             ok = false;
             break;
         }
@@ -436,7 +455,7 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
         for (int ck = 0; ck < nch; ++ck) {
             int ready = 1;
             if (lane == 0)
-                ready = wait_bounded(B.acc_full(acc), acc_phase, abort_flag, p.timeout_ns, kWaitEpiAccFull);
+                ready = wait_bounded_idle(B.acc_full(acc), acc_phase, abort_flag, p.timeout_ns, kWaitEpiAccFull, 256);
             ready = __shfl_sync(0xffffffffu, ready, 0);
             if (!ready) {
                 ok = false;
@@ -458,7 +477,7 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
             __syncwarp();
             if (lane == 0) {
                 // the accumulator-empty barriers are 8 bytes apart
-                if (PAIR) ptx::mbar_arrive_cluster(acce_target + 8u * acc);
+                if (PAIR) ptx::mbar_arrive_remote(acce_target + 8u * acc);
                 else ptx::mbar_arrive(B.acc_empty(acc));
             }
             if (++acc == 2) {
