@@ -290,17 +290,26 @@ __device__ __forceinline__ int64_t src_take(const ItemSource& S, int j, const Ge
     return item;
 }
 
-// Scheduler: decode item j and publish it to slot j % kQueue of this CTA's
-// queue and of the other n_ctas - 1 CTAs of the cluster (the slot is free).
-__device__ __forceinline__ void sched_publish(const ItemSource& S, int j, int item, const GemmParams& p, int n_ctas) {
-    const int q = j % kQueue;
-    int e[4] = {item, 0, 0, 0};
+// Scheduler: the queue entry of an item (decoded tile and K layer).
+struct QueueEntry {
+    int e[4];
+};
+__device__ __forceinline__ QueueEntry sched_entry(int item, const GemmParams& p) {
+    QueueEntry x{{item, 0, 0, 0}};
     if (item >= 0) {
         const WorkItem w = decode_item(item, p);
-        e[1] = w.tm;
-        e[2] = w.tn;
-        e[3] = w.layer;
+        x.e[1] = w.tm;
+        x.e[2] = w.tn;
+        x.e[3] = w.layer;
     }
+    return x;
+}
+
+// Scheduler: publish entry x as item j, to slot j % kQueue of this CTA's queue
+// and of the other n_ctas - 1 CTAs of the cluster (the slot is free).
+__device__ __forceinline__ void sched_send(const ItemSource& S, int j, const QueueEntry& x, int n_ctas) {
+    const int q = j % kQueue;
+    const int(&e)[4] = x.e;
 #pragma unroll
     for (int k = 0; k < 4; ++k) S.q_entry[4 * q + k] = e[k];
     ptx::mbar_arrive(S.q_full0 + 8u * q);
@@ -342,7 +351,7 @@ __device__ __forceinline__ bool run_scheduler(const ItemSource& S, int item0, co
             break;
         }
         const int item = sched_next(S, j, p);
-        sched_publish(S, j, item, p, n_ctas);
+        sched_send(S, j, sched_entry(item, p), n_ctas);
         if (item < 0) break;
     }
     if (S.dynamic) {
@@ -555,6 +564,24 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
     const int warp = threadIdx.x / 32;
     const int lane = threadIdx.x % 32;
 
+    ItemSource src;
+    worker_items(p, blockIdx.x, gridDim.x, src.first, src.end, src.step);
+    src.worker = blockIdx.x;
+    src.workers = gridDim.x;
+    src.dynamic = p.dynamic;
+    src.q_full0 = B.q_full(0);
+    src.q_empty0 = B.q_empty(0);
+    src.q_entry = reinterpret_cast<volatile int*>(smem + L::kQueueOffset);
+    // the first item needs no memory at all: the scheduler decodes it while
+    // the other warps set up, and publishes it before the wait for the previous grid
+    const bool sched_thread = (warp == scheduler_warp(BN) && lane == 0);
+    int item0 = -1;
+    QueueEntry entry0{};
+    if (sched_thread) {
+        item0 = sched_next(src, 0, p);
+        entry0 = sched_entry(item0, p);
+    }
+
     if (threadIdx.x == 0) {
         ptx::pdl_launch_dependents();
         for (int s = 0; s < STAGES; ++s) {
@@ -588,22 +615,7 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
-
-    ItemSource src;
-    worker_items(p, blockIdx.x, gridDim.x, src.first, src.end, src.step);
-    src.worker = blockIdx.x;
-    src.workers = gridDim.x;
-    src.dynamic = p.dynamic;
-    src.q_full0 = B.q_full(0);
-    src.q_empty0 = B.q_empty(0);
-    src.q_entry = reinterpret_cast<volatile int*>(smem + L::kQueueOffset);
-    // the first item needs no global memory: decode and publish it before the wait below
-    const bool sched_thread = (warp == scheduler_warp(BN) && lane == 0);
-    int item0 = -1;
-    if (sched_thread) {
-        item0 = sched_next(src, 0, p);
-        sched_publish(src, 0, item0, p, 1);
-    }
+    if (sched_thread) sched_send(src, 0, entry0, 1);
     ptx::pdl_wait();  // on-chip set-up above overlaps the previous kernel; global memory only after it
 
     if (warp == 0) {

@@ -79,6 +79,24 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
     const bool leader = (r == 0);
     const uint16_t pair_mask = static_cast<uint16_t>(0x3u << (2 * pair_idx));
     const uint16_t stage_mask = QUAD ? 0xF : 0x3;  // CTAs whose smem a stage's loads write
+    ItemSource src;
+    worker_items(p, blockIdx.x / kCtas, gridDim.x / kCtas, src.first, src.end, src.step);
+    src.worker = blockIdx.x / kCtas;
+    src.workers = gridDim.x / kCtas;
+    src.dynamic = p.dynamic;
+    src.q_full0 = B.q_full(0);
+    src.q_empty0 = ptx::map_to_cta(B.q_empty(0), 0);
+    src.q_entry = reinterpret_cast<volatile int*>(smem + L::kQueueOffset);
+    // CTA 0's scheduler deals the cluster's items.  The first needs no memory
+    // at all: it is decoded while the other warps set up and published before
+    // the wait for the previous grid.
+    const bool sched_thread = (rank == 0 && warp == scheduler_warp(BN) && lane == 0);
+    int item0 = -1;
+    QueueEntry entry0{};
+    if (sched_thread) {
+        item0 = sched_next(src, 0, p);
+        entry0 = sched_entry(item0, p);
+    }
 
     if (threadIdx.x == 0) {
         ptx::pdl_launch_dependents();
@@ -117,22 +135,7 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
     ptx::tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
 
-    ItemSource src;
-    worker_items(p, blockIdx.x / kCtas, gridDim.x / kCtas, src.first, src.end, src.step);
-    src.worker = blockIdx.x / kCtas;
-    src.workers = gridDim.x / kCtas;
-    src.dynamic = p.dynamic;
-    src.q_full0 = B.q_full(0);
-    src.q_empty0 = ptx::map_to_cta(B.q_empty(0), 0);
-    src.q_entry = reinterpret_cast<volatile int*>(smem + L::kQueueOffset);
-    // CTA 0's scheduler deals the cluster's items; the first needs no global
-    // memory, so it is decoded and published before the wait below
-    const bool sched_thread = (rank == 0 && warp == scheduler_warp(BN) && lane == 0);
-    int item0 = -1;
-    if (sched_thread) {
-        item0 = sched_next(src, 0, p);
-        sched_publish(src, 0, item0, p, kCtas);
-    }
+    if (sched_thread) sched_send(src, 0, entry0, kCtas);
     ptx::pdl_wait();  // on-chip set-up above overlaps the previous kernel; global memory only after it
 
     if (warp == 0) {
