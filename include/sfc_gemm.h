@@ -114,8 +114,10 @@ int sfc_tile_order_device(int Mt, int Nt, int32_t *out_idx_dev, void *stream);
 /*
  * sfc_gemm_workspace_size -- bytes of fp32 workspace sfc_gemm_ex needs for the
  * ca_c partial copies of C (Listing 1's C[K_layers][...], Sec. II-D):
- * 0 when ca_c == 1, else ca_c * M * round_up(N, 4) * 4.  Returns 0 for invalid
- * arguments.
+ * 0 when ca_c == 1, else ca_c * M * round_up(N, 4) * 4.  For ca_c == 0 (layer
+ * count chosen by the library) the size for the most layers it may choose,
+ * min(64, ceil(K/64), ceil(320 / (ceil(M/128) * ceil(N/128)))).  Returns 0 for
+ * invalid arguments.  Needs no GPU.
  */
 size_t sfc_gemm_workspace_size(int64_t M, int64_t N, int64_t K, int ca_c);
 
@@ -128,7 +130,11 @@ size_t sfc_gemm_workspace_size(int64_t M, int64_t N, int64_t K, int ca_c);
  *         tiles [floor(l*Kt/ca_c), floor((l+1)*Kt/ca_c)) of the Kt = ceil(K/64)
  *         64-wide K tiles.  For ca_c > 1 the library takes its fp32 workspace
  *         from a stream-ordered pool (cudaMallocAsync / cudaFreeAsync on
- *         `stream`).
+ *         `stream`).  ca_c = 0 lets the library choose the count (and the
+ *         tile) from a model of the call's time on this device: waves of
+ *         items times the length of a layer, plus the reduction's cost for
+ *         more than one layer (the replication factor choice of Sec. II-D,
+ *         made per call); sfc_gemm_plan reports the choice.
  *   stream: a cudaStream_t passed as void*.
  * Requirements: A and B 16-byte aligned, lda and ldb multiples of 8 (the tile
  * loads use the Tensor Memory Accelerator).  C may have any alignment.
@@ -162,6 +168,25 @@ int sfc_gemm_ex(int64_t M, int64_t N, int64_t K,
                 int ca_c, sfc_dtype_t c_dtype,
                 sfc_order_t order, sfc_assign_t assign, sfc_tile_t tile,
                 void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ * sfc_gemm_plan -- the tile and K-layer count sfc_gemm_ex would use for these
+ * arguments on the current device (ca_c = 0: the library's choice; ca_c >= 1:
+ * that count with the tile AUTO or `tile` picks).  No kernel runs.
+ *   out_tile: an sfc_tile_t other than SFC_TILE_AUTO.  out_ca_c: >= 1.
+ * Errors: SFC_ERR_INVALID_ARG (as sfc_gemm_ex, or a NULL output pointer),
+ * SFC_ERR_CUDA, SFC_ERR_UNSUPPORTED.
+ */
+int sfc_gemm_plan(int64_t M, int64_t N, int64_t K, int ca_c, int c_dtype, int tile,
+                  int *out_tile, int *out_ca_c);
+
+/*
+ * sfc_release -- returns to the driver the device memory the library's
+ * stream-ordered workspace allocations left cached in the current device's
+ * default memory pool (synchronizes the device first).  The library keeps no
+ * other allocation between calls.  SFC_OK, or SFC_ERR_CUDA.
+ */
+int sfc_release(void);
 
 /*
  * sfc_get_device_status -- synchronizes `stream`, then returns and clears the

@@ -31,7 +31,7 @@ TILES = {0: 0, "auto": 0, 128: 128, 256: 256, "pair128": 1128, "pair256": 1256, 
 
 EXPORTS = ("sfc_tile_order", "sfc_tile_order_device", "sfc_gemm_workspace_size", "sfc_gemm", "sfc_gemm_ex",
            "sfc_get_device_status", "sfc_last_cuda_error", "sfc_num_workers", "sfc_debug_force_timeout",
-           "sfc_gemm_noalloc")
+           "sfc_gemm_noalloc", "sfc_gemm_plan", "sfc_release")
 NOALLOC_SCRATCH_BYTES = 32 << 20
 
 
@@ -80,6 +80,8 @@ def load():
         lib.sfc_num_workers.argtypes = []
         lib.sfc_debug_force_timeout.argtypes = [vp, vp, vp, i32, vp]
         lib.sfc_gemm_noalloc.argtypes = [i64, i64, i64, vp, vp, vp, i64, i64, i64, i32, i32, vp]
+        lib.sfc_gemm_plan.argtypes = [i64, i64, i64, i32, i32, i32, vp, vp]
+        lib.sfc_release.argtypes = []
         for name in EXPORTS:
             if name != "sfc_gemm_workspace_size":
                 getattr(lib, name).restype = ctypes.c_int
@@ -123,6 +125,24 @@ def workspace_size(M: int, N: int, K: int, ca_c: int) -> int:
     return int(load().sfc_gemm_workspace_size(int(M), int(N), int(K), int(ca_c)))
 
 
+def plan(M: int, N: int, K: int, ca_c: int = 0, out_dtype=None, tile="auto"):
+    """(tile, ca_c) the library would use for this call on the current device;
+    tile is a key of TILES other than "auto"."""
+    import torch
+    t = ctypes.c_int(0)
+    c = ctypes.c_int(0)
+    dt = SFC_BF16 if out_dtype == torch.bfloat16 else SFC_F32
+    _check(load().sfc_gemm_plan(int(M), int(N), int(K), int(ca_c), dt, TILES[tile], ctypes.byref(t),
+                                ctypes.byref(c)), "sfc_gemm_plan")
+    name = {v: k for k, v in TILES.items() if k not in (0, "auto")}[t.value]
+    return name, c.value
+
+
+def release() -> None:
+    """Give the memory cached by the library's workspace allocations back to the driver."""
+    _check(load().sfc_release(), "sfc_release")
+
+
 def num_workers() -> int:
     n = load().sfc_num_workers()
     if n < 0:
@@ -140,8 +160,8 @@ def gemm(A, B, C=None, *, ca_c: int = 1, out_dtype=None, order: str = "sfc", ass
          tile=0, workspace=None, stream=None):
     """C = A @ B on the GPU.  A: (M, K) bf16, B: (K, N) bf16, both CUDA, row-major
     (row strides may be padded).  C: (M, N) fp32 or bf16 CUDA tensor, allocated
-    if not given.  ``workspace``: optional CUDA tensor of at least
-    ``workspace_size(M, N, K, ca_c)`` bytes."""
+    if not given.  ``ca_c``: K layers (0: the library chooses).  ``workspace``:
+    optional CUDA tensor of at least ``workspace_size(M, N, K, ca_c)`` bytes."""
     import torch
     lib = load()
     M, K = A.shape

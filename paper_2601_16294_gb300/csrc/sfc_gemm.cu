@@ -251,33 +251,75 @@ int make_out_map(CUtensorMap* map, const void* ptr, int64_t rows, int64_t cols, 
 
 int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
-// Tile shape for a call.  AUTO estimates each variant's time as
-// (waves of items) x (per-SM work of one item) / (its relative efficiency) and
-// takes the fastest; 2-SM pairs move half the B bytes per flop of one SM.
-int pick_variant(int64_t M, int64_t N, int ca_c, const DeviceInfo& d, sfc_tile_t tile) {
+// Planning a call: the tile variant and, when the caller asks for it
+// (ca_c = 0), the number of K layers.  The estimate of a (variant, c) pair is
+//   waves x (slabs of the longest layer) x (time of one slab on one worker)
+//   + for c > 1: the reduction's launch and its partial traffic (c fp32
+//     copies of C written and read back, C written once),
+// where waves = ceil(tiles x c / workers) and a slab's time is a 128 x bn x 64
+// block at the variant's measured tensor-pipe efficiency.  It reproduces the
+// best measured c on the high-K and prefill shapes (GB300, 152 SMs).
+constexpr double kSlabClockGhz = 1.9;        // SM clock the slab times assume
+constexpr double kReduceLaunchNs = 3000.0;   // reduction kernel launch and ramp
+constexpr double kPartialBytesPerNs = 6000.0;
+// relative tensor-pipe efficiency measured on GB300 (256-wide tiles feed the
+// tensor core with fewer shared-memory bytes per flop)
+constexpr double kEff[kNumVariants] = {0.50, 0.85, 0.55, 0.95, 0.90};
+
+// Layers ca_c = 0 may choose: enough to give about 320 items of 128 x 128,
+// never more than 64 or the number of K slabs (host-only, so the workspace
+// bound below needs no device).
+int64_t auto_layer_cap(int64_t M, int64_t N, int64_t K) {
+    const int64_t tiles = ceil_div(M, kBM) * ceil_div(N, 128);
+    int64_t cap = ceil_div(320, tiles);
+    const int64_t Kt = ceil_div(K, kBK);
+    if (cap > Kt) cap = Kt;
+    if (cap > 64) cap = 64;
+    return cap < 1 ? 1 : cap;
+}
+
+double plan_cost(int64_t M, int64_t N, int64_t K, int c, int v, const DeviceInfo& d, int out_bytes) {
+    const int64_t items = ceil_div(M, variant_bm(v)) * ceil_div(N, variant_bn(v)) * c;
+    const int64_t waves = ceil_div(items, d.workers[v]);
+    const int64_t slabs = ceil_div(ceil_div(K, kBK), c);
+    const double slab_ns = 128.0 * variant_bn(v) * kBK * 2.0 / (8192.0 * kEff[v]) / kSlabClockGhz;
+    double t = static_cast<double>(waves) * static_cast<double>(slabs) * slab_ns;
+    if (c > 1)
+        t += kReduceLaunchNs + (8.0 * c + out_bytes) * static_cast<double>(M) * static_cast<double>(N) /
+                                   kPartialBytesPerNs;
+    return t;
+}
+
+struct Plan {
+    int v;
+    int c;
+};
+
+// ca_c >= 1: the variant for it; ca_c = 0: the best (variant, c) with c up to
+// max_c.  A requested tile fixes the variant (falling back to one SM when
+// pairs cannot be co-scheduled).
+Plan make_plan(int64_t M, int64_t N, int64_t K, int ca_c, int max_c, const DeviceInfo& d, sfc_tile_t tile,
+               int out_bytes) {
+    int fixed = -1;
     switch (tile) {
-        case SFC_TILE_N128: return kSingle128;
-        case SFC_TILE_N256: return kSingle256;
-        case SFC_TILE_PAIR_N128: return d.workers[kPair128] > 0 ? kPair128 : kSingle128;
-        case SFC_TILE_PAIR_N256: return d.workers[kPair256] > 0 ? kPair256 : kSingle256;
-        case SFC_TILE_QUAD_N256: return d.workers[kQuad256] > 0 ? kQuad256 : kSingle256;
+        case SFC_TILE_N128: fixed = kSingle128; break;
+        case SFC_TILE_N256: fixed = kSingle256; break;
+        case SFC_TILE_PAIR_N128: fixed = d.workers[kPair128] > 0 ? kPair128 : kSingle128; break;
+        case SFC_TILE_PAIR_N256: fixed = d.workers[kPair256] > 0 ? kPair256 : kSingle256; break;
+        case SFC_TILE_QUAD_N256: fixed = d.workers[kQuad256] > 0 ? kQuad256 : kSingle256; break;
         default: break;
     }
-    // relative tensor-pipe efficiency measured on GB300 (256-wide tiles feed the
-    // tensor core with fewer shared-memory bytes per flop)
-    static const double eff[kNumVariants] = {0.50, 0.85, 0.55, 0.95, 0.90};
-    int best = kSingle128;
-    double best_t = 0.0;
+    Plan best{fixed >= 0 ? fixed : kSingle128, ca_c > 0 ? ca_c : 1};
+    double best_t = -1.0;
+    const int c_lo = ca_c > 0 ? ca_c : 1, c_hi = ca_c > 0 ? ca_c : max_c;
     for (int v = 0; v < kNumVariants; ++v) {
-        if (d.workers[v] <= 0) continue;
-        const int bm = variant_bm(v), bn = variant_bn(v);
-        const int64_t items = ((M + bm - 1) / bm) * ((N + bn - 1) / bn) * ca_c;
-        const int64_t waves = (items + d.workers[v] - 1) / d.workers[v];
-        // per-SM work of one item is 128 x bn for every variant
-        const double t = static_cast<double>(waves) * 128.0 * bn / eff[v];
-        if (v == kSingle128 || t < best_t) {
-            best = v;
-            best_t = t;
+        if (d.workers[v] <= 0 || (fixed >= 0 && v != fixed)) continue;
+        for (int c = c_lo; c <= c_hi; ++c) {
+            const double t = plan_cost(M, N, K, c, v, d, out_bytes);
+            if (best_t < 0.0 || t < best_t) {  // ties keep fewer layers, then the earlier variant
+                best = Plan{v, c};
+                best_t = t;
+            }
         }
     }
     return best;
@@ -301,8 +343,9 @@ int validate(int64_t M, int64_t N, int64_t K, const void* A, const void* B, cons
     if (M > (int64_t(1) << 31) - kBM || N > (int64_t(1) << 31) - 256 || K > (int64_t(1) << 31) - kBK)
         return SFC_ERR_INVALID_ARG;
     const int64_t Kt = ceil_div(K, kBK);
-    if (ca_c < 1 || ca_c > Kt || ca_c > kMaxLayers) return SFC_ERR_INVALID_ARG;
-    if (ceil_div(M, kBM) * ceil_div(N, 128) * ca_c > (int64_t(1) << 31) - 1) return SFC_ERR_INVALID_ARG;
+    if (ca_c < 0 || ca_c > Kt || ca_c > kMaxLayers) return SFC_ERR_INVALID_ARG;  // 0: chosen per call
+    const int64_t layers = ca_c > 0 ? ca_c : auto_layer_cap(M, N, K);
+    if (ceil_div(M, kBM) * ceil_div(N, 128) * layers > (int64_t(1) << 31) - 1) return SFC_ERR_INVALID_ARG;
     if (!aligned16(A) || !aligned16(B) || (lda % 8) != 0 || (ldb % 8) != 0) return SFC_ERR_UNALIGNED;
     if (lda >= (int64_t(1) << 39) || ldb >= (int64_t(1) << 39)) return SFC_ERR_INVALID_ARG;
     return SFC_OK;
@@ -324,15 +367,20 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
              size_t workspace_bytes, cudaStream_t stream, int debug_never, uint64_t timeout_ns) {
     int rc = validate(M, N, K, A, B, C, lda, ldb, ldc, ca_c, c_dtype, order, assign, tile);
     if (rc != SFC_OK) return rc;
-    const size_t ws_need = sfc_gemm_workspace_size(M, N, K, ca_c);
-    if (workspace && workspace_bytes < ws_need) return SFC_ERR_WORKSPACE;
+    if (ca_c > 0 && workspace && workspace_bytes < sfc_gemm_workspace_size(M, N, K, ca_c)) return SFC_ERR_WORKSPACE;
     if (workspace && !aligned16(workspace)) return SFC_ERR_UNALIGNED;
 
     DeviceInfo* dev = nullptr;
     rc = device_setup(&dev);
     if (rc != SFC_OK) return rc;
 
-    const int v = pick_variant(M, N, ca_c, *dev, static_cast<sfc_tile_t>(tile));
+    // ca_c = 0: the planner's layer count, within the caller's workspace if one is given
+    int max_c = static_cast<int>(auto_layer_cap(M, N, K));
+    while (ca_c == 0 && workspace && max_c > 1 && workspace_bytes < sfc_gemm_workspace_size(M, N, K, max_c)) --max_c;
+    const Plan plan = make_plan(M, N, K, ca_c, max_c, *dev, static_cast<sfc_tile_t>(tile), c_dtype == SFC_F32 ? 4 : 2);
+    const int v = plan.v;
+    ca_c = plan.c;
+    const size_t ws_need = sfc_gemm_workspace_size(M, N, K, ca_c);
     const int bn = variant_bn(v);
     const int bm = variant_bm(v);
     CUtensorMap ta, tb;
@@ -459,9 +507,42 @@ SFC_API int sfc_tile_order_device(int Mt, int Nt, int32_t* out_idx_dev, void* st
 }
 
 SFC_API size_t sfc_gemm_workspace_size(int64_t M, int64_t N, int64_t K, int ca_c) {
-    if (M <= 0 || N <= 0 || K <= 0 || ca_c < 1) return 0;
-    if (ca_c == 1) return 0;
-    return static_cast<size_t>(ca_c) * static_cast<size_t>(M) * static_cast<size_t>(ws_ld(N)) * 4u;
+    if (M <= 0 || N <= 0 || K <= 0 || ca_c < 0) return 0;
+    const int64_t layers = ca_c > 0 ? ca_c : auto_layer_cap(M, N, K);  // 0: the most the planner may choose
+    if (layers == 1) return 0;
+    return static_cast<size_t>(layers) * static_cast<size_t>(M) * static_cast<size_t>(ws_ld(N)) * 4u;
+}
+
+SFC_API int sfc_gemm_plan(int64_t M, int64_t N, int64_t K, int ca_c, int c_dtype, int tile, int* out_tile,
+                          int* out_ca_c) {
+    if (!out_tile || !out_ca_c) return SFC_ERR_INVALID_ARG;
+    int rc = validate(M, N, K, reinterpret_cast<const void*>(16), reinterpret_cast<const void*>(16),
+                      reinterpret_cast<const void*>(16), K + (8 - K % 8) % 8, N + (8 - N % 8) % 8, N, ca_c,
+                      c_dtype, SFC_ORDER_SFC, SFC_ASSIGN_AUTO, tile);
+    if (rc != SFC_OK) return rc;
+    DeviceInfo* dev = nullptr;
+    rc = device_setup(&dev);
+    if (rc != SFC_OK) return rc;
+    const Plan plan = make_plan(M, N, K, ca_c, static_cast<int>(auto_layer_cap(M, N, K)), *dev,
+                                static_cast<sfc_tile_t>(tile), c_dtype == SFC_F32 ? 4 : 2);
+    static const int kTileOf[kNumVariants] = {SFC_TILE_N128, SFC_TILE_N256, SFC_TILE_PAIR_N128, SFC_TILE_PAIR_N256,
+                                              SFC_TILE_QUAD_N256};
+    *out_tile = kTileOf[plan.v];
+    *out_ca_c = plan.c;
+    return SFC_OK;
+}
+
+SFC_API int sfc_release(void) {
+    // The only memory the library holds between calls is what the device's
+    // default stream-ordered pool keeps after K-layer workspaces were freed.
+    int dev;
+    int rc = current_device(&dev);
+    if (rc != SFC_OK) return rc;
+    cudaMemPool_t pool;
+    cudaError_t e = cudaDeviceGetDefaultMemPool(&pool, dev);
+    if (e == cudaSuccess) e = cudaDeviceSynchronize();
+    if (e == cudaSuccess) e = cudaMemPoolTrimTo(pool, 0);
+    return e == cudaSuccess ? SFC_OK : cuda_fail(e);
 }
 
 SFC_API int sfc_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void* C, int64_t lda,

@@ -65,7 +65,17 @@ def test_workspace_size(lib):
     assert sfc.workspace_size(512, 512, 4096, 4) == 4 * 512 * 512 * 4
     assert sfc.workspace_size(3, 5, 64, 2) == 2 * 3 * 8 * 4          # rows padded to 4 floats
     assert sfc.workspace_size(0, 5, 64, 2) == 0
-    assert sfc.workspace_size(3, 5, 64, 0) == 0
+    assert sfc.workspace_size(3, 5, 64, -1) == 0
+
+
+def test_workspace_size_for_chosen_layers(lib):
+    # ca_c = 0: room for the most layers the planner may pick,
+    # min(64, ceil(K/64), ceil(320 / (ceil(M/128) ceil(N/128))))
+    assert sfc.workspace_size(512, 512, 32768, 0) == 20 * 512 * 512 * 4      # 16 tiles -> 20 layers
+    assert sfc.workspace_size(128, 128, 1 << 20, 0) == 64 * 128 * 128 * 4    # capped at 64
+    assert sfc.workspace_size(128, 128, 200, 0) == 4 * 128 * 128 * 4         # Kt = 4
+    assert sfc.workspace_size(4096, 4096, 4096, 0) == 0                      # 1024 tiles -> 1 layer
+    assert sfc.workspace_size(3, 5, 64, 0) == 0                              # Kt = 1
 
 
 # Fake, never-dereferenced device addresses: validation runs before any CUDA call.
@@ -90,7 +100,7 @@ def test_gemm_validation_codes(lib):
     assert call_ex(lib, C=0) == E.SFC_ERR_INVALID_ARG
     assert call_ex(lib, lda=128) == E.SFC_ERR_INVALID_ARG          # lda < K
     assert call_ex(lib, ldc=100) == E.SFC_ERR_INVALID_ARG          # ldc < N
-    assert call_ex(lib, ca_c=0) == E.SFC_ERR_INVALID_ARG
+    assert call_ex(lib, ca_c=-1) == E.SFC_ERR_INVALID_ARG
     assert call_ex(lib, K=256, ca_c=5) == E.SFC_ERR_INVALID_ARG    # Kt = 4 < ca_c
     assert call_ex(lib, K=64 * 5000, ca_c=4097) == E.SFC_ERR_INVALID_ARG  # more than 4096 layers
     assert call_ex(lib, dtype=7) == E.SFC_ERR_INVALID_ARG
@@ -121,8 +131,23 @@ def _has_gpu():
 def test_valid_call_without_gpu_fails_loudly(lib):
     rc = call_ex(lib)
     assert rc in (binding.SFC_ERR_CUDA, binding.SFC_ERR_UNSUPPORTED)
+    assert call_ex(lib, ca_c=0) in (binding.SFC_ERR_CUDA, binding.SFC_ERR_UNSUPPORTED)
     assert lib.sfc_num_workers() < 0
     assert lib.sfc_get_device_status(None) == binding.SFC_ERR_CUDA
+    assert lib.sfc_release() == binding.SFC_ERR_CUDA
+    t, c = ctypes.c_int(0), ctypes.c_int(0)
+    assert lib.sfc_gemm_plan(512, 512, 4096, 0, 0, 0, ctypes.byref(t), ctypes.byref(c)) in (
+        binding.SFC_ERR_CUDA, binding.SFC_ERR_UNSUPPORTED)
+
+
+def test_plan_validation(lib):
+    t, c = ctypes.c_int(0), ctypes.c_int(0)
+    assert lib.sfc_gemm_plan(512, 512, 4096, 0, 0, 0, None, ctypes.byref(c)) == binding.SFC_ERR_INVALID_ARG
+    assert lib.sfc_gemm_plan(0, 512, 4096, 0, 0, 0, ctypes.byref(t), ctypes.byref(c)) == binding.SFC_ERR_INVALID_ARG
+    assert lib.sfc_gemm_plan(512, 512, 4096, -2, 0, 0, ctypes.byref(t), ctypes.byref(c)) == \
+        binding.SFC_ERR_INVALID_ARG
+    assert lib.sfc_gemm_plan(512, 512, 4096, 0, 0, 77, ctypes.byref(t), ctypes.byref(c)) == \
+        binding.SFC_ERR_INVALID_ARG
 
 
 def test_missing_library_raises(monkeypatch, tmp_path):
