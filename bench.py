@@ -9,8 +9,9 @@ step's shapes, sum(2 M N K) / time, in TFLOP/s, with inputs resident in HBM.
 
 Other workloads (``--workload``) measure the remaining shape sets the same way:
 ``prefill`` (LLM-prefill projections), ``irregular`` (odd tile grids),
-``highk`` (the communication-avoiding K split), ``cube512`` (the small parity
-case).  Where a shape lists several K-layer counts, each is timed and the best
+``highk`` (the communication-avoiding K split), ``sweep125`` (the paper's
+125-shape sweep over {512..8192}^3), ``cube512`` (the small parity case).
+Where a shape lists several K-layer counts, each is timed and the best
 one is used in the step (the paper reports the best replication factor too).
 
 Prints one JSON line (rank 0).  ``--impl reference`` times the CPU oracle (the
@@ -42,8 +43,10 @@ TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic_square_sweep.json")
 CS = (1, 2, 4, 8)
 
 
-def _shape(M, N, K, kind="uniform", out="bf16", cs=(1,)):
-    return {"M": M, "N": N, "K": K, "kind": kind, "out": out, "cs": tuple(cs)}
+def _shape(M, N, K, kind="uniform", out="bf16", cs=(1,), shared=False):
+    # shared: A (M x K) and B (K x N) are drawn per operand shape, from seeds of
+    # their own, and reused by every shape of the workload that has them
+    return {"M": M, "N": N, "K": K, "kind": kind, "out": out, "cs": tuple(cs), "shared": shared}
 
 
 WORKLOADS = {
@@ -70,6 +73,12 @@ WORKLOADS = {
                 "uniform [-1,1], fp32 output, ca_c in {1,2,4,8} each timed, best in the step",
         "shapes": [_shape(m, m, k, "uniform", "f32", CS) for m in (512, 1024, 2048)
                    for k in (32768, 65536, 131072)],
+    },
+    "sweep125": {
+        "desc": "the paper's shape sweep: M, N, K each in {512, 1024, 2048, 4096, 8192} (125 shapes), uniform "
+                "[-1,1] seeded inputs, bf16 output, best ca_c in {1,2,4,8}",
+        "shapes": [_shape(m, n, k, "uniform", "bf16", CS, shared=True) for m in (512, 1024, 2048, 4096, 8192)
+                   for n in (512, 1024, 2048, 4096, 8192) for k in (512, 1024, 2048, 4096, 8192)],
     },
     "cube512": {
         "desc": "single GEMM M=N=K=512, uniform [-1,1] seed 0, fp32 output, 4x4 grid of 128x128 tiles, ca_c=1",
@@ -220,17 +229,29 @@ class ClockSampler:
 
 # ------------------------------------------------------------------- our arm
 
-def make_inputs(s, synth, torch):
-    lda = synth.pad8(s["K"])
-    ldb = synth.pad8(s["N"])
-    A, B = synth.gemm_inputs(s["M"], s["N"], s["K"], s["kind"], seed=0, lda=lda, ldb=ldb)
+_SHARED = {}
 
+
+def make_inputs(s, synth, torch):
     def dev(t):
         full = t.as_strided((t.shape[0], t.stride(0)), (t.stride(0), 1))
         return full.contiguous().cuda()[:, : t.shape[1]]
 
     out_dtype = torch.float32 if s["out"] == "f32" else torch.bfloat16
     C = torch.empty((s["M"], s["N"]), dtype=out_dtype, device="cuda")
+    if s.get("shared"):
+        def operand(rows, cols, seed):
+            key = (rows, cols, seed)
+            if key not in _SHARED:
+                t = synth.uniform_bf16((rows, cols), seed=seed)
+                _SHARED[key] = (t, dev(t))
+            return _SHARED[key]
+        A, Ad = operand(s["M"], s["K"], 1000003 * s["M"] + s["K"])
+        B, Bd = operand(s["K"], s["N"], 2000003 * s["K"] + s["N"] + 7)
+        return A, B, Ad, Bd, C
+    lda = synth.pad8(s["K"])
+    ldb = synth.pad8(s["N"])
+    A, B = synth.gemm_inputs(s["M"], s["N"], s["K"], s["kind"], seed=0, lda=lda, ldb=ldb)
     return A, B, dev(A), dev(B), C
 
 
@@ -478,10 +499,16 @@ def run_e2e(args, mats, stream, world):
     import torch
     import paper_2601_16294_gb300 as sfc
 
+    pinned = {}  # operands shared between shapes are pinned once (each shape still copies them)
+
+    def pin(t):
+        if id(t) not in pinned:
+            pinned[id(t)] = t.contiguous().pin_memory()
+        return pinned[id(t)]
+
     host = []
     for m in mats:
-        host.append((m, m["A"].contiguous().pin_memory(), m["B"].contiguous().pin_memory(),
-                     torch.empty(m["C"].shape, dtype=m["C"].dtype, pin_memory=True)))
+        host.append((m, pin(m["A"]), pin(m["B"]), torch.empty(m["C"].shape, dtype=m["C"].dtype, pin_memory=True)))
     h2d = sum(Ah.numel() * 2 + Bh.numel() * 2 for _, Ah, Bh, _ in host)
     d2h = sum(Ch.numel() * Ch.element_size() for _, _, _, Ch in host)
 

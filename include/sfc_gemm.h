@@ -54,6 +54,12 @@ typedef enum {
 
 typedef enum { SFC_F32 = 0, SFC_BF16 = 1 } sfc_dtype_t;
 
+/* Storage of B (sfc_gemm_ex2).  KN: B is K x N row-major, the paper's
+ * statement of the problem (Sec. II-A).  NK: the caller holds B transposed,
+ * N x K row-major (a linear layer's weight matrix); the kernels then load B
+ * K-major like A.  Not part of the paper, which fixes the KN layout. */
+typedef enum { SFC_B_KN = 0, SFC_B_NK = 1 } sfc_b_layout_t;
+
 /* Order of the output tiles along which workers take their items.
  * SFC:    generalized Hilbert curve (Sec. II-B) -- the method.
  * RASTER: row-major tile order s -> (s / Nt, s % Nt), a comparison baseline. */
@@ -168,6 +174,31 @@ int sfc_gemm_ex(int64_t M, int64_t N, int64_t K,
                 int ca_c, sfc_dtype_t c_dtype,
                 sfc_order_t order, sfc_assign_t assign, sfc_tile_t tile,
                 void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ * sfc_gemm_ex2 -- sfc_gemm_ex extended with the operand layout and epilogue of
+ * a BLAS-style GEMM (no counterpart in the paper, which computes C = A B with
+ * C zeroed first, Listing 1):
+ *     C = A B + beta * C + bias[j]     (fp32 arithmetic, then rounded to c_dtype)
+ *   b_layout: SFC_B_KN (B is K x N, ldb >= N) or SFC_B_NK (B is stored as its
+ *             transpose, N x K, ldb >= K).  SFC_TILE_QUAD_N256 is served by
+ *             SFC_TILE_PAIR_N256 with SFC_B_NK.
+ *   beta:     0 leaves C write-only (its contents may be anything, even NaN);
+ *             otherwise C is read once, before it is written.
+ *   bias:     NULL or N fp32 device values, 4-byte aligned, added per column.
+ * With ca_c > 1 the beta and bias terms are applied by the layer reduction,
+ * after the layer partials are summed; with ca_c == 1 by the GEMM epilogue.
+ * Other arguments, requirements and errors as sfc_gemm_ex; ldb must be a
+ * multiple of 8 in either layout, and an invalid b_layout is
+ * SFC_ERR_INVALID_ARG, a misaligned bias SFC_ERR_UNALIGNED.
+ */
+int sfc_gemm_ex2(int64_t M, int64_t N, int64_t K,
+                 const void *A, const void *B, void *C,
+                 int64_t lda, int64_t ldb, int64_t ldc,
+                 int b_layout, float beta, const float *bias,
+                 int ca_c, sfc_dtype_t c_dtype,
+                 sfc_order_t order, sfc_assign_t assign, sfc_tile_t tile,
+                 void *workspace, size_t workspace_bytes, void *stream);
 
 /*
  * sfc_gemm_plan -- the tile and K-layer count sfc_gemm_ex would use for these

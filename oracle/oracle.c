@@ -40,6 +40,12 @@
  *     this sum, so it has no separate oracle; oracle_gemm_sub_f64 takes a k
  *     range so one layer's partial product can be formed too.
  *
+ *  3. oracle_gemm_affine_f64 -- an extension beyond the paper (which zeroes C
+ *     and takes B as K x N): the BLAS-style C = A B + beta * C_in + bias[j],
+ *     with B given either K x N or transposed (N x K, a linear layer's weight
+ *     matrix).  It is written independently of part 2: one dot product per
+ *     output element (j-k loop order), then the two affine terms, in double.
+ *
  *  oracle_round_bf16 rounds a double to the nearest bf16 (ties to even) in a
  *  single step, used to compare bf16 outputs against the fp64 reference.
  */
@@ -186,6 +192,35 @@ void oracle_gemm_sub_f64(const int64_t *rows, int64_t nrows,
             double a = widen_bf16(A[rows[r] * lda + k]);
             const uint16_t *b = B + k * ldb;
             for (int64_t c = 0; c < ncols; ++c) o[c] += a * widen_bf16(b[cols[c]]);
+        }
+    }
+}
+
+/* ------------------------------------------------------------------------- */
+/* 3. GEMM with a transposed-B option and the beta / bias epilogue            */
+/* ------------------------------------------------------------------------- */
+
+/* C[i*ldc + j] = sum_k A[i][k] * B(k, j) + beta * C_in[i*ldcin + j] + bias[j],
+ * B(k, j) = B[k*ldb + j] (b_nk == 0) or B[j*ldb + k] (b_nk == 1).  C_in and
+ * bias may be NULL (terms left out). */
+void oracle_gemm_affine_f64(int64_t M, int64_t N, int64_t K,
+                            const uint16_t *A, int64_t lda,
+                            const uint16_t *B, int64_t ldb, int b_nk,
+                            double beta, const double *C_in, int64_t ldcin,
+                            const double *bias,
+                            double *C, int64_t ldc)
+{
+    #pragma omp parallel for schedule(static)
+    for (int64_t i = 0; i < M; ++i) {
+        for (int64_t j = 0; j < N; ++j) {
+            double dot = 0.0;
+            for (int64_t k = 0; k < K; ++k) {
+                uint16_t b = b_nk ? B[j * ldb + k] : B[k * ldb + j];
+                dot += widen_bf16(A[i * lda + k]) * widen_bf16(b);
+            }
+            if (C_in) dot += beta * C_in[i * ldcin + j];
+            if (bias) dot += bias[j];
+            C[i * ldc + j] = dot;
         }
     }
 }

@@ -59,6 +59,10 @@ def _load():
         lib.oracle_gemm_sub_f64.argtypes = [ctypes.c_void_p, i64, ctypes.c_void_p, i64, i64, i64,
                                             u16p, i64, u16p, i64, ctypes.c_void_p]
         lib.oracle_gemm_sub_f64.restype = None
+        lib.oracle_gemm_affine_f64.argtypes = [i64, i64, i64, u16p, i64, u16p, i64, ctypes.c_int,
+                                               ctypes.c_double, ctypes.c_void_p, i64, ctypes.c_void_p,
+                                               ctypes.c_void_p, i64]
+        lib.oracle_gemm_affine_f64.restype = None
         lib.oracle_round_bf16.argtypes = [ctypes.c_double]
         lib.oracle_round_bf16.restype = ctypes.c_uint16
         lib.oracle_round_bf16_array.argtypes = [ctypes.c_void_p, i64, ctypes.c_void_p]
@@ -122,6 +126,37 @@ def gemm_sub_f64(A, B, rows=None, cols=None, k0: int = 0, k1: int | None = None)
                                 int(k0), int(k1), a.ctypes.data, K, b.ctypes.data, N,
                                 out.ctypes.data)
     return out
+
+
+def gemm_affine_f64(A, B, *, b_layout: str = "kn", beta: float = 0.0, C_in=None, bias=None) -> np.ndarray:
+    """C = A @ B + beta * C_in + bias (broadcast over rows) in fp64 -- an
+    extension beyond the paper.  B is K x N (``b_layout="kn"``) or its
+    transpose N x K (``"nk"``).  C_in (M x N) and bias (N) are float arrays;
+    either may be None (term left out)."""
+    a = _bf16_bits(A)
+    b = _bf16_bits(B)
+    M, K = a.shape
+    if b_layout == "kn":
+        K2, N = b.shape
+        nk = 0
+    elif b_layout == "nk":
+        N, K2 = b.shape
+        nk = 1
+    else:
+        raise ValueError("b_layout must be 'kn' or 'nk'")
+    if K != K2:
+        raise ValueError("inner dimensions differ")
+    cin = None if C_in is None else np.ascontiguousarray(C_in, dtype=np.float64)
+    if cin is not None and cin.shape != (M, N):
+        raise ValueError("C_in must be M x N")
+    bv = None if bias is None else np.ascontiguousarray(bias, dtype=np.float64)
+    if bv is not None and bv.shape != (N,):
+        raise ValueError("bias must have N entries")
+    C = np.empty((M, N), dtype=np.float64)
+    _load().oracle_gemm_affine_f64(M, N, K, a.ctypes.data, K, b.ctypes.data, b.shape[1], nk, float(beta),
+                                   None if cin is None else cin.ctypes.data, N,
+                                   None if bv is None else bv.ctypes.data, C.ctypes.data, N)
+    return C
 
 
 def round_bf16_bits(x) -> np.ndarray:

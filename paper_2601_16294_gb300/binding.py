@@ -28,10 +28,11 @@ SFC_F32, SFC_BF16 = 0, 1
 ORDERS = {"sfc": 0, "raster": 1}
 ASSIGNS = {"segment": 0, "wave": 1, "auto": 2, "wave_static": 3}
 TILES = {0: 0, "auto": 0, 128: 128, 256: 256, "pair128": 1128, "pair256": 1256, "quad256": 2256}
+B_LAYOUTS = {"kn": 0, "nk": 1}
 
 EXPORTS = ("sfc_tile_order", "sfc_tile_order_device", "sfc_gemm_workspace_size", "sfc_gemm", "sfc_gemm_ex",
            "sfc_get_device_status", "sfc_last_cuda_error", "sfc_num_workers", "sfc_debug_force_timeout",
-           "sfc_gemm_noalloc", "sfc_gemm_plan", "sfc_release")
+           "sfc_gemm_noalloc", "sfc_gemm_plan", "sfc_release", "sfc_gemm_ex2")
 NOALLOC_SCRATCH_BYTES = 32 << 20
 
 
@@ -81,6 +82,8 @@ def load():
         lib.sfc_debug_force_timeout.argtypes = [vp, vp, vp, i32, vp]
         lib.sfc_gemm_noalloc.argtypes = [i64, i64, i64, vp, vp, vp, i64, i64, i64, i32, i32, vp]
         lib.sfc_gemm_plan.argtypes = [i64, i64, i64, i32, i32, i32, vp, vp]
+        lib.sfc_gemm_ex2.argtypes = [i64, i64, i64, vp, vp, vp, i64, i64, i64, i32, ctypes.c_float, vp, i32, i32,
+                                     i32, i32, i32, vp, sz, vp]
         lib.sfc_release.argtypes = []
         for name in EXPORTS:
             if name != "sfc_gemm_workspace_size":
@@ -157,34 +160,49 @@ def _row_major_2d(t, name):
 
 
 def gemm(A, B, C=None, *, ca_c: int = 1, out_dtype=None, order: str = "sfc", assign: str = "auto",
-         tile=0, workspace=None, stream=None):
-    """C = A @ B on the GPU.  A: (M, K) bf16, B: (K, N) bf16, both CUDA, row-major
-    (row strides may be padded).  C: (M, N) fp32 or bf16 CUDA tensor, allocated
-    if not given.  ``ca_c``: K layers (0: the library chooses).  ``workspace``:
-    optional CUDA tensor of at least ``workspace_size(M, N, K, ca_c)`` bytes."""
+         tile=0, workspace=None, stream=None, b_layout: str = "kn", beta: float = 0.0, bias=None):
+    """C = A @ B (+ beta * C + bias) on the GPU.  A: (M, K) bf16 CUDA tensor,
+    row-major (row stride may be padded).  B: bf16, (K, N) for ``b_layout="kn"``
+    or its transpose (N, K) for ``"nk"`` (a linear layer's weight).  C: (M, N)
+    fp32 or bf16 CUDA tensor, allocated if not given (then ``beta`` must be 0).
+    ``bias``: optional fp32 CUDA tensor of N values.  ``ca_c``: K layers (0: the
+    library chooses).  ``workspace``: optional CUDA tensor of at least
+    ``workspace_size(M, N, K, ca_c)`` bytes."""
     import torch
     lib = load()
     M, K = A.shape
-    K2, N = B.shape
+    if b_layout == "kn":
+        K2, N = B.shape
+    elif b_layout == "nk":
+        N, K2 = B.shape
+    else:
+        raise ValueError("b_layout must be 'kn' or 'nk'")
     if K != K2:
         raise ValueError("inner dimensions differ: %d vs %d" % (K, K2))
     if A.dtype != torch.bfloat16 or B.dtype != torch.bfloat16:
         raise TypeError("A and B must be bfloat16")
     if C is None:
+        if beta != 0.0:
+            raise ValueError("beta != 0 needs an input C")
         C = torch.empty((M, N), dtype=out_dtype or torch.float32, device=A.device)
     if C.dtype not in (torch.float32, torch.bfloat16) or tuple(C.shape) != (M, N):
         raise ValueError("C must be (M, N) float32 or bfloat16")
+    bias_ptr = None
+    if bias is not None:
+        if bias.dtype != torch.float32 or bias.numel() != N or not bias.is_contiguous():
+            raise ValueError("bias must be a contiguous float32 tensor of N values")
+        bias_ptr = ctypes.c_void_p(bias.data_ptr())
     lda = _row_major_2d(A, "A")
     ldb = _row_major_2d(B, "B")
     ldc = _row_major_2d(C, "C")
     ws_ptr, ws_bytes = None, 0
     if workspace is not None:
         ws_ptr, ws_bytes = ctypes.c_void_p(workspace.data_ptr()), workspace.numel() * workspace.element_size()
-    rc = lib.sfc_gemm_ex(M, N, K, ctypes.c_void_p(A.data_ptr()), ctypes.c_void_p(B.data_ptr()),
-                         ctypes.c_void_p(C.data_ptr()), lda, ldb, ldc, int(ca_c),
-                         SFC_F32 if C.dtype == torch.float32 else SFC_BF16, ORDERS[order], ASSIGNS[assign],
-                         TILES[tile], ws_ptr, ws_bytes, _stream_ptr(stream))
-    _check(rc, "sfc_gemm_ex")
+    rc = lib.sfc_gemm_ex2(M, N, K, ctypes.c_void_p(A.data_ptr()), ctypes.c_void_p(B.data_ptr()),
+                          ctypes.c_void_p(C.data_ptr()), lda, ldb, ldc, B_LAYOUTS[b_layout], float(beta), bias_ptr,
+                          int(ca_c), SFC_F32 if C.dtype == torch.float32 else SFC_BF16, ORDERS[order],
+                          ASSIGNS[assign], TILES[tile], ws_ptr, ws_bytes, _stream_ptr(stream))
+    _check(rc, "sfc_gemm_ex2")
     return C
 
 

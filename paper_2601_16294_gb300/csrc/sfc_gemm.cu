@@ -299,8 +299,10 @@ struct Plan {
 // max_c.  A requested tile fixes the variant (falling back to one SM when
 // pairs cannot be co-scheduled).
 Plan make_plan(int64_t M, int64_t N, int64_t K, int ca_c, int max_c, const DeviceInfo& d, sfc_tile_t tile,
-               int out_bytes) {
+               int out_bytes, bool b_kmajor = false) {
     int fixed = -1;
+    // the quad variant splits the B slab along K between its pairs, which needs N-major B
+    if (b_kmajor && tile == SFC_TILE_QUAD_N256) tile = SFC_TILE_PAIR_N256;
     switch (tile) {
         case SFC_TILE_N128: fixed = kSingle128; break;
         case SFC_TILE_N256: fixed = kSingle256; break;
@@ -313,7 +315,7 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, int ca_c, int max_c, const Devic
     double best_t = -1.0;
     const int c_lo = ca_c > 0 ? ca_c : 1, c_hi = ca_c > 0 ? ca_c : max_c;
     for (int v = 0; v < kNumVariants; ++v) {
-        if (d.workers[v] <= 0 || (fixed >= 0 && v != fixed)) continue;
+        if (d.workers[v] <= 0 || (fixed >= 0 && v != fixed) || (b_kmajor && v == kQuad256)) continue;
         for (int c = c_lo; c <= c_hi; ++c) {
             const double t = plan_cost(M, N, K, c, v, d, out_bytes);
             if (best_t < 0.0 || t < best_t) {  // ties keep fewer layers, then the earlier variant
@@ -328,9 +330,11 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, int ca_c, int max_c, const Devic
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
 int validate(int64_t M, int64_t N, int64_t K, const void* A, const void* B, const void* C, int64_t lda,
-             int64_t ldb, int64_t ldc, int ca_c, int c_dtype, int order, int assign, int tile) {
+             int64_t ldb, int64_t ldc, int ca_c, int c_dtype, int order, int assign, int tile,
+             int b_layout = SFC_B_KN) {
     if (M <= 0 || N <= 0 || K <= 0 || !A || !B || !C) return SFC_ERR_INVALID_ARG;
-    if (lda < K || ldb < N || ldc < N) return SFC_ERR_INVALID_ARG;
+    if (b_layout != SFC_B_KN && b_layout != SFC_B_NK) return SFC_ERR_INVALID_ARG;
+    if (lda < K || ldb < (b_layout == SFC_B_NK ? K : N) || ldc < N) return SFC_ERR_INVALID_ARG;
     if (c_dtype != SFC_F32 && c_dtype != SFC_BF16) return SFC_ERR_INVALID_ARG;
     if (order != SFC_ORDER_SFC && order != SFC_ORDER_RASTER) return SFC_ERR_INVALID_ARG;
     if (assign != SFC_ASSIGN_SEGMENT && assign != SFC_ASSIGN_WAVE && assign != SFC_ASSIGN_AUTO &&
@@ -364,9 +368,12 @@ cudaError_t launch_gemm(int v, const CUtensorMap& ta, const CUtensorMap& tb, con
 
 int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void* C, int64_t lda, int64_t ldb,
              int64_t ldc, int ca_c, int c_dtype, int order, int assign, int tile, void* workspace,
-             size_t workspace_bytes, cudaStream_t stream, int debug_never, uint64_t timeout_ns) {
-    int rc = validate(M, N, K, A, B, C, lda, ldb, ldc, ca_c, c_dtype, order, assign, tile);
+             size_t workspace_bytes, cudaStream_t stream, int debug_never, uint64_t timeout_ns,
+             int b_layout = SFC_B_KN, float beta = 0.0f, const float* bias = nullptr) {
+    int rc = validate(M, N, K, A, B, C, lda, ldb, ldc, ca_c, c_dtype, order, assign, tile, b_layout);
     if (rc != SFC_OK) return rc;
+    if (bias && (reinterpret_cast<uintptr_t>(bias) & 3u) != 0) return SFC_ERR_UNALIGNED;
+    const bool b_kmajor = (b_layout == SFC_B_NK);
     if (ca_c > 0 && workspace && workspace_bytes < sfc_gemm_workspace_size(M, N, K, ca_c)) return SFC_ERR_WORKSPACE;
     if (workspace && !aligned16(workspace)) return SFC_ERR_UNALIGNED;
 
@@ -377,7 +384,8 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     // ca_c = 0: the planner's layer count, within the caller's workspace if one is given
     int max_c = static_cast<int>(auto_layer_cap(M, N, K));
     while (ca_c == 0 && workspace && max_c > 1 && workspace_bytes < sfc_gemm_workspace_size(M, N, K, max_c)) --max_c;
-    const Plan plan = make_plan(M, N, K, ca_c, max_c, *dev, static_cast<sfc_tile_t>(tile), c_dtype == SFC_F32 ? 4 : 2);
+    const Plan plan =
+        make_plan(M, N, K, ca_c, max_c, *dev, static_cast<sfc_tile_t>(tile), c_dtype == SFC_F32 ? 4 : 2, b_kmajor);
     const int v = plan.v;
     ca_c = plan.c;
     const size_t ws_need = sfc_gemm_workspace_size(M, N, K, ca_c);
@@ -386,8 +394,13 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     CUtensorMap ta, tb;
     rc = make_bf16_map(&ta, A, M, K, lda, kBM, kBK);  // each CTA loads 128 rows of A
     if (rc != SFC_OK) return rc;
-    // B boxes: 64 K rows x 64 columns; with two pairs sharing B each CTA loads 32 K rows
-    rc = make_bf16_map(&tb, B, K, N, ldb, v == kQuad256 ? kBK / 2 : kBK, kBBox);
+    if (b_kmajor) {
+        // B given as N x K: boxes of (this CTA's share of the tile's N rows) x 64 k, like A
+        rc = make_bf16_map(&tb, B, N, K, ldb, variant_pair(v) ? bn / 2 : bn, kBK);
+    } else {
+        // B boxes: 64 K rows x 64 columns; with two pairs sharing B each CTA loads 32 K rows
+        rc = make_bf16_map(&tb, B, K, N, ldb, v == kQuad256 ? kBK / 2 : kBK, kBBox);
+    }
     if (rc != SFC_OK) return rc;
 
     GemmParams p;
@@ -410,6 +423,11 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     p.sched_slot = static_cast<int>(g_launch_seq.fetch_add(1, std::memory_order_relaxed) % kSchedSlots);
     p.debug_never = debug_never;
     p.timeout_ns = timeout_ns;
+    p.b_kmajor = b_kmajor ? 1 : 0;
+    p.beta = beta;
+    p.c_in = C;
+    p.ldc_in = ldc;
+    p.bias = bias;
     const int64_t workers = dev->one_item_per_worker ? p.num_items : dev->workers[v];
     const int64_t used = p.num_items < workers ? p.num_items : workers;
     const int grid = static_cast<int>(variant_cluster(v) * used);
@@ -460,10 +478,10 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
             const float* wsf = static_cast<const float*>(ws);
             if (c_dtype == SFC_F32)
                 e = cudaLaunchKernelEx(&cfg, ca_reduce_kernel<float>, wsf, p.ldo, p.layer_stride, ca_c, M, N,
-                                       static_cast<float*>(C), ldc, vec);
+                                       static_cast<float*>(C), ldc, vec, beta, bias);
             else
                 e = cudaLaunchKernelEx(&cfg, ca_reduce_kernel<__nv_bfloat16>, wsf, p.ldo, p.layer_stride, ca_c, M,
-                                       N, static_cast<__nv_bfloat16*>(C), ldc, vec);
+                                       N, static_cast<__nv_bfloat16*>(C), ldc, vec, beta, bias);
             if (e == cudaSuccess) e = cudaGetLastError();
         }
     }
@@ -557,6 +575,14 @@ SFC_API int sfc_gemm_ex(int64_t M, int64_t N, int64_t K, const void* A, const vo
                         void* stream) {
     return run_gemm(M, N, K, A, B, C, lda, ldb, ldc, ca_c, c_dtype, order, assign, tile, workspace,
                     workspace_bytes, static_cast<cudaStream_t>(stream), 0, kDefaultTimeoutNs);
+}
+
+SFC_API int sfc_gemm_ex2(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void* C, int64_t lda,
+                         int64_t ldb, int64_t ldc, int b_layout, float beta, const float* bias, int ca_c,
+                         sfc_dtype_t c_dtype, sfc_order_t order, sfc_assign_t assign, sfc_tile_t tile,
+                         void* workspace, size_t workspace_bytes, void* stream) {
+    return run_gemm(M, N, K, A, B, C, lda, ldb, ldc, ca_c, c_dtype, order, assign, tile, workspace,
+                    workspace_bytes, static_cast<cudaStream_t>(stream), 0, kDefaultTimeoutNs, b_layout, beta, bias);
 }
 
 SFC_API int sfc_get_device_status(void* stream) {

@@ -102,6 +102,11 @@ struct GemmParams {
     int serpentine;        // 1: alternate the K direction between a worker's consecutive items
     int debug_never;       // test hook: MMA warp waits on a barrier nobody arrives at
     uint64_t timeout_ns;   // bound for every mbarrier wait
+    int b_kmajor;          // 1: B is given as N x K row-major (B transposed), loaded K-major
+    float beta;            // C = A B + beta C_in + bias (ca_c == 1: applied by the epilogue)
+    const void* c_in;      // C_in (the output array, read before it is written) when beta != 0
+    int64_t ldc_in;        // its row stride in elements
+    const float* bias;     // N fp32 values or null
 };
 
 struct WorkItem {
@@ -225,6 +230,23 @@ __device__ __forceinline__ void store_chunk(OutT* row_ptr, int64_t col0, int64_t
 #pragma unroll
         for (int j = 0; j < 32; ++j)
             if (col0 + j < N) row_ptr[col0 + j] = cvt_out<OutT>(v[j]);
+    }
+}
+
+// beta * C_in + bias for columns [col0, col0 + n) of one row, added into v
+// (fp32, before rounding to the output type).  Columns >= N are left alone.
+template <typename OutT, int n>
+__device__ __forceinline__ void apply_affine(const GemmParams& p, int64_t row, int64_t col0, float* v) {
+    if (p.beta != 0.0f && row < p.M) {
+        const OutT* src = static_cast<const OutT*>(p.c_in) + row * p.ldc_in + col0;
+#pragma unroll
+        for (int j = 0; j < n; ++j)
+            if (col0 + j < p.N) v[j] = __fmaf_rn(p.beta, static_cast<float>(src[j]), v[j]);
+    }
+    if (p.bias) {
+#pragma unroll
+        for (int j = 0; j < n; ++j)
+            if (col0 + j < p.N) v[j] = __fadd_rn(v[j], __ldg(p.bias + col0 + j));
     }
 }
 
@@ -447,6 +469,8 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
     const uint32_t acce_target = PAIR ? ptx::map_to_cta(B.acc_empty(0), pair_leader) : B.acc_empty(0);
     float run[kEpiCols];
     int nbox = 0;  // boxes this warp has stored (selects the staging half)
+    // beta C_in + bias in this epilogue only without K layers (else the reduction applies it)
+    const bool affine = p.ca_c == 1 && (p.beta != 0.0f || p.bias != nullptr);
     for (int j = 0;; ++j) {
         // lane 0 takes the item, the warp follows (tcgen05.ld needs the whole warp)
         int64_t it = 0;
@@ -505,6 +529,7 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
             for (int g = 0; g < kEpiCols / kCols; ++g) {
                 if (col_base + g * kCols >= p.N) break;  // warp-uniform
                 uint8_t* box = staging + ew * kStageBufBytes + (nbox & 1) * kBoxBytes;
+                if (affine) apply_affine<OutT, kCols>(p, warp_row + lane, col_base + g * kCols, run + g * kCols);
                 if (lane == 0) ptx::bulk_wait_read_1();  // the store that last used this box has read it
                 __syncwarp();
                 stage_row<OutT>(box, lane, run + g * kCols);
@@ -527,8 +552,10 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
             if (row < p.M) {
                 OutT* row_ptr = out + static_cast<int64_t>(w.layer) * p.layer_stride + row * p.ldo;
 #pragma unroll
-                for (int g = 0; g < kEpiCols / 32; ++g)
+                for (int g = 0; g < kEpiCols / 32; ++g) {
+                    if (affine) apply_affine<OutT, 32>(p, row, col_base + g * 32, run + g * 32);
                     store_chunk<OutT>(row_ptr, col_base + g * 32, p.N, run + g * 32, p.vec_store != 0);
+                }
             }
         }
     }
@@ -550,6 +577,7 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
     constexpr int kEpiWarps = BN / 32;
     using L = RingLayout<kStageBytes, STAGES, kEpiWarps>;
     constexpr uint32_t kIdesc = ptx::idesc_bf16_f32(kBM, BN, /*A K-major*/ 0, /*B MN-major*/ 1);
+    constexpr uint32_t kIdescBK = ptx::idesc_bf16_f32(kBM, BN, /*A K-major*/ 0, /*B K-major*/ 0);
     constexpr uint32_t kTmemCols = 2 * BN;
 
     extern __shared__ uint8_t smem_raw[];
@@ -628,10 +656,15 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
                 const uint32_t sa = ring + stage * kStageBytes;
                 const uint32_t sb = sa + kABytes;
                 ptx::tma_load_2d(sa, &tmap_a, B.full(stage), kt * kBK, w.tm * kBM);
+                if (p.b_kmajor) {
+                    // B^T rows (N) x 64 k, K-major like A
+                    ptx::tma_load_2d(sb, &tmap_b, B.full(stage), kt * kBK, w.tn * BN);
+                } else {
 #pragma unroll
-                for (int jb = 0; jb < BN / kBBox; ++jb)
-                    ptx::tma_load_2d(sb + jb * (kBBox * kBK * 2), &tmap_b, B.full(stage), w.tn * BN + jb * kBBox,
-                                     kt * kBK);
+                    for (int jb = 0; jb < BN / kBBox; ++jb)
+                        ptx::tma_load_2d(sb + jb * (kBBox * kBK * 2), &tmap_b, B.full(stage),
+                                         w.tn * BN + jb * kBBox, kt * kBK);
+                }
             });
             // Tail: the last STAGES issues.  On success wait until the MMA warp's
             // commits have released them (no arrive may land after exit); after a
@@ -682,10 +715,13 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
                         for (int kk = 0; kk < kBK / kUmmaK; ++kk) {
                             // A: K-major, 128-byte rows, 8-row atoms 1024 B apart; 32 B per K=16
                             const uint64_t adesc = ptx::smem_desc_sw128(sa + kk * (kUmmaK * 2), 16, 1024);
-                            // B: MN-major, 64-column boxes 8 KB apart, 8-row atoms 1 KB apart; 2 KB per K=16
-                            const uint64_t bdesc =
-                                ptx::smem_desc_sw128(sb + kk * (kUmmaK * 128), kBBox * kBK * 2, 1024);
-                            ptx::tc_mma_f16(d_tmem, adesc, bdesc, kIdesc, (q > kb || kk > 0) ? 1u : 0u);
+                            // B MN-major: 64-column boxes 8 KB apart, 8-row atoms 1 KB apart, 2 KB per
+                            // K=16; B K-major: as A
+                            const uint64_t bdesc = p.b_kmajor
+                                ? ptx::smem_desc_sw128(sb + kk * (kUmmaK * 2), 16, 1024)
+                                : ptx::smem_desc_sw128(sb + kk * (kUmmaK * 128), kBBox * kBK * 2, 1024);
+                            ptx::tc_mma_f16(d_tmem, adesc, bdesc, p.b_kmajor ? kIdescBK : kIdesc,
+                                            (q > kb || kk > 0) ? 1u : 0u);
                         }
                         ptx::tc_commit(B.empty(stage));  // frees the stage once these MMAs finish
                         if (++stage == STAGES) {
@@ -723,10 +759,12 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
 
 // C = cvt(sum_{l=0}^{c-1} P_l), summed in layer order, 4 columns per thread.
 // P_l rows are `ldw` floats apart (ldw % 4 == 0), layers `layer_stride` apart.
+// Then, if asked, C = that + beta * C_in + bias (C_in is C read first).
 template <typename OutT>
 __global__ void __launch_bounds__(256)
 ca_reduce_kernel(const float* __restrict__ ws, int64_t ldw, int64_t layer_stride, int c, int64_t M,
-                 int64_t N, OutT* __restrict__ C, int64_t ldc, int vec_store) {
+                 int64_t N, OutT* __restrict__ C, int64_t ldc, int vec_store, float beta,
+                 const float* __restrict__ bias) {
     ptx::pdl_launch_dependents();
     ptx::pdl_wait();  // the partials come from the GEMM kernel just before
     const int64_t n4 = (N + 3) / 4;
@@ -745,6 +783,14 @@ ca_reduce_kernel(const float* __restrict__ ws, int64_t ldw, int64_t layer_stride
             acc.w += v.w;
         }
         OutT* dst = C + i * ldc + j;
+        if (beta != 0.0f || bias) {
+            float v[4] = {acc.x, acc.y, acc.z, acc.w};
+            for (int h = 0; h < 4 && j + h < N; ++h) {
+                if (beta != 0.0f) v[h] = __fmaf_rn(beta, static_cast<float>(dst[h]), v[h]);
+                if (bias) v[h] = __fadd_rn(v[h], bias[j + h]);
+            }
+            acc = make_float4(v[0], v[1], v[2], v[3]);
+        }
         if (vec_store && j + 4 <= N) {
             if constexpr (sizeof(OutT) == 4) {
                 *reinterpret_cast<float4*>(dst) = acc;

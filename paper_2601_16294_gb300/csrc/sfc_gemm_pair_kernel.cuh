@@ -56,6 +56,7 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
     using L = RingLayout<S::kBytes, STAGES, kEpiWarps>;
     constexpr int kHalfN = S::kHalfN;
     constexpr uint32_t kIdesc = ptx::idesc_bf16_f32(kPairBM, BN, /*A K-major*/ 0, /*B MN-major*/ 1);
+    constexpr uint32_t kIdescBK = ptx::idesc_bf16_f32(kPairBM, BN, /*A K-major*/ 0, /*B K-major*/ 0);
     constexpr uint32_t kTmemCols = 2 * BN;
     // QUAD: a cluster of two pairs stacked in M (a 512 x BN item) sharing the B slab
     constexpr int kCtas = QUAD ? 4 : 2;
@@ -151,7 +152,10 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
                 const uint32_t sa = ring + stage * S::kBytes;
                 const uint32_t sb = sa + S::kABytes;
                 ptx::tma_load_2d_pair(sa, &tmap_a, leader_full, kt * kBK, a_row);
-                if constexpr (QUAD) {
+                if (!QUAD && p.b_kmajor) {
+                    // this CTA's half of the B^T rows (N) x 64 k, K-major like A
+                    ptx::tma_load_2d_pair(sb, &tmap_b, leader_full, kt * kBK, b_col);
+                } else if constexpr (QUAD) {
                     // the same B half-slab goes to this CTA and its counterpart in the
                     // other pair: each loads 32 of the 64 K rows for both
                     const uint16_t mask = static_cast<uint16_t>((1u << r) | (1u << (r + 2)));
@@ -225,10 +229,13 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
                         for (int kk = 0; kk < kBK / kUmmaK; ++kk) {
                             // A half: K-major, 128-byte rows, 8-row atoms 1 KB apart; 32 B per K=16
                             const uint64_t adesc = ptx::smem_desc_sw128(sa + kk * (kUmmaK * 2), 16, 1024);
-                            // B half: MN-major, 64-column boxes 8 KB apart; 2 KB per K=16
-                            const uint64_t bdesc =
-                                ptx::smem_desc_sw128(sb + kk * (kUmmaK * 128), kBBox * kBK * 2, 1024);
-                            ptx::tc_mma_f16_pair(d_tmem, adesc, bdesc, kIdesc, (q > kb || kk > 0) ? 1u : 0u);
+                            // B half MN-major: 64-column boxes 8 KB apart, 2 KB per K=16; K-major: as A
+                            const bool bk = !QUAD && p.b_kmajor;
+                            const uint64_t bdesc = bk
+                                ? ptx::smem_desc_sw128(sb + kk * (kUmmaK * 2), 16, 1024)
+                                : ptx::smem_desc_sw128(sb + kk * (kUmmaK * 128), kBBox * kBK * 2, 1024);
+                            ptx::tc_mma_f16_pair(d_tmem, adesc, bdesc, bk ? kIdescBK : kIdesc,
+                                                 (q > kb || kk > 0) ? 1u : 0u);
                         }
                         // the stage is free in every CTA whose smem this pair read (and, with
                         // QUAD, whose producer also wrote into this pair's smem)

@@ -155,3 +155,19 @@ def test_missing_library_raises(monkeypatch, tmp_path):
     monkeypatch.setattr(binding, "library_path", lambda: str(tmp_path / "absent.so"))
     with pytest.raises(binding.SfcLibraryMissing):
         binding.load()
+
+
+def call_ex2(lib, M=256, N=256, K=256, ldb=None, b_layout=0, beta=0.0, bias=None, ca_c=1):
+    ldb = (N if b_layout == 0 else K) if ldb is None else ldb
+    return lib.sfc_gemm_ex2(M, N, K, ctypes.c_void_p(PA), ctypes.c_void_p(PB), ctypes.c_void_p(PC), K, ldb, N,
+                            b_layout, beta, ctypes.c_void_p(bias) if bias else None, ca_c, 0, 0, 2, 0, None, 0,
+                            None)
+
+
+def test_gemm_ex2_validation_codes(lib):
+    E = binding
+    assert call_ex2(lib, b_layout=2) == E.SFC_ERR_INVALID_ARG
+    assert call_ex2(lib, N=512, K=256, b_layout=1, ldb=200) == E.SFC_ERR_INVALID_ARG    # B^T rows shorter than K
+    assert call_ex2(lib, N=512, K=256, b_layout=0, ldb=256) == E.SFC_ERR_INVALID_ARG    # B rows shorter than N
+    assert call_ex2(lib, N=512, K=256, b_layout=1, ldb=260) == E.SFC_ERR_UNALIGNED
+    assert call_ex2(lib, bias=0x50002) == E.SFC_ERR_UNALIGNED                           # bias not 4-byte aligned

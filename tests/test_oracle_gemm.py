@@ -126,3 +126,42 @@ def test_round_bf16_single_step(oracle):
     vals = torch.randn(5000, generator=torch.Generator().manual_seed(0), dtype=torch.float32) * 100
     ref = vals.to(torch.bfloat16).float().numpy().astype(np.float64)
     assert np.array_equal(oracle.round_bf16(vals.numpy().astype(np.float64)), ref)
+
+
+# --- the BLAS-style extension: transposed B, beta * C_in, bias (no paper counterpart)
+
+def test_affine_without_terms_is_the_plain_product(oracle):
+    A, B = synth.gemm_inputs(37, 29, 53, "uniform", seed=3)
+    plain = oracle.gemm_f64(A, B)
+    assert np.array_equal(oracle.gemm_affine_f64(A, B), plain)
+    # the transposed storage of the same B gives the same sums in the same order
+    assert np.array_equal(oracle.gemm_affine_f64(A, B.t().contiguous(), b_layout="nk"), plain)
+
+
+def test_affine_closed_forms(oracle):
+    M, N, K = 12, 20, 12
+    Bt = synth.uniform_bf16((N, K), seed=9)              # B stored transposed
+    C_in = np.arange(M * N, dtype=np.float64).reshape(M, N) / 8.0
+    bias = np.linspace(-3.0, 3.0, N)
+    I = torch.eye(M, dtype=torch.bfloat16)
+    # A = I: C = B = Bt^T exactly, then + bias
+    assert np.array_equal(oracle.gemm_affine_f64(I, Bt, b_layout="nk"), bf16_values(Bt).T)
+    assert np.array_equal(oracle.gemm_affine_f64(I, Bt, b_layout="nk", bias=bias), bf16_values(Bt).T + bias)
+    # A = 0: only the affine terms remain
+    Z = torch.zeros(M, K, dtype=torch.bfloat16)
+    got = oracle.gemm_affine_f64(Z, Bt, b_layout="nk", beta=-2.5, C_in=C_in, bias=bias)
+    assert np.array_equal(got, -2.5 * C_in + bias)
+
+
+def test_affine_small_integers_exact(oracle):
+    M, N, K = 33, 18, 70
+    A, B = synth.gemm_inputs(M, N, K, "int", seed=21)
+    g = np.random.default_rng(4)
+    C_in = g.integers(-50, 50, size=(M, N)).astype(np.float64)
+    bias = g.integers(-9, 9, size=N).astype(np.float64)
+    ai = bf16_values(A).astype(np.int64)
+    bi = bf16_values(B).astype(np.int64)
+    want = (ai @ bi) + 3 * C_in.astype(np.int64) + bias.astype(np.int64)
+    for layout, b in (("kn", B), ("nk", B.t().contiguous())):
+        got = oracle.gemm_affine_f64(A, b, b_layout=layout, beta=3.0, C_in=C_in, bias=bias)
+        assert np.array_equal(got, want.astype(np.float64)), layout
