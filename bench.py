@@ -99,6 +99,8 @@ def parse_args():
     ap.add_argument("--sizes", type=str, default=None,
                     help="square workload only: comma-separated sizes instead of the full sweep")
     ap.add_argument("--ca-c", type=int, default=None, help="force one K-layer count for every shape")
+    ap.add_argument("--b-layout", choices=("kn", "nk"), default="kn",
+                    help="storage of B: K x N row-major (the paper's), or N x K (a linear layer's weight)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
@@ -268,13 +270,26 @@ def run_ours(args, rank, local, world):
 
     # inputs resident in HBM before timing (seeded on the CPU, copied once)
     mats = []
+    transposed = {}  # B stored N x K: one transposed device copy per B
+
+    def as_nk(Bd):
+        if id(Bd) not in transposed:
+            K, N = Bd.shape
+            buf = torch.zeros(N, synth.pad8(K), dtype=torch.bfloat16, device="cuda")
+            buf[:, :K] = Bd.t()
+            transposed[id(Bd)] = buf[:, :K]
+        return transposed[id(Bd)]
+
     for s in shapes:
         A, B, Ad, Bd, C = make_inputs(s, synth, torch)
+        if args.b_layout == "nk":
+            Bd = as_nk(Bd)
         mats.append({"s": s, "A": A, "B": B, "Ad": Ad, "Bd": Bd, "C": C, "c": s["cs"][0]})
     torch.cuda.synchronize()
 
     def call(m, c):
-        sfc.gemm(m["Ad"], m["Bd"], m["C"], ca_c=c, order=args.order, assign=args.assign, stream=stream)
+        sfc.gemm(m["Ad"], m["Bd"], m["C"], ca_c=c, order=args.order, assign=args.assign, stream=stream,
+                 b_layout=args.b_layout)
 
     # pick the K-layer count per shape where several are listed (timed, warm)
     cs_report = {}
@@ -372,12 +387,14 @@ def run_ours(args, rank, local, world):
             extra.append((clone_strided(m["Ad"]), clone_strided(m["Bd"])))
         reps = max(2 * copies, min(400, int(0.05 / max(roofline_time_s(s_, peaks)[0], 1e-6))))
         for a, b in extra:
-            sfc.gemm(a, b, m["C"], ca_c=m["c"], order=args.order, assign=args.assign, stream=stream)
+            sfc.gemm(a, b, m["C"], ca_c=m["c"], order=args.order, assign=args.assign, stream=stream,
+                     b_layout=args.b_layout)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
         for r in range(reps):
             a, b = extra[r % copies]
-            sfc.gemm(a, b, m["C"], ca_c=m["c"], order=args.order, assign=args.assign, stream=stream)
+            sfc.gemm(a, b, m["C"], ca_c=m["c"], order=args.order, assign=args.assign, stream=stream,
+                     b_layout=args.b_layout)
         e1.record(stream)
         torch.cuda.synchronize()
         b2b_ms.append(e0.elapsed_time(e1) / reps)
@@ -431,7 +448,7 @@ def run_ours(args, rank, local, world):
         "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded %s bf16)" % ",".join(sorted({m["s"]["kind"] for m in mats})),
-        "config": {"workload": desc, "order": args.order, "assign": args.assign,
+        "config": {"workload": desc, "order": args.order, "assign": args.assign, "b_layout": args.b_layout,
                    "parallelism": "replicas" if world > 1 else "single GPU",
                    "l2": "inputs larger than L2 between reuses: one step runs every shape once, so a shape's "
                          "operands are re-read only after the other shapes' traffic has passed through L2",
@@ -460,10 +477,11 @@ def run_cublas_compare(args, mats, stream, call):
     import torch
 
     def cublas(m):
+        Bd = m["Bd"].t() if args.b_layout == "nk" else m["Bd"]
         if m["C"].dtype == torch.bfloat16:
-            torch.matmul(m["Ad"], m["Bd"], out=m["C"])
+            torch.matmul(m["Ad"], Bd, out=m["C"])
         else:
-            m["C"].copy_(torch.matmul(m["Ad"], m["Bd"]))
+            m["C"].copy_(torch.matmul(m["Ad"], Bd))
 
     steps = max(3, min(args.steps, 50))
     t = [[0.0, 0.0] for _ in mats]
@@ -506,15 +524,24 @@ def run_e2e(args, mats, stream, world):
             pinned[id(t)] = t.contiguous().pin_memory()
         return pinned[id(t)]
 
+    nk = {}  # host copies of B stored N x K, one per B
+
+    def host_b(B):
+        if args.b_layout == "kn":
+            return pin(B)
+        if id(B) not in nk:
+            nk[id(B)] = B.t().contiguous().pin_memory()
+        return nk[id(B)]
+
     host = []
     for m in mats:
-        host.append((m, pin(m["A"]), pin(m["B"]), torch.empty(m["C"].shape, dtype=m["C"].dtype, pin_memory=True)))
+        host.append((m, pin(m["A"]), host_b(m["B"]), torch.empty(m["C"].shape, dtype=m["C"].dtype, pin_memory=True)))
     h2d = sum(Ah.numel() * 2 + Bh.numel() * 2 for _, Ah, Bh, _ in host)
     d2h = sum(Ch.numel() * Ch.element_size() for _, _, _, Ch in host)
 
     def step():
         for m, Ah, Bh, Ch in host:
-            sfc.matmul_host(Ah, Bh, Ch, ca_c=m["c"], out_dtype=Ch.dtype, stream=stream)
+            sfc.matmul_host(Ah, Bh, Ch, ca_c=m["c"], out_dtype=Ch.dtype, stream=stream, b_layout=args.b_layout)
 
     for _ in range(2):
         step()
