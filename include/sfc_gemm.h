@@ -60,6 +60,13 @@ typedef enum { SFC_F32 = 0, SFC_BF16 = 1 } sfc_dtype_t;
  * K-major like A.  Not part of the paper, which fixes the KN layout. */
 typedef enum { SFC_B_KN = 0, SFC_B_NK = 1 } sfc_b_layout_t;
 
+/* Element type of A and B (sfc_gemm_ex2): bf16, or one of the two 8-bit float
+ * formats (e4m3: 4 exponent bits, bias 7, no infinities; e5m2: 5 exponent
+ * bits, bias 15).  The paper notes the method is independent of the data type
+ * and evaluates bf16 (Sec. III, Sec. IV-A); the 8-bit kinds use the tensor
+ * cores' 8-bit path (32 values of k per instruction) with fp32 accumulation. */
+typedef enum { SFC_AB_BF16 = 0, SFC_AB_E4M3 = 1, SFC_AB_E5M2 = 2 } sfc_ab_t;
+
 /* Order of the output tiles along which workers take their items.
  * SFC:    generalized Hilbert curve (Sec. II-B) -- the method.
  * RASTER: row-major tile order s -> (s / Nt, s % Nt), a comparison baseline. */
@@ -176,10 +183,14 @@ int sfc_gemm_ex(int64_t M, int64_t N, int64_t K,
                 void *workspace, size_t workspace_bytes, void *stream);
 
 /*
- * sfc_gemm_ex2 -- sfc_gemm_ex extended with the operand layout and epilogue of
- * a BLAS-style GEMM (no counterpart in the paper, which computes C = A B with
- * C zeroed first, Listing 1):
+ * sfc_gemm_ex2 -- sfc_gemm_ex extended with the input type, and with the
+ * operand layout and epilogue of a BLAS-style GEMM (no counterpart in the
+ * paper, which computes C = A B with C zeroed first, Listing 1):
  *     C = A B + beta * C + bias[j]     (fp32 arithmetic, then rounded to c_dtype)
+ *   ab_dtype: sfc_ab_t of both A and B.  For the 8-bit kinds lda and ldb are
+ *             multiples of 16 elements, K layers split ceil(K/128) slabs of
+ *             128 values of k, and the N-major (SFC_B_KN) layout is not served
+ *             by SFC_TILE_PAIR_N128 (SFC_TILE_N128 is used instead).
  *   b_layout: SFC_B_KN (B is K x N, ldb >= N) or SFC_B_NK (B is stored as its
  *             transpose, N x K, ldb >= K).  SFC_TILE_QUAD_N256 is served by
  *             SFC_TILE_PAIR_N256 with SFC_B_NK.
@@ -195,21 +206,22 @@ int sfc_gemm_ex(int64_t M, int64_t N, int64_t K,
 int sfc_gemm_ex2(int64_t M, int64_t N, int64_t K,
                  const void *A, const void *B, void *C,
                  int64_t lda, int64_t ldb, int64_t ldc,
-                 int b_layout, float beta, const float *bias,
+                 int ab_dtype, int b_layout, float beta, const float *bias,
                  int ca_c, sfc_dtype_t c_dtype,
                  sfc_order_t order, sfc_assign_t assign, sfc_tile_t tile,
                  void *workspace, size_t workspace_bytes, void *stream);
 
 /*
- * sfc_gemm_plan -- the tile and K-layer count sfc_gemm_ex would use for these
+ * sfc_gemm_plan -- the tile and K-layer count sfc_gemm_ex2 would use for these
  * arguments on the current device (ca_c = 0: the library's choice; ca_c >= 1:
  * that count with the tile AUTO or `tile` picks).  No kernel runs.
+ *   ab_dtype, b_layout: as sfc_gemm_ex2 (SFC_AB_BF16, SFC_B_KN for sfc_gemm_ex).
  *   out_tile: an sfc_tile_t other than SFC_TILE_AUTO.  out_ca_c: >= 1.
- * Errors: SFC_ERR_INVALID_ARG (as sfc_gemm_ex, or a NULL output pointer),
+ * Errors: SFC_ERR_INVALID_ARG (as sfc_gemm_ex2, or a NULL output pointer),
  * SFC_ERR_CUDA, SFC_ERR_UNSUPPORTED.
  */
 int sfc_gemm_plan(int64_t M, int64_t N, int64_t K, int ca_c, int c_dtype, int tile,
-                  int *out_tile, int *out_ca_c);
+                  int ab_dtype, int b_layout, int *out_tile, int *out_ca_c);
 
 /*
  * sfc_release -- returns to the driver the device memory the library's

@@ -46,6 +46,13 @@
  *     matrix).  It is written independently of part 2: one dot product per
  *     output element (j-k loop order), then the two affine terms, in double.
  *
+ *  4. oracle_decode_f8 / oracle_gemm_f8_f64 -- the same products for 8-bit
+ *     float inputs (the method is independent of the data type, Sec. III):
+ *     each byte is decoded to its exact value from the format's definition
+ *     (e4m3: sign, 4 exponent bits with bias 7, 3 mantissa bits, no
+ *     infinities, S.1111.111 is NaN; e5m2: sign, 5 exponent bits with bias 15,
+ *     2 mantissa bits, IEEE-style infinities and NaNs), then summed in double.
+ *
  *  oracle_round_bf16 rounds a double to the nearest bf16 (ties to even) in a
  *  single step, used to compare bf16 outputs against the fp64 reference.
  */
@@ -220,6 +227,49 @@ void oracle_gemm_affine_f64(int64_t M, int64_t N, int64_t K,
             }
             if (C_in) dot += beta * C_in[i * ldcin + j];
             if (bias) dot += bias[j];
+            C[i * ldc + j] = dot;
+        }
+    }
+}
+
+/* ------------------------------------------------------------------------- */
+/* 4. 8-bit float inputs                                                      */
+/* ------------------------------------------------------------------------- */
+
+/* Exact value of an 8-bit float; fmt 1 = e4m3, 2 = e5m2. */
+double oracle_decode_f8(uint8_t code, int fmt)
+{
+    int sign = code >> 7;
+    int ebits = fmt == 1 ? 4 : 5;
+    int mbits = 7 - ebits;
+    int bias = fmt == 1 ? 7 : 15;
+    int e = (code >> mbits) & ((1 << ebits) - 1);
+    int m = code & ((1 << mbits) - 1);
+    double v;
+    if (fmt == 1 && e == 15 && m == 7) return NAN;
+    if (fmt == 2 && e == 31) v = (m == 0) ? INFINITY : NAN;
+    else if (e == 0) v = ldexp((double)m, 1 - bias - mbits);               /* subnormal */
+    else v = ldexp((double)((1 << mbits) + m), e - bias - mbits);          /* normal    */
+    return sign ? -v : v;
+}
+
+/* C[i*ldc + j] = sum_k A[i][k] * B(k, j) over 8-bit float inputs of format fmt,
+ * B(k, j) = B[k*ldb + j] (b_nk == 0) or B[j*ldb + k] (b_nk == 1). */
+void oracle_gemm_f8_f64(int64_t M, int64_t N, int64_t K,
+                        const uint8_t *A, int64_t lda,
+                        const uint8_t *B, int64_t ldb, int b_nk, int fmt,
+                        double *C, int64_t ldc)
+{
+    double table[256];
+    for (int c = 0; c < 256; ++c) table[c] = oracle_decode_f8((uint8_t)c, fmt);
+    #pragma omp parallel for schedule(static)
+    for (int64_t i = 0; i < M; ++i) {
+        for (int64_t j = 0; j < N; ++j) {
+            double dot = 0.0;
+            for (int64_t k = 0; k < K; ++k) {
+                uint8_t b = b_nk ? B[j * ldb + k] : B[k * ldb + j];
+                dot += table[A[i * lda + k]] * table[b];
+            }
             C[i * ldc + j] = dot;
         }
     }

@@ -63,6 +63,11 @@ def _load():
                                                ctypes.c_double, ctypes.c_void_p, i64, ctypes.c_void_p,
                                                ctypes.c_void_p, i64]
         lib.oracle_gemm_affine_f64.restype = None
+        lib.oracle_decode_f8.argtypes = [ctypes.c_uint8, ctypes.c_int]
+        lib.oracle_decode_f8.restype = ctypes.c_double
+        lib.oracle_gemm_f8_f64.argtypes = [i64, i64, i64, ctypes.c_void_p, i64, ctypes.c_void_p, i64, ctypes.c_int,
+                                           ctypes.c_int, ctypes.c_void_p, i64]
+        lib.oracle_gemm_f8_f64.restype = None
         lib.oracle_round_bf16.argtypes = [ctypes.c_double]
         lib.oracle_round_bf16.restype = ctypes.c_uint16
         lib.oracle_round_bf16_array.argtypes = [ctypes.c_void_p, i64, ctypes.c_void_p]
@@ -156,6 +161,45 @@ def gemm_affine_f64(A, B, *, b_layout: str = "kn", beta: float = 0.0, C_in=None,
     _load().oracle_gemm_affine_f64(M, N, K, a.ctypes.data, K, b.ctypes.data, b.shape[1], nk, float(beta),
                                    None if cin is None else cin.ctypes.data, N,
                                    None if bv is None else bv.ctypes.data, C.ctypes.data, N)
+    return C
+
+
+F8_FORMATS = {"e4m3": 1, "e5m2": 2}
+
+
+def decode_f8(code: int, fmt: str) -> float:
+    """Exact value of one 8-bit float code (0..255) of format "e4m3" or "e5m2"."""
+    return float(_load().oracle_decode_f8(int(code), F8_FORMATS[fmt]))
+
+
+def _f8_bytes(x) -> np.ndarray:
+    """Accept a torch float8 tensor or a uint8 array of codes."""
+    if hasattr(x, "dtype") and str(x.dtype).startswith("torch.float8"):
+        import torch
+        return x.detach().cpu().contiguous().view(torch.uint8).numpy()
+    arr = np.ascontiguousarray(x)
+    if arr.dtype != np.uint8:
+        raise TypeError("expected 8-bit float codes (uint8) or a torch float8 tensor")
+    return arr
+
+
+def gemm_f8_f64(A, B, fmt: str, *, b_layout: str = "kn") -> np.ndarray:
+    """C = A @ B in fp64 over 8-bit float inputs of format ``fmt`` ("e4m3" or
+    "e5m2"); B is K x N (``"kn"``) or its transpose N x K (``"nk"``)."""
+    a = _f8_bytes(A)
+    b = _f8_bytes(B)
+    M, K = a.shape
+    if b_layout == "kn":
+        K2, N = b.shape
+    elif b_layout == "nk":
+        N, K2 = b.shape
+    else:
+        raise ValueError("b_layout must be 'kn' or 'nk'")
+    if K != K2:
+        raise ValueError("inner dimensions differ")
+    C = np.empty((M, N), dtype=np.float64)
+    _load().oracle_gemm_f8_f64(M, N, K, a.ctypes.data, K, b.ctypes.data, b.shape[1], 1 if b_layout == "nk" else 0,
+                               F8_FORMATS[fmt], C.ctypes.data, N)
     return C
 
 

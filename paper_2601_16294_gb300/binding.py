@@ -30,6 +30,18 @@ ASSIGNS = {"segment": 0, "wave": 1, "auto": 2, "wave_static": 3}
 TILES = {0: 0, "auto": 0, 128: 128, 256: 256, "pair128": 1128, "pair256": 1256, "quad256": 2256}
 B_LAYOUTS = {"kn": 0, "nk": 1}
 
+
+def _ab_code(dtype) -> int:
+    """sfc_ab_t of a torch dtype of A and B."""
+    import torch
+    codes = {torch.bfloat16: 0}
+    for name, code in (("float8_e4m3fn", 1), ("float8_e5m2", 2)):
+        if hasattr(torch, name):
+            codes[getattr(torch, name)] = code
+    if dtype not in codes:
+        raise TypeError("A and B must be bfloat16, float8_e4m3fn or float8_e5m2 (got %s)" % dtype)
+    return codes[dtype]
+
 EXPORTS = ("sfc_tile_order", "sfc_tile_order_device", "sfc_gemm_workspace_size", "sfc_gemm", "sfc_gemm_ex",
            "sfc_get_device_status", "sfc_last_cuda_error", "sfc_num_workers", "sfc_debug_force_timeout",
            "sfc_gemm_noalloc", "sfc_gemm_plan", "sfc_release", "sfc_gemm_ex2")
@@ -81,9 +93,9 @@ def load():
         lib.sfc_num_workers.argtypes = []
         lib.sfc_debug_force_timeout.argtypes = [vp, vp, vp, i32, vp]
         lib.sfc_gemm_noalloc.argtypes = [i64, i64, i64, vp, vp, vp, i64, i64, i64, i32, i32, vp]
-        lib.sfc_gemm_plan.argtypes = [i64, i64, i64, i32, i32, i32, vp, vp]
-        lib.sfc_gemm_ex2.argtypes = [i64, i64, i64, vp, vp, vp, i64, i64, i64, i32, ctypes.c_float, vp, i32, i32,
-                                     i32, i32, i32, vp, sz, vp]
+        lib.sfc_gemm_plan.argtypes = [i64, i64, i64, i32, i32, i32, i32, i32, vp, vp]
+        lib.sfc_gemm_ex2.argtypes = [i64, i64, i64, vp, vp, vp, i64, i64, i64, i32, i32, ctypes.c_float, vp, i32,
+                                     i32, i32, i32, i32, vp, sz, vp]
         lib.sfc_release.argtypes = []
         for name in EXPORTS:
             if name != "sfc_gemm_workspace_size":
@@ -128,15 +140,18 @@ def workspace_size(M: int, N: int, K: int, ca_c: int) -> int:
     return int(load().sfc_gemm_workspace_size(int(M), int(N), int(K), int(ca_c)))
 
 
-def plan(M: int, N: int, K: int, ca_c: int = 0, out_dtype=None, tile="auto"):
+def plan(M: int, N: int, K: int, ca_c: int = 0, out_dtype=None, tile="auto", in_dtype=None,
+         b_layout: str = "kn"):
     """(tile, ca_c) the library would use for this call on the current device;
-    tile is a key of TILES other than "auto"."""
+    tile is a key of TILES other than "auto".  in_dtype: the dtype of A and B
+    (bfloat16 when None)."""
     import torch
     t = ctypes.c_int(0)
     c = ctypes.c_int(0)
     dt = SFC_BF16 if out_dtype == torch.bfloat16 else SFC_F32
-    _check(load().sfc_gemm_plan(int(M), int(N), int(K), int(ca_c), dt, TILES[tile], ctypes.byref(t),
-                                ctypes.byref(c)), "sfc_gemm_plan")
+    ab = _ab_code(in_dtype or torch.bfloat16)
+    _check(load().sfc_gemm_plan(int(M), int(N), int(K), int(ca_c), dt, TILES[tile], ab, B_LAYOUTS[b_layout],
+                                ctypes.byref(t), ctypes.byref(c)), "sfc_gemm_plan")
     name = {v: k for k, v in TILES.items() if k not in (0, "auto")}[t.value]
     return name, c.value
 
@@ -161,9 +176,10 @@ def _row_major_2d(t, name):
 
 def gemm(A, B, C=None, *, ca_c: int = 1, out_dtype=None, order: str = "sfc", assign: str = "auto",
          tile=0, workspace=None, stream=None, b_layout: str = "kn", beta: float = 0.0, bias=None):
-    """C = A @ B (+ beta * C + bias) on the GPU.  A: (M, K) bf16 CUDA tensor,
-    row-major (row stride may be padded).  B: bf16, (K, N) for ``b_layout="kn"``
-    or its transpose (N, K) for ``"nk"`` (a linear layer's weight).  C: (M, N)
+    """C = A @ B (+ beta * C + bias) on the GPU.  A: (M, K) CUDA tensor, bf16
+    or an 8-bit float (float8_e4m3fn, float8_e5m2), row-major (row stride may
+    be padded).  B: the same dtype, (K, N) for ``b_layout="kn"`` or its
+    transpose (N, K) for ``"nk"`` (a linear layer's weight).  C: (M, N)
     fp32 or bf16 CUDA tensor, allocated if not given (then ``beta`` must be 0).
     ``bias``: optional fp32 CUDA tensor of N values.  ``ca_c``: K layers (0: the
     library chooses).  ``workspace``: optional CUDA tensor of at least
@@ -179,8 +195,9 @@ def gemm(A, B, C=None, *, ca_c: int = 1, out_dtype=None, order: str = "sfc", ass
         raise ValueError("b_layout must be 'kn' or 'nk'")
     if K != K2:
         raise ValueError("inner dimensions differ: %d vs %d" % (K, K2))
-    if A.dtype != torch.bfloat16 or B.dtype != torch.bfloat16:
-        raise TypeError("A and B must be bfloat16")
+    if A.dtype != B.dtype:
+        raise TypeError("A and B must have the same dtype")
+    ab = _ab_code(A.dtype)
     if C is None:
         if beta != 0.0:
             raise ValueError("beta != 0 needs an input C")
@@ -199,7 +216,7 @@ def gemm(A, B, C=None, *, ca_c: int = 1, out_dtype=None, order: str = "sfc", ass
     if workspace is not None:
         ws_ptr, ws_bytes = ctypes.c_void_p(workspace.data_ptr()), workspace.numel() * workspace.element_size()
     rc = lib.sfc_gemm_ex2(M, N, K, ctypes.c_void_p(A.data_ptr()), ctypes.c_void_p(B.data_ptr()),
-                          ctypes.c_void_p(C.data_ptr()), lda, ldb, ldc, B_LAYOUTS[b_layout], float(beta), bias_ptr,
+                          ctypes.c_void_p(C.data_ptr()), lda, ldb, ldc, ab, B_LAYOUTS[b_layout], float(beta), bias_ptr,
                           int(ca_c), SFC_F32 if C.dtype == torch.float32 else SFC_BF16, ORDERS[order],
                           ASSIGNS[assign], TILES[tile], ws_ptr, ws_bytes, _stream_ptr(stream))
     _check(rc, "sfc_gemm_ex2")

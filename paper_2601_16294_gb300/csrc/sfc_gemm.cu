@@ -47,23 +47,21 @@ constexpr int variant_cluster(int v) { return v == kQuad256 ? 4 : (variant_pair(
 constexpr int variant_bm(int v) { return v == kQuad256 ? 512 : (variant_pair(v) ? 256 : 128); }
 
 template <int BN, int STAGES>
-constexpr int single_smem() { return RingLayout<(kBM + BN) * kBK * 2, STAGES, BN / 32>::kDynamicBytes; }
+constexpr int single_smem() { return RingLayout<(kBM + BN) * 128, STAGES, BN / 32>::kDynamicBytes; }
 template <int BN, int STAGES>
 constexpr int pair_smem() { return RingLayout<PairStage<BN>::kBytes, STAGES, BN / 32>::kDynamicBytes; }
 
-template <typename OutT>
+// Kernel of each variant for one output type and input kind (F8: 8-bit float
+// inputs; their table has no quad kernel, so its entry repeats pair256).
+template <typename OutT, bool F8>
 struct Kernels {
-    static constexpr void (*single128)(CUtensorMap, CUtensorMap, CUtensorMap, GemmParams) =
-        sfc_gemm_kernel<128, kStagesSingle128, OutT>;
-    static constexpr void (*single256)(CUtensorMap, CUtensorMap, CUtensorMap, GemmParams) =
-        sfc_gemm_kernel<256, kStagesSingle256, OutT>;
-    static constexpr void (*pair128)(CUtensorMap, CUtensorMap, CUtensorMap, GemmParams) =
-        sfc_gemm_pair_kernel<128, kStagesPair128, OutT, false>;
-    static constexpr void (*pair256)(CUtensorMap, CUtensorMap, CUtensorMap, GemmParams) =
-        sfc_gemm_pair_kernel<256, kStagesPair256, OutT, false>;
-    static constexpr void (*quad256)(CUtensorMap, CUtensorMap, CUtensorMap, GemmParams) =
-        sfc_gemm_pair_kernel<256, kStagesPair256, OutT, true>;
-    static void (*get(int v))(CUtensorMap, CUtensorMap, CUtensorMap, GemmParams) {
+    using Fn = void (*)(CUtensorMap, CUtensorMap, CUtensorMap, GemmParams);
+    static constexpr Fn single128 = sfc_gemm_kernel<128, kStagesSingle128, OutT, F8>;
+    static constexpr Fn single256 = sfc_gemm_kernel<256, kStagesSingle256, OutT, F8>;
+    static constexpr Fn pair128 = sfc_gemm_pair_kernel<128, kStagesPair128, OutT, false, F8>;
+    static constexpr Fn pair256 = sfc_gemm_pair_kernel<256, kStagesPair256, OutT, false, F8>;
+    static constexpr Fn quad256 = F8 ? pair256 : sfc_gemm_pair_kernel<256, kStagesPair256, OutT, !F8, false>;
+    static Fn get(int v) {
         switch (v) {
             case kSingle128: return single128;
             case kSingle256: return single256;
@@ -125,11 +123,11 @@ int current_device(int* dev) {
     return SFC_OK;
 }
 
-template <typename OutT>
+template <typename OutT, bool F8>
 cudaError_t set_attrs() {
     for (int v = 0; v < kNumVariants; ++v) {
-        cudaError_t e = cudaFuncSetAttribute(Kernels<OutT>::get(v), cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             variant_smem(v));
+        cudaError_t e = cudaFuncSetAttribute(Kernels<OutT, F8>::get(v),
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, variant_smem(v));
         if (e != cudaSuccess) return e;
     }
     return cudaSuccess;
@@ -159,8 +157,10 @@ int device_setup(DeviceInfo** info) {
         // experiment override: launch one block (pair) per item instead of one per SM, so the
         // hardware dispatches the items in curve order as SMs free up
         if (const char* env = std::getenv("SFC_GEMM_ONE_ITEM_PER_WORKER")) d.one_item_per_worker = std::atoi(env) != 0;
-        e = set_attrs<float>();
-        if (e == cudaSuccess) e = set_attrs<__nv_bfloat16>();
+        e = set_attrs<float, false>();
+        if (e == cudaSuccess) e = set_attrs<__nv_bfloat16, false>();
+        if (e == cudaSuccess) e = set_attrs<float, true>();
+        if (e == cudaSuccess) e = set_attrs<__nv_bfloat16, true>();
         if (e != cudaSuccess) { d.status = cuda_fail(e); return; }
         for (int v = 0; v < kNumVariants; ++v) {
             if (!variant_pair(v)) {
@@ -170,7 +170,7 @@ int device_setup(DeviceInfo** info) {
             cudaLaunchAttribute attr[2];
             cudaLaunchConfig_t cfg = launch_config(v, d.num_sms, nullptr, attr, false);
             int clusters = 0;
-            e = cudaOccupancyMaxActiveClusters(&clusters, Kernels<float>::get(v), &cfg);
+            e = cudaOccupancyMaxActiveClusters(&clusters, Kernels<float, false>::get(v), &cfg);
             if (e != cudaSuccess) { d.status = cuda_fail(e); return; }
             d.workers[v] = clusters;
         }
@@ -198,18 +198,20 @@ int get_encoder(PFN_cuTensorMapEncodeTiled_v12000* fn) {
     return g_encode ? SFC_OK : SFC_ERR_UNSUPPORTED;
 }
 
-// Row-major bf16 matrix rows x cols with row stride ld (elements), boxes of
-// box_rows x box_cols with 128-byte swizzle; out-of-range elements read as 0.
-int make_bf16_map(CUtensorMap* map, const void* ptr, int64_t rows, int64_t cols, int64_t ld,
-                  uint32_t box_rows, uint32_t box_cols) {
+// Row-major input matrix (bf16, or 8-bit floats with elem_bytes 1) rows x cols
+// with row stride ld (elements), boxes of box_rows x box_cols with 128-byte
+// swizzle; out-of-range elements read as 0.
+int make_in_map(CUtensorMap* map, const void* ptr, int64_t rows, int64_t cols, int64_t ld, int elem_bytes,
+                uint32_t box_rows, uint32_t box_cols) {
     PFN_cuTensorMapEncodeTiled_v12000 encode;
     int rc = get_encoder(&encode);
     if (rc != SFC_OK) return rc;
     cuuint64_t dims[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(rows)};
-    cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * 2};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(ld) * elem_bytes};
     cuuint32_t box[2] = {box_cols, box_rows};
     cuuint32_t estr[2] = {1, 1};
-    CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(ptr), dims, strides, box,
+    const CUtensorMapDataType dt = elem_bytes == 1 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16;
+    CUresult r = encode(map, dt, 2, const_cast<void*>(ptr), dims, strides, box,
                         estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) {
@@ -269,19 +271,24 @@ constexpr double kEff[kNumVariants] = {0.50, 0.85, 0.55, 0.95, 0.90};
 // Layers ca_c = 0 may choose: enough to give about 320 items of 128 x 128,
 // never more than 64 or the number of K slabs (host-only, so the workspace
 // bound below needs no device).
-int64_t auto_layer_cap(int64_t M, int64_t N, int64_t K) {
+// K values per 128-byte slab row: 64 bf16, 128 8-bit floats.
+constexpr int slab_k(int ab) { return ab == SFC_AB_BF16 ? kBK : 2 * kBK; }
+constexpr int in_bytes(int ab) { return ab == SFC_AB_BF16 ? 2 : 1; }
+
+int64_t auto_layer_cap(int64_t M, int64_t N, int64_t K, int ab = SFC_AB_BF16) {
     const int64_t tiles = ceil_div(M, kBM) * ceil_div(N, 128);
     int64_t cap = ceil_div(320, tiles);
-    const int64_t Kt = ceil_div(K, kBK);
+    const int64_t Kt = ceil_div(K, slab_k(ab));
     if (cap > Kt) cap = Kt;
     if (cap > 64) cap = 64;
     return cap < 1 ? 1 : cap;
 }
 
-double plan_cost(int64_t M, int64_t N, int64_t K, int c, int v, const DeviceInfo& d, int out_bytes) {
+double plan_cost(int64_t M, int64_t N, int64_t K, int c, int v, const DeviceInfo& d, int out_bytes, int ab) {
     const int64_t items = ceil_div(M, variant_bm(v)) * ceil_div(N, variant_bn(v)) * c;
     const int64_t waves = ceil_div(items, d.workers[v]);
-    const int64_t slabs = ceil_div(ceil_div(K, kBK), c);
+    // a slab of 8-bit inputs holds twice the k at twice the rate: the same time per slab
+    const int64_t slabs = ceil_div(ceil_div(K, slab_k(ab)), c);
     const double slab_ns = 128.0 * variant_bn(v) * kBK * 2.0 / (8192.0 * kEff[v]) / kSlabClockGhz;
     double t = static_cast<double>(waves) * static_cast<double>(slabs) * slab_ns;
     if (c > 1)
@@ -298,11 +305,20 @@ struct Plan {
 // ca_c >= 1: the variant for it; ca_c = 0: the best (variant, c) with c up to
 // max_c.  A requested tile fixes the variant (falling back to one SM when
 // pairs cannot be co-scheduled).
+// Variants that can serve a call: the quad variant takes bf16 with N-major B
+// only; 8-bit N-major B needs 128-byte (128-column) boxes per CTA, which the
+// 256 x 128 pair tile (64 columns per CTA) does not have.
+bool variant_allowed(int v, bool b_kmajor, int ab) {
+    if (v == kQuad256) return !b_kmajor && ab == SFC_AB_BF16;
+    if (v == kPair128 && ab != SFC_AB_BF16 && !b_kmajor) return false;
+    return true;
+}
+
 Plan make_plan(int64_t M, int64_t N, int64_t K, int ca_c, int max_c, const DeviceInfo& d, sfc_tile_t tile,
-               int out_bytes, bool b_kmajor = false) {
+               int out_bytes, bool b_kmajor = false, int ab = SFC_AB_BF16) {
     int fixed = -1;
-    // the quad variant splits the B slab along K between its pairs, which needs N-major B
-    if (b_kmajor && tile == SFC_TILE_QUAD_N256) tile = SFC_TILE_PAIR_N256;
+    if (tile == SFC_TILE_QUAD_N256 && !variant_allowed(kQuad256, b_kmajor, ab)) tile = SFC_TILE_PAIR_N256;
+    if (tile == SFC_TILE_PAIR_N128 && !variant_allowed(kPair128, b_kmajor, ab)) tile = SFC_TILE_N128;
     switch (tile) {
         case SFC_TILE_N128: fixed = kSingle128; break;
         case SFC_TILE_N256: fixed = kSingle256; break;
@@ -315,9 +331,9 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, int ca_c, int max_c, const Devic
     double best_t = -1.0;
     const int c_lo = ca_c > 0 ? ca_c : 1, c_hi = ca_c > 0 ? ca_c : max_c;
     for (int v = 0; v < kNumVariants; ++v) {
-        if (d.workers[v] <= 0 || (fixed >= 0 && v != fixed) || (b_kmajor && v == kQuad256)) continue;
+        if (d.workers[v] <= 0 || (fixed >= 0 && v != fixed) || !variant_allowed(v, b_kmajor, ab)) continue;
         for (int c = c_lo; c <= c_hi; ++c) {
-            const double t = plan_cost(M, N, K, c, v, d, out_bytes);
+            const double t = plan_cost(M, N, K, c, v, d, out_bytes, ab);
             if (best_t < 0.0 || t < best_t) {  // ties keep fewer layers, then the earlier variant
                 best = Plan{v, c};
                 best_t = t;
@@ -331,9 +347,10 @@ bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) ==
 
 int validate(int64_t M, int64_t N, int64_t K, const void* A, const void* B, const void* C, int64_t lda,
              int64_t ldb, int64_t ldc, int ca_c, int c_dtype, int order, int assign, int tile,
-             int b_layout = SFC_B_KN) {
+             int b_layout = SFC_B_KN, int ab = SFC_AB_BF16) {
     if (M <= 0 || N <= 0 || K <= 0 || !A || !B || !C) return SFC_ERR_INVALID_ARG;
     if (b_layout != SFC_B_KN && b_layout != SFC_B_NK) return SFC_ERR_INVALID_ARG;
+    if (ab != SFC_AB_BF16 && ab != SFC_AB_E4M3 && ab != SFC_AB_E5M2) return SFC_ERR_INVALID_ARG;
     if (lda < K || ldb < (b_layout == SFC_B_NK ? K : N) || ldc < N) return SFC_ERR_INVALID_ARG;
     if (c_dtype != SFC_F32 && c_dtype != SFC_BF16) return SFC_ERR_INVALID_ARG;
     if (order != SFC_ORDER_SFC && order != SFC_ORDER_RASTER) return SFC_ERR_INVALID_ARG;
@@ -344,13 +361,15 @@ int validate(int64_t M, int64_t N, int64_t K, const void* A, const void* B, cons
         tile != SFC_TILE_PAIR_N256 && tile != SFC_TILE_QUAD_N256)
         return SFC_ERR_INVALID_ARG;
     // TMA coordinates and tile indices are 32-bit
-    if (M > (int64_t(1) << 31) - kBM || N > (int64_t(1) << 31) - 256 || K > (int64_t(1) << 31) - kBK)
+    if (M > (int64_t(1) << 31) - kBM || N > (int64_t(1) << 31) - 256 || K > (int64_t(1) << 31) - slab_k(ab))
         return SFC_ERR_INVALID_ARG;
-    const int64_t Kt = ceil_div(K, kBK);
+    const int64_t Kt = ceil_div(K, slab_k(ab));
     if (ca_c < 0 || ca_c > Kt || ca_c > kMaxLayers) return SFC_ERR_INVALID_ARG;  // 0: chosen per call
-    const int64_t layers = ca_c > 0 ? ca_c : auto_layer_cap(M, N, K);
+    const int64_t layers = ca_c > 0 ? ca_c : auto_layer_cap(M, N, K, ab);
     if (ceil_div(M, kBM) * ceil_div(N, 128) * layers > (int64_t(1) << 31) - 1) return SFC_ERR_INVALID_ARG;
-    if (!aligned16(A) || !aligned16(B) || (lda % 8) != 0 || (ldb % 8) != 0) return SFC_ERR_UNALIGNED;
+    // the tile loads use the Tensor Memory Accelerator: 16-byte rows and bases
+    const int64_t row_align = 16 / in_bytes(ab);
+    if (!aligned16(A) || !aligned16(B) || (lda % row_align) != 0 || (ldb % row_align) != 0) return SFC_ERR_UNALIGNED;
     if (lda >= (int64_t(1) << 39) || ldb >= (int64_t(1) << 39)) return SFC_ERR_INVALID_ARG;
     return SFC_OK;
 }
@@ -358,20 +377,23 @@ int validate(int64_t M, int64_t N, int64_t K, const void* A, const void* B, cons
 int64_t ws_ld(int64_t N) { return (N + 3) / 4 * 4; }
 
 template <typename OutT>
-cudaError_t launch_gemm(int v, const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc,
+cudaError_t launch_gemm(int v, bool f8, const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc,
                         const GemmParams& p, int grid, cudaStream_t s) {
     cudaLaunchAttribute attr[2];
     cudaLaunchConfig_t cfg = launch_config(v, grid, s, attr, true);
-    cudaError_t e = cudaLaunchKernelEx(&cfg, Kernels<OutT>::get(v), ta, tb, tc, p);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, f8 ? Kernels<OutT, true>::get(v) : Kernels<OutT, false>::get(v), ta, tb,
+                                       tc, p);
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void* C, int64_t lda, int64_t ldb,
              int64_t ldc, int ca_c, int c_dtype, int order, int assign, int tile, void* workspace,
              size_t workspace_bytes, cudaStream_t stream, int debug_never, uint64_t timeout_ns,
-             int b_layout = SFC_B_KN, float beta = 0.0f, const float* bias = nullptr) {
-    int rc = validate(M, N, K, A, B, C, lda, ldb, ldc, ca_c, c_dtype, order, assign, tile, b_layout);
+             int b_layout = SFC_B_KN, float beta = 0.0f, const float* bias = nullptr, int ab = SFC_AB_BF16) {
+    int rc = validate(M, N, K, A, B, C, lda, ldb, ldc, ca_c, c_dtype, order, assign, tile, b_layout, ab);
     if (rc != SFC_OK) return rc;
+    const bool f8 = (ab != SFC_AB_BF16);
+    const int sk = slab_k(ab), eb = in_bytes(ab);
     if (bias && (reinterpret_cast<uintptr_t>(bias) & 3u) != 0) return SFC_ERR_UNALIGNED;
     const bool b_kmajor = (b_layout == SFC_B_NK);
     if (ca_c > 0 && workspace && workspace_bytes < sfc_gemm_workspace_size(M, N, K, ca_c)) return SFC_ERR_WORKSPACE;
@@ -382,24 +404,25 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     if (rc != SFC_OK) return rc;
 
     // ca_c = 0: the planner's layer count, within the caller's workspace if one is given
-    int max_c = static_cast<int>(auto_layer_cap(M, N, K));
+    int max_c = static_cast<int>(auto_layer_cap(M, N, K, ab));
     while (ca_c == 0 && workspace && max_c > 1 && workspace_bytes < sfc_gemm_workspace_size(M, N, K, max_c)) --max_c;
-    const Plan plan =
-        make_plan(M, N, K, ca_c, max_c, *dev, static_cast<sfc_tile_t>(tile), c_dtype == SFC_F32 ? 4 : 2, b_kmajor);
+    const Plan plan = make_plan(M, N, K, ca_c, max_c, *dev, static_cast<sfc_tile_t>(tile), c_dtype == SFC_F32 ? 4 : 2,
+                                b_kmajor, ab);
     const int v = plan.v;
     ca_c = plan.c;
     const size_t ws_need = sfc_gemm_workspace_size(M, N, K, ca_c);
     const int bn = variant_bn(v);
     const int bm = variant_bm(v);
     CUtensorMap ta, tb;
-    rc = make_bf16_map(&ta, A, M, K, lda, kBM, kBK);  // each CTA loads 128 rows of A
+    rc = make_in_map(&ta, A, M, K, lda, eb, kBM, sk);  // each CTA loads 128 rows of A, one slab of k
     if (rc != SFC_OK) return rc;
     if (b_kmajor) {
-        // B given as N x K: boxes of (this CTA's share of the tile's N rows) x 64 k, like A
-        rc = make_bf16_map(&tb, B, N, K, ldb, variant_pair(v) ? bn / 2 : bn, kBK);
+        // B given as N x K: boxes of (this CTA's share of the tile's N rows) x one slab of k, like A
+        rc = make_in_map(&tb, B, N, K, ldb, eb, variant_pair(v) ? bn / 2 : bn, sk);
     } else {
-        // B boxes: 64 K rows x 64 columns; with two pairs sharing B each CTA loads 32 K rows
-        rc = make_bf16_map(&tb, B, K, N, ldb, v == kQuad256 ? kBK / 2 : kBK, kBBox);
+        // N-major B boxes: one slab of k rows x 128 bytes of columns; with two pairs
+        // sharing B each CTA loads half the slab's rows
+        rc = make_in_map(&tb, B, K, N, ldb, eb, v == kQuad256 ? sk / 2 : sk, 128 / eb);
     }
     if (rc != SFC_OK) return rc;
 
@@ -408,7 +431,7 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     p.N = N;
     p.Mt = static_cast<int>(ceil_div(M, bm));
     p.Nt = static_cast<int>(ceil_div(N, bn));
-    p.Kt = static_cast<int>(ceil_div(K, kBK));
+    p.Kt = static_cast<int>(ceil_div(K, sk));
     p.ca_c = ca_c;
     p.grid_tiles = p.Mt * p.Nt;
     p.kq = p.Kt / ca_c;
@@ -428,6 +451,7 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     p.c_in = C;
     p.ldc_in = ldc;
     p.bias = bias;
+    p.ab_fmt = (ab == SFC_AB_E4M3) ? 0 : 1;  // bf16 (kind::f16) and e5m2 (kind::f8f6f4) are both code 1
     const int64_t workers = dev->one_item_per_worker ? p.num_items : dev->workers[v];
     const int64_t used = p.num_items < workers ? p.num_items : workers;
     const int grid = static_cast<int>(variant_cluster(v) * used);
@@ -450,15 +474,15 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
         const int esz = (c_dtype == SFC_F32) ? 4 : 2;
         p.vec_store = aligned16(C) && ((ldc * esz) % 16 == 0);
         p.tma_store = p.vec_store && make_out_map(&tc, C, M, N, ldc, esz, 1) == SFC_OK;
-        e = (c_dtype == SFC_F32) ? launch_gemm<float>(v, ta, tb, tc, p, grid, stream)
-                                 : launch_gemm<__nv_bfloat16>(v, ta, tb, tc, p, grid, stream);
+        e = (c_dtype == SFC_F32) ? launch_gemm<float>(v, f8, ta, tb, tc, p, grid, stream)
+                                 : launch_gemm<__nv_bfloat16>(v, f8, ta, tb, tc, p, grid, stream);
     } else {
         p.out = ws;
         p.ldo = ws_ld(N);
         p.layer_stride = M * p.ldo;
         p.vec_store = 1;
         p.tma_store = make_out_map(&tc, ws, M, N, p.ldo, 4, ca_c) == SFC_OK;
-        e = launch_gemm<float>(v, ta, tb, tc, p, grid, stream);
+        e = launch_gemm<float>(v, f8, ta, tb, tc, p, grid, stream);
         if (e == cudaSuccess) {
             const int64_t work = M * ((N + 3) / 4);
             int64_t blocks = ceil_div(work, 256);
@@ -531,18 +555,20 @@ SFC_API size_t sfc_gemm_workspace_size(int64_t M, int64_t N, int64_t K, int ca_c
     return static_cast<size_t>(layers) * static_cast<size_t>(M) * static_cast<size_t>(ws_ld(N)) * 4u;
 }
 
-SFC_API int sfc_gemm_plan(int64_t M, int64_t N, int64_t K, int ca_c, int c_dtype, int tile, int* out_tile,
-                          int* out_ca_c) {
+SFC_API int sfc_gemm_plan(int64_t M, int64_t N, int64_t K, int ca_c, int c_dtype, int tile, int ab_dtype,
+                          int b_layout, int* out_tile, int* out_ca_c) {
     if (!out_tile || !out_ca_c) return SFC_ERR_INVALID_ARG;
+    const int64_t kp = K + (16 - K % 16) % 16, np = N + (16 - N % 16) % 16;  // strides that pass the checks
     int rc = validate(M, N, K, reinterpret_cast<const void*>(16), reinterpret_cast<const void*>(16),
-                      reinterpret_cast<const void*>(16), K + (8 - K % 8) % 8, N + (8 - N % 8) % 8, N, ca_c,
-                      c_dtype, SFC_ORDER_SFC, SFC_ASSIGN_AUTO, tile);
+                      reinterpret_cast<const void*>(16), kp, b_layout == SFC_B_NK ? kp : np, N, ca_c, c_dtype,
+                      SFC_ORDER_SFC, SFC_ASSIGN_AUTO, tile, b_layout, ab_dtype);
     if (rc != SFC_OK) return rc;
     DeviceInfo* dev = nullptr;
     rc = device_setup(&dev);
     if (rc != SFC_OK) return rc;
-    const Plan plan = make_plan(M, N, K, ca_c, static_cast<int>(auto_layer_cap(M, N, K)), *dev,
-                                static_cast<sfc_tile_t>(tile), c_dtype == SFC_F32 ? 4 : 2);
+    const Plan plan = make_plan(M, N, K, ca_c, static_cast<int>(auto_layer_cap(M, N, K, ab_dtype)), *dev,
+                                static_cast<sfc_tile_t>(tile), c_dtype == SFC_F32 ? 4 : 2, b_layout == SFC_B_NK,
+                                ab_dtype);
     static const int kTileOf[kNumVariants] = {SFC_TILE_N128, SFC_TILE_N256, SFC_TILE_PAIR_N128, SFC_TILE_PAIR_N256,
                                               SFC_TILE_QUAD_N256};
     *out_tile = kTileOf[plan.v];
@@ -578,11 +604,12 @@ SFC_API int sfc_gemm_ex(int64_t M, int64_t N, int64_t K, const void* A, const vo
 }
 
 SFC_API int sfc_gemm_ex2(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void* C, int64_t lda,
-                         int64_t ldb, int64_t ldc, int b_layout, float beta, const float* bias, int ca_c,
-                         sfc_dtype_t c_dtype, sfc_order_t order, sfc_assign_t assign, sfc_tile_t tile,
+                         int64_t ldb, int64_t ldc, int ab_dtype, int b_layout, float beta, const float* bias,
+                         int ca_c, sfc_dtype_t c_dtype, sfc_order_t order, sfc_assign_t assign, sfc_tile_t tile,
                          void* workspace, size_t workspace_bytes, void* stream) {
     return run_gemm(M, N, K, A, B, C, lda, ldb, ldc, ca_c, c_dtype, order, assign, tile, workspace,
-                    workspace_bytes, static_cast<cudaStream_t>(stream), 0, kDefaultTimeoutNs, b_layout, beta, bias);
+                    workspace_bytes, static_cast<cudaStream_t>(stream), 0, kDefaultTimeoutNs, b_layout, beta, bias,
+                    ab_dtype);
 }
 
 SFC_API int sfc_get_device_status(void* stream) {

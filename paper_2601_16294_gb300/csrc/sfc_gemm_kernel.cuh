@@ -45,10 +45,19 @@
 namespace sfc {
 
 constexpr int kBM = 128;          // output tile rows per CTA (UMMA M of one CTA)
-constexpr int kBK = 64;           // K slab: 64 bf16 = one 128-byte swizzle row
-constexpr int kUmmaK = 16;        // K per tcgen05.mma for 16-bit inputs
-constexpr int kBBox = 64;         // B is loaded in 64-column boxes (128 bytes)
+constexpr int kBK = 64;           // K slab of bf16 inputs: 64 values = one 128-byte swizzle row
 constexpr int kEpiCols = 128;     // accumulator columns each epilogue thread owns
+
+// Per input kind (bf16, or 8-bit floats with F8): the K values of one
+// 128-byte shared-memory row (a slab), of one tcgen05.mma, and the columns of
+// an N-major B box (also 128 bytes).  Every stage row is 128 bytes either way.
+template <bool F8>
+struct InKind {
+    static constexpr int kSlabK = F8 ? 128 : 64;
+    static constexpr int kMmaK = F8 ? 32 : 16;
+    static constexpr int kBCols = F8 ? 128 : 64;
+    static constexpr int kBBoxBytes = kSlabK * 128;  // one N-major box: slab rows x 128 bytes
+};
 
 // Threads of a block: producer warp, MMA warp, BN/32 epilogue warps
 // (4 warps per 128 columns: one warp per TMEM lane quarter), scheduler warp.
@@ -107,6 +116,7 @@ struct GemmParams {
     const void* c_in;      // C_in (the output array, read before it is written) when beta != 0
     int64_t ldc_in;        // its row stride in elements
     const float* bias;     // N fp32 values or null
+    int ab_fmt;            // A/B format code of the instruction descriptor (bf16: 1; e4m3: 0, e5m2: 1)
 };
 
 struct WorkItem {
@@ -566,18 +576,17 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
 // -------------------------------------------------------------------------
 // Single-SM kernel: 128 x BN tiles, UMMA 128 x BN x 16.
 // -------------------------------------------------------------------------
-template <int BN, int STAGES, typename OutT>
+template <int BN, int STAGES, typename OutT, bool F8>
 __global__ void __launch_bounds__(block_threads(BN), 1)
 sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_b,
                 const __grid_constant__ CUtensorMap tmap_c, const GemmParams p) {
     static_assert(BN == 128 || BN == 256, "tiles are 128 x 128 or 128 x 256");
-    constexpr int kABytes = kBM * kBK * 2;
-    constexpr int kBBytes = BN * kBK * 2;
+    using I = InKind<F8>;
+    constexpr int kABytes = kBM * 128;  // 128-byte rows
+    constexpr int kBBytes = BN * 128;
     constexpr int kStageBytes = kABytes + kBBytes;
     constexpr int kEpiWarps = BN / 32;
     using L = RingLayout<kStageBytes, STAGES, kEpiWarps>;
-    constexpr uint32_t kIdesc = ptx::idesc_bf16_f32(kBM, BN, /*A K-major*/ 0, /*B MN-major*/ 1);
-    constexpr uint32_t kIdescBK = ptx::idesc_bf16_f32(kBM, BN, /*A K-major*/ 0, /*B K-major*/ 0);
     constexpr uint32_t kTmemCols = 2 * BN;
 
     extern __shared__ uint8_t smem_raw[];
@@ -655,15 +664,15 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
                 ptx::mbar_arrive_expect_tx(B.full(stage), kStageBytes);
                 const uint32_t sa = ring + stage * kStageBytes;
                 const uint32_t sb = sa + kABytes;
-                ptx::tma_load_2d(sa, &tmap_a, B.full(stage), kt * kBK, w.tm * kBM);
+                ptx::tma_load_2d(sa, &tmap_a, B.full(stage), kt * I::kSlabK, w.tm * kBM);
                 if (p.b_kmajor) {
-                    // B^T rows (N) x 64 k, K-major like A
-                    ptx::tma_load_2d(sb, &tmap_b, B.full(stage), kt * kBK, w.tn * BN);
+                    // B^T rows (N) x one slab of k, K-major like A
+                    ptx::tma_load_2d(sb, &tmap_b, B.full(stage), kt * I::kSlabK, w.tn * BN);
                 } else {
 #pragma unroll
-                    for (int jb = 0; jb < BN / kBBox; ++jb)
-                        ptx::tma_load_2d(sb + jb * (kBBox * kBK * 2), &tmap_b, B.full(stage),
-                                         w.tn * BN + jb * kBBox, kt * kBK);
+                    for (int jb = 0; jb < BN / I::kBCols; ++jb)
+                        ptx::tma_load_2d(sb + jb * I::kBBoxBytes, &tmap_b, B.full(stage), w.tn * BN + jb * I::kBCols,
+                                         kt * I::kSlabK);
                 }
             });
             // Tail: the last STAGES issues.  On success wait until the MMA warp's
@@ -686,6 +695,7 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
             int acc = 0;
             uint32_t acc_phase = 0;
             bool ok = true;
+            const uint32_t idesc = ptx::idesc_f32(kBM, BN, /*A K-major*/ 0, p.b_kmajor ? 0u : 1u, p.ab_fmt);
             if (p.debug_never) ok = wait_bounded(B.never(), 0, abort_flag, p.timeout_ns, kWaitDebugNever);
             for (int j = 0; ok; ++j) {
                 WorkItem w;
@@ -712,16 +722,15 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
                         const uint32_t sa = ring + stage * kStageBytes;
                         const uint32_t sb = sa + kABytes;
 #pragma unroll
-                        for (int kk = 0; kk < kBK / kUmmaK; ++kk) {
-                            // A: K-major, 128-byte rows, 8-row atoms 1024 B apart; 32 B per K=16
-                            const uint64_t adesc = ptx::smem_desc_sw128(sa + kk * (kUmmaK * 2), 16, 1024);
-                            // B MN-major: 64-column boxes 8 KB apart, 8-row atoms 1 KB apart, 2 KB per
-                            // K=16; B K-major: as A
+                        for (int kk = 0; kk < I::kSlabK / I::kMmaK; ++kk) {
+                            // A: K-major, 128-byte rows, 8-row atoms 1024 B apart; 32 B per instruction
+                            const uint64_t adesc = ptx::smem_desc_sw128(sa + kk * 32, 16, 1024);
+                            // B N-major: 128-byte-wide boxes one box apart, 8-row atoms 1 KB apart,
+                            // kMmaK rows per instruction; B K-major: as A
                             const uint64_t bdesc = p.b_kmajor
-                                ? ptx::smem_desc_sw128(sb + kk * (kUmmaK * 2), 16, 1024)
-                                : ptx::smem_desc_sw128(sb + kk * (kUmmaK * 128), kBBox * kBK * 2, 1024);
-                            ptx::tc_mma_f16(d_tmem, adesc, bdesc, p.b_kmajor ? kIdescBK : kIdesc,
-                                            (q > kb || kk > 0) ? 1u : 0u);
+                                ? ptx::smem_desc_sw128(sb + kk * 32, 16, 1024)
+                                : ptx::smem_desc_sw128(sb + kk * (I::kMmaK * 128), I::kBBoxBytes, 1024);
+                            ptx::tc_mma<F8>(d_tmem, adesc, bdesc, idesc, (q > kb || kk > 0) ? 1u : 0u);
                         }
                         ptx::tc_commit(B.empty(stage));  // frees the stage once these MMAs finish
                         if (++stage == STAGES) {

@@ -40,23 +40,24 @@ constexpr int kPairBM = 256;  // output tile rows of a pair (128 per CTA)
 template <int BN>
 struct PairStage {
     static constexpr int kHalfN = BN / 2;
-    static constexpr int kABytes = 128 * kBK * 2;
-    static constexpr int kBBytes = kHalfN * kBK * 2;
+    static constexpr int kABytes = 128 * 128;     // 128 rows of 128 bytes
+    static constexpr int kBBytes = kHalfN * 128;  // this CTA's half of the B slab
     static constexpr int kBytes = kABytes + kBBytes;
     static_assert(kABytes % 1024 == 0 && kBBytes % 1024 == 0, "swizzle atoms need 1 KB alignment");
 };
 
-template <int BN, int STAGES, typename OutT, bool QUAD>
+template <int BN, int STAGES, typename OutT, bool QUAD, bool F8>
 __global__ void __launch_bounds__(block_threads(BN), 1)
 sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_b,
                      const __grid_constant__ CUtensorMap tmap_c, const GemmParams p) {
     static_assert(BN == 128 || BN == 256, "pair tiles are 256 x 128 or 256 x 256");
+    static_assert(!(QUAD && F8), "the quad variant takes bf16 inputs");
+    using I = InKind<F8>;
     using S = PairStage<BN>;
     constexpr int kEpiWarps = BN / 32;
     using L = RingLayout<S::kBytes, STAGES, kEpiWarps>;
     constexpr int kHalfN = S::kHalfN;
-    constexpr uint32_t kIdesc = ptx::idesc_bf16_f32(kPairBM, BN, /*A K-major*/ 0, /*B MN-major*/ 1);
-    constexpr uint32_t kIdescBK = ptx::idesc_bf16_f32(kPairBM, BN, /*A K-major*/ 0, /*B K-major*/ 0);
+
     constexpr uint32_t kTmemCols = 2 * BN;
     // QUAD: a cluster of two pairs stacked in M (a 512 x BN item) sharing the B slab
     constexpr int kCtas = QUAD ? 4 : 2;
@@ -151,24 +152,26 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
                 const uint32_t leader_full = ptx::map_to_cta(B.full(stage), pair_leader);
                 const uint32_t sa = ring + stage * S::kBytes;
                 const uint32_t sb = sa + S::kABytes;
-                ptx::tma_load_2d_pair(sa, &tmap_a, leader_full, kt * kBK, a_row);
+                ptx::tma_load_2d_pair(sa, &tmap_a, leader_full, kt * I::kSlabK, a_row);
                 if (!QUAD && p.b_kmajor) {
-                    // this CTA's half of the B^T rows (N) x 64 k, K-major like A
-                    ptx::tma_load_2d_pair(sb, &tmap_b, leader_full, kt * kBK, b_col);
+                    // this CTA's half of the B^T rows (N) x one slab of k, K-major like A
+                    ptx::tma_load_2d_pair(sb, &tmap_b, leader_full, kt * I::kSlabK, b_col);
                 } else if constexpr (QUAD) {
                     // the same B half-slab goes to this CTA and its counterpart in the
                     // other pair: each loads 32 of the 64 K rows for both
                     const uint16_t mask = static_cast<uint16_t>((1u << r) | (1u << (r + 2)));
 #pragma unroll
-                    for (int jb = 0; jb < kHalfN / kBBox; ++jb)
-                        ptx::tma_load_2d_pair_multicast(sb + jb * (kBBox * kBK * 2) + pair_idx * (32 * 128),
-                                                        &tmap_b, leader_full, b_col + jb * kBBox,
-                                                        kt * kBK + static_cast<int32_t>(pair_idx) * 32, mask);
+                    for (int jb = 0; jb < kHalfN / I::kBCols; ++jb)
+                        ptx::tma_load_2d_pair_multicast(sb + jb * I::kBBoxBytes + pair_idx * (I::kSlabK / 2 * 128),
+                                                        &tmap_b, leader_full, b_col + jb * I::kBCols,
+                                                        kt * I::kSlabK + static_cast<int32_t>(pair_idx) * (I::kSlabK / 2),
+                                                        mask);
                 } else {
+                    // N-major boxes of 128-byte rows (the host keeps 8-bit inputs with BN/2 >= 128 here)
 #pragma unroll
-                    for (int jb = 0; jb < kHalfN / kBBox; ++jb)
-                        ptx::tma_load_2d_pair(sb + jb * (kBBox * kBK * 2), &tmap_b, leader_full, b_col + jb * kBBox,
-                                              kt * kBK);
+                    for (int jb = 0; jb < kHalfN / I::kBCols; ++jb)
+                        ptx::tma_load_2d_pair(sb + jb * I::kBBoxBytes, &tmap_b, leader_full, b_col + jb * I::kBCols,
+                                              kt * I::kSlabK);
                 }
             });
             // Tail: on success wait until the last STAGES issues are released
@@ -200,6 +203,8 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
             int acc = 0;
             uint32_t acc_phase = 0;
             bool ok = true;
+            const bool bk = !QUAD && p.b_kmajor;
+            const uint32_t idesc = ptx::idesc_f32(kPairBM, BN, /*A K-major*/ 0, bk ? 0u : 1u, p.ab_fmt);
             if (p.debug_never) ok = wait_bounded(B.never(), 0, abort_flag, p.timeout_ns, kWaitDebugNever);
             for (int j = 0; ok; ++j) {
                 WorkItem w;
@@ -226,16 +231,15 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
                         const uint32_t sa = ring + stage * S::kBytes;
                         const uint32_t sb = sa + S::kABytes;
 #pragma unroll
-                        for (int kk = 0; kk < kBK / kUmmaK; ++kk) {
-                            // A half: K-major, 128-byte rows, 8-row atoms 1 KB apart; 32 B per K=16
-                            const uint64_t adesc = ptx::smem_desc_sw128(sa + kk * (kUmmaK * 2), 16, 1024);
-                            // B half MN-major: 64-column boxes 8 KB apart, 2 KB per K=16; K-major: as A
-                            const bool bk = !QUAD && p.b_kmajor;
+                        for (int kk = 0; kk < I::kSlabK / I::kMmaK; ++kk) {
+                            // A half: K-major, 128-byte rows, 8-row atoms 1 KB apart; 32 B per instruction
+                            const uint64_t adesc = ptx::smem_desc_sw128(sa + kk * 32, 16, 1024);
+                            // B half N-major: 128-byte-wide boxes one box apart, kMmaK rows per
+                            // instruction; K-major: as A
                             const uint64_t bdesc = bk
-                                ? ptx::smem_desc_sw128(sb + kk * (kUmmaK * 2), 16, 1024)
-                                : ptx::smem_desc_sw128(sb + kk * (kUmmaK * 128), kBBox * kBK * 2, 1024);
-                            ptx::tc_mma_f16_pair(d_tmem, adesc, bdesc, bk ? kIdescBK : kIdesc,
-                                                 (q > kb || kk > 0) ? 1u : 0u);
+                                ? ptx::smem_desc_sw128(sb + kk * 32, 16, 1024)
+                                : ptx::smem_desc_sw128(sb + kk * (I::kMmaK * 128), I::kBBoxBytes, 1024);
+                            ptx::tc_mma_pair<F8>(d_tmem, adesc, bdesc, idesc, (q > kb || kk > 0) ? 1u : 0u);
                         }
                         // the stage is free in every CTA whose smem this pair read (and, with
                         // QUAD, whose producer also wrote into this pair's smem)

@@ -9,7 +9,8 @@ Workload recipes (the paper's shapes, Sec. IV-A and IV-D):
   * ``uniform``  -- entries uniform in [-1, 1]           (square / irregular / high-K sweeps)
   * ``prefill``  -- A (activations) ~ N(0, 1), B (weights, stored K x N) ~ N(0, 0.02)
   * ``int``      -- integers in {-2, ..., 2} (exact in fp32 accumulation for K < 2^21)
-For a pair (A, B) one generator draws A first, then B.
+For a pair (A, B) one generator draws A first, then B.  ``gemm_inputs_f8``
+draws the same distributions and rounds them to an 8-bit float format.
 """
 from __future__ import annotations
 
@@ -73,6 +74,28 @@ def gemm_inputs(M: int, N: int, K: int, kind: str = "uniform", seed: int = 0,
         buf[:, :N] = B
         B = buf[:, :N]
     return A, B
+
+
+def f8_dtype(fmt: str):
+    """torch dtype of an 8-bit float format ("e4m3" or "e5m2")."""
+    return {"e4m3": torch.float8_e4m3fn, "e5m2": torch.float8_e5m2}[fmt]
+
+
+def gemm_inputs_f8(M: int, N: int, K: int, fmt: str = "e4m3", kind: str = "uniform", seed: int = 0):
+    """(A, B) as CPU 8-bit float tensors of format ``fmt``: A is M x K, B is
+    K x N.  Values are drawn in fp32 exactly as for ``gemm_inputs`` (uniform in
+    [-1, 1], or integers in {-2, ..., 2}) and rounded to the format by torch."""
+    g = _gen(seed)
+    if kind == "uniform":
+        A = torch.rand((M, K), generator=g, dtype=torch.float32) * 2.0 - 1.0
+        B = torch.rand((K, N), generator=g, dtype=torch.float32) * 2.0 - 1.0
+    elif kind == "int":
+        A = torch.randint(-2, 3, (M, K), generator=g, dtype=torch.int32).float()
+        B = torch.randint(-2, 3, (K, N), generator=g, dtype=torch.int32).float()
+    else:
+        raise ValueError("unknown input kind %r" % kind)
+    dt = f8_dtype(fmt)
+    return A.to(dt), B.to(dt)
 
 
 def pad8(n: int) -> int:

@@ -136,18 +136,21 @@ def test_valid_call_without_gpu_fails_loudly(lib):
     assert lib.sfc_get_device_status(None) == binding.SFC_ERR_CUDA
     assert lib.sfc_release() == binding.SFC_ERR_CUDA
     t, c = ctypes.c_int(0), ctypes.c_int(0)
-    assert lib.sfc_gemm_plan(512, 512, 4096, 0, 0, 0, ctypes.byref(t), ctypes.byref(c)) in (
+    assert lib.sfc_gemm_plan(512, 512, 4096, 0, 0, 0, 0, 0, ctypes.byref(t), ctypes.byref(c)) in (
         binding.SFC_ERR_CUDA, binding.SFC_ERR_UNSUPPORTED)
 
 
 def test_plan_validation(lib):
     t, c = ctypes.c_int(0), ctypes.c_int(0)
-    assert lib.sfc_gemm_plan(512, 512, 4096, 0, 0, 0, None, ctypes.byref(c)) == binding.SFC_ERR_INVALID_ARG
-    assert lib.sfc_gemm_plan(0, 512, 4096, 0, 0, 0, ctypes.byref(t), ctypes.byref(c)) == binding.SFC_ERR_INVALID_ARG
-    assert lib.sfc_gemm_plan(512, 512, 4096, -2, 0, 0, ctypes.byref(t), ctypes.byref(c)) == \
-        binding.SFC_ERR_INVALID_ARG
-    assert lib.sfc_gemm_plan(512, 512, 4096, 0, 0, 77, ctypes.byref(t), ctypes.byref(c)) == \
-        binding.SFC_ERR_INVALID_ARG
+    def plan(M, N, K, c_, tile=0, ab=0, layout=0, out=True):
+        return lib.sfc_gemm_plan(M, N, K, c_, 0, tile, ab, layout, ctypes.byref(t) if out else None,
+                                 ctypes.byref(c))
+    assert plan(512, 512, 4096, 0, out=False) == binding.SFC_ERR_INVALID_ARG
+    assert plan(0, 512, 4096, 0) == binding.SFC_ERR_INVALID_ARG
+    assert plan(512, 512, 4096, -2) == binding.SFC_ERR_INVALID_ARG
+    assert plan(512, 512, 4096, 0, tile=77) == binding.SFC_ERR_INVALID_ARG
+    assert plan(512, 512, 4096, 0, ab=5) == binding.SFC_ERR_INVALID_ARG
+    assert plan(512, 512, 4096, 0, layout=3) == binding.SFC_ERR_INVALID_ARG
 
 
 def test_missing_library_raises(monkeypatch, tmp_path):
@@ -157,11 +160,11 @@ def test_missing_library_raises(monkeypatch, tmp_path):
         binding.load()
 
 
-def call_ex2(lib, M=256, N=256, K=256, ldb=None, b_layout=0, beta=0.0, bias=None, ca_c=1):
+def call_ex2(lib, M=256, N=256, K=256, ldb=None, b_layout=0, beta=0.0, bias=None, ca_c=1, ab=0, lda=None):
     ldb = (N if b_layout == 0 else K) if ldb is None else ldb
-    return lib.sfc_gemm_ex2(M, N, K, ctypes.c_void_p(PA), ctypes.c_void_p(PB), ctypes.c_void_p(PC), K, ldb, N,
-                            b_layout, beta, ctypes.c_void_p(bias) if bias else None, ca_c, 0, 0, 2, 0, None, 0,
-                            None)
+    return lib.sfc_gemm_ex2(M, N, K, ctypes.c_void_p(PA), ctypes.c_void_p(PB), ctypes.c_void_p(PC), lda or K, ldb,
+                            N, ab, b_layout, beta, ctypes.c_void_p(bias) if bias else None, ca_c, 0, 0, 2, 0, None,
+                            0, None)
 
 
 def test_gemm_ex2_validation_codes(lib):
@@ -171,3 +174,6 @@ def test_gemm_ex2_validation_codes(lib):
     assert call_ex2(lib, N=512, K=256, b_layout=0, ldb=256) == E.SFC_ERR_INVALID_ARG    # B rows shorter than N
     assert call_ex2(lib, N=512, K=256, b_layout=1, ldb=260) == E.SFC_ERR_UNALIGNED
     assert call_ex2(lib, bias=0x50002) == E.SFC_ERR_UNALIGNED                           # bias not 4-byte aligned
+    assert call_ex2(lib, ab=3) == E.SFC_ERR_INVALID_ARG                                 # unknown input type
+    assert call_ex2(lib, ab=1, K=264, lda=264, b_layout=1, ldb=264) == E.SFC_ERR_UNALIGNED  # 8-bit rows need 16 values
+    assert call_ex2(lib, ab=1, K=256 * 129, ca_c=259) == E.SFC_ERR_INVALID_ARG          # 258 slabs of 128 k

@@ -165,3 +165,48 @@ def test_affine_small_integers_exact(oracle):
     for layout, b in (("kn", B), ("nk", B.t().contiguous())):
         got = oracle.gemm_affine_f64(A, b, b_layout=layout, beta=3.0, C_in=C_in, bias=bias)
         assert np.array_equal(got, want.astype(np.float64)), layout
+
+
+# --- 8-bit float inputs (the method is independent of the data type, Sec. III)
+
+@pytest.mark.parametrize("fmt,tdtype", [("e4m3", "float8_e4m3fn"), ("e5m2", "float8_e5m2")])
+def test_f8_decode_matches_the_library_format_for_every_code(oracle, fmt, tdtype):
+    # torch's float8 -> float32 conversion is an independent implementation of the formats
+    codes = torch.arange(256, dtype=torch.int32).to(torch.uint8)
+    ref = codes.view(getattr(torch, tdtype)).float().numpy().astype(np.float64)
+    got = np.array([oracle.decode_f8(c, fmt) for c in range(256)])
+    nan = np.isnan(ref)
+    assert np.array_equal(np.isnan(got), nan)
+    assert np.array_equal(got[~nan], ref[~nan])
+
+
+def test_f8_decode_fixed_points(oracle):
+    # values the format definitions fix
+    assert oracle.decode_f8(0x38, "e4m3") == 1.0
+    assert oracle.decode_f8(0xC0, "e4m3") == -2.0
+    assert oracle.decode_f8(0x7E, "e4m3") == 448.0           # largest finite e4m3
+    assert oracle.decode_f8(0x01, "e4m3") == 2.0 ** -9       # smallest subnormal
+    assert np.isnan(oracle.decode_f8(0x7F, "e4m3"))
+    assert oracle.decode_f8(0x3C, "e5m2") == 1.0
+    assert oracle.decode_f8(0x7B, "e5m2") == 57344.0         # largest finite e5m2
+    assert oracle.decode_f8(0x01, "e5m2") == 2.0 ** -16
+    assert oracle.decode_f8(0x7C, "e5m2") == float("inf")
+
+
+@pytest.mark.parametrize("fmt", ["e4m3", "e5m2"])
+def test_f8_gemm_small_integers_exact(oracle, fmt):
+    M, N, K = 21, 34, 90
+    A, B = synth.gemm_inputs_f8(M, N, K, fmt, "int", seed=6)
+    ai = A.float().numpy().astype(np.int64)
+    bi = B.float().numpy().astype(np.int64)
+    assert set(np.unique(ai)) <= {-2, -1, 0, 1, 2}
+    want = (ai @ bi).astype(np.float64)
+    assert np.array_equal(oracle.gemm_f8_f64(A, B, fmt), want)
+    assert np.array_equal(oracle.gemm_f8_f64(A, B.t().contiguous(), fmt, b_layout="nk"), want)
+
+
+def test_f8_gemm_equals_bf16_gemm_of_the_same_values(oracle):
+    # every e4m3 value is a bf16 value, so the bf16 oracle on the widened inputs gives the same sums
+    A, B = synth.gemm_inputs_f8(17, 23, 61, "e4m3", "uniform", seed=2)
+    assert np.array_equal(oracle.gemm_f8_f64(A, B, "e4m3"),
+                          oracle.gemm_f64(A.float().to(torch.bfloat16), B.float().to(torch.bfloat16)))
