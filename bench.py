@@ -101,6 +101,8 @@ def parse_args():
     ap.add_argument("--ca-c", type=int, default=None, help="force one K-layer count for every shape")
     ap.add_argument("--b-layout", choices=("kn", "nk"), default="kn",
                     help="storage of B: K x N row-major (the paper's), or N x K (a linear layer's weight)")
+    ap.add_argument("--ab", choices=("bf16", "e4m3", "e5m2"), default="bf16",
+                    help="element type of A and B (8-bit floats use the tensor cores' 8-bit path)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
@@ -140,12 +142,17 @@ def load_peaks():
         return dict(FALLBACK_PEAKS, source="fallback")
 
 
-def roofline_time_s(s, peaks):
-    """max(compute time at the dense peak, compulsory bytes at HBM bandwidth)."""
+F8_PEAK_RATIO = 2.0  # dense 8-bit / bf16 tensor rate, nominal (4.5 / 2.25 PFLOP/s)
+
+
+def roofline_time_s(s, peaks, ab="bf16"):
+    """max(compute time at the dense peak, compulsory bytes at HBM bandwidth);
+    8-bit inputs: one byte per element and the bf16 peak x F8_PEAK_RATIO."""
     o = 4 if s["out"] == "f32" else 2
+    ib = 2 if ab == "bf16" else 1
     flops = 2.0 * s["M"] * s["N"] * s["K"]
-    bytes_min = 2.0 * (s["M"] * s["K"] + s["K"] * s["N"]) + o * s["M"] * s["N"]
-    t_tc = flops / (peaks["bf16_tflops"] * 1e12)
+    bytes_min = ib * (s["M"] * s["K"] + s["K"] * s["N"]) + o * s["M"] * s["N"]
+    t_tc = flops / (peaks["bf16_tflops"] * (1.0 if ab == "bf16" else F8_PEAK_RATIO) * 1e12)
     t_hbm = bytes_min / (peaks["hbm_gbs"] * 1e9)
     return max(t_tc, t_hbm), ("tensor" if t_tc >= t_hbm else "hbm")
 
@@ -234,7 +241,7 @@ class ClockSampler:
 _SHARED = {}
 
 
-def make_inputs(s, synth, torch):
+def make_inputs(s, synth, torch, ab="bf16"):
     def dev(t):
         full = t.as_strided((t.shape[0], t.stride(0)), (t.stride(0), 1))
         return full.contiguous().cuda()[:, : t.shape[1]]
@@ -245,12 +252,23 @@ def make_inputs(s, synth, torch):
         def operand(rows, cols, seed):
             key = (rows, cols, seed)
             if key not in _SHARED:
-                t = synth.uniform_bf16((rows, cols), seed=seed)
+                t = (synth.uniform_bf16((rows, cols), seed=seed) if ab == "bf16"
+                     else synth.uniform_f8((rows, cols), ab, seed=seed))
                 _SHARED[key] = (t, dev(t))
             return _SHARED[key]
         A, Ad = operand(s["M"], s["K"], 1000003 * s["M"] + s["K"])
         B, Bd = operand(s["K"], s["N"], 2000003 * s["K"] + s["N"] + 7)
         return A, B, Ad, Bd, C
+    if ab != "bf16":
+        # 8-bit rows padded to 16 elements (16 bytes)
+        A, B = synth.gemm_inputs_f8(s["M"], s["N"], s["K"], ab, s["kind"], seed=0)
+
+        def dev16(t):
+            ld = (t.shape[1] + 15) // 16 * 16
+            d = torch.zeros(t.shape[0], ld, dtype=t.dtype, device="cuda")
+            d[:, : t.shape[1]] = t.cuda()
+            return d[:, : t.shape[1]]
+        return A, B, dev16(A), dev16(B), C
     lda = synth.pad8(s["K"])
     ldb = synth.pad8(s["N"])
     A, B = synth.gemm_inputs(s["M"], s["N"], s["K"], s["kind"], seed=0, lda=lda, ldb=ldb)
@@ -275,13 +293,13 @@ def run_ours(args, rank, local, world):
     def as_nk(Bd):
         if id(Bd) not in transposed:
             K, N = Bd.shape
-            buf = torch.zeros(N, synth.pad8(K), dtype=torch.bfloat16, device="cuda")
+            buf = torch.zeros(N, (K + 15) // 16 * 16, dtype=Bd.dtype, device="cuda")
             buf[:, :K] = Bd.t()
             transposed[id(Bd)] = buf[:, :K]
         return transposed[id(Bd)]
 
     for s in shapes:
-        A, B, Ad, Bd, C = make_inputs(s, synth, torch)
+        A, B, Ad, Bd, C = make_inputs(s, synth, torch, args.ab)
         if args.b_layout == "nk":
             Bd = as_nk(Bd)
         mats.append({"s": s, "A": A, "B": B, "Ad": Ad, "Bd": Bd, "C": C, "c": s["cs"][0]})
@@ -313,7 +331,8 @@ def run_ours(args, rank, local, world):
                 best = (c, t)
         m["c"] = best[0]
         # the library's own choice (ca_c = 0), reported beside the configured set
-        tile, c_auto = sfc.plan(m["s"]["M"], m["s"]["N"], m["s"]["K"], 0, out_dtype=m["C"].dtype)
+        tile, c_auto = sfc.plan(m["s"]["M"], m["s"]["N"], m["s"]["K"], 0, out_dtype=m["C"].dtype,
+                                in_dtype=m["Ad"].dtype, b_layout=args.b_layout)
         for _ in range(2):
             call(m, 0)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -377,7 +396,7 @@ def run_ours(args, rank, local, world):
     b2b_ms = []
     for m in mats:
         s_ = m["s"]
-        in_bytes = 2 * (s_["M"] * s_["K"] + s_["K"] * s_["N"])
+        in_bytes = (2 if args.ab == "bf16" else 1) * (s_["M"] * s_["K"] + s_["K"] * s_["N"])
         copies = max(1, min(16, -(-(256 << 20) // in_bytes)))
         extra = [(m["Ad"], m["Bd"])]
         def clone_strided(t):  # keeps the padded row stride (16-byte aligned rows)
@@ -385,7 +404,7 @@ def run_ours(args, rank, local, world):
 
         for _ in range(copies - 1):
             extra.append((clone_strided(m["Ad"]), clone_strided(m["Bd"])))
-        reps = max(2 * copies, min(400, int(0.05 / max(roofline_time_s(s_, peaks)[0], 1e-6))))
+        reps = max(2 * copies, min(400, int(0.05 / max(roofline_time_s(s_, peaks, args.ab)[0], 1e-6))))
         for a, b in extra:
             sfc.gemm(a, b, m["C"], ca_c=m["c"], order=args.order, assign=args.assign, stream=stream,
                      b_layout=args.b_layout)
@@ -409,7 +428,7 @@ def run_ours(args, rank, local, world):
         mean = sum(ts) / len(ts)
         tot_ms += sum(ts)
         flops = 2.0 * s["M"] * s["N"] * s["K"]
-        t_roof, bound = roofline_time_s(s, peaks)
+        t_roof, bound = roofline_time_s(s, peaks, args.ab)
         row = {"M": s["M"], "N": s["N"], "K": s["K"], "out": s["out"], "ca_c": m["c"],
                "ms_mean": round(mean, 4), "ms_min": round(min(ts), 4),
                "tflops": round(flops / (mean * 1e-3) / 1e12, 1), "bound": bound,
@@ -432,30 +451,35 @@ def run_ours(args, rank, local, world):
             traffic = tr["dram_bytes_per_launch"]
     except Exception:
         traffic = None
-    # burst peak for a short timed region, sustained (power-capped) peak for a long one
+    # burst peak for a short timed region, sustained (power-capped) peak for a long one;
+    # 8-bit inputs: the measured bf16 peak times the nominal 8-bit / bf16 ratio
     sustained = elapsed_ms > 500.0
-    peak = peaks["bf16_tflops_sustained"] if sustained else peaks["bf16_tflops"]
-    roofline = {"bound": "tensor", "achieved": round(achieved, 1), "peak": peak, "unit": "TFLOP/s",
+    ratio = 1.0 if args.ab == "bf16" else F8_PEAK_RATIO
+    burst = peaks["bf16_tflops"] * ratio
+    peak = (peaks["bf16_tflops_sustained"] if sustained else peaks["bf16_tflops"]) * ratio
+    roofline = {"bound": "tensor", "achieved": round(achieved, 1), "peak": round(peak, 1), "unit": "TFLOP/s",
                 "frac": round(achieved / peak, 4), "traffic": traffic,
                 "kernel": "sfc_gemm_pair_kernel<256> (the tile AUTO picks for the dominant shapes)",
-                "peak_source": "%s dense bf16 %s (timed region %.0f ms)" % (
-                    peaks["source"], "sustained" if sustained else "burst", elapsed_ms),
-                "frac_of_burst_peak": round(achieved / peaks["bf16_tflops"], 4)}
+                "peak_source": "%s dense bf16 %s (timed region %.0f ms)%s" % (
+                    peaks["source"], "sustained" if sustained else "burst", elapsed_ms,
+                    "" if args.ab == "bf16" else " x %.1f, the nominal 8-bit / bf16 ratio" % ratio),
+                "frac_of_burst_peak": round(achieved / burst, 4)}
     launches = args.steps * sum(1 if m["c"] == 1 else 2 for m in mats)
     desc = WORKLOADS[args.workload]["desc"] if not args.sizes else "square sweep sizes %s" % args.sizes
     result = {
         "metric": METRIC, "value": round(value, 1), "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4), "higher_is_better": True,
-        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
-        "data": "synthetic (seeded %s bf16)" % ",".join(sorted({m["s"]["kind"] for m in mats})),
+        "scaling": "weak", "vs_baseline": None, "dtype": args.ab,
+        "data": "synthetic (seeded %s %s)" % (",".join(sorted({m["s"]["kind"] for m in mats})), args.ab),
         "config": {"workload": desc, "order": args.order, "assign": args.assign, "b_layout": args.b_layout,
+                   "inputs": args.ab,
                    "parallelism": "replicas" if world > 1 else "single GPU",
                    "l2": "inputs larger than L2 between reuses: one step runs every shape once, so a shape's "
                          "operands are re-read only after the other shapes' traffic has passed through L2",
                    "timing": "value: one event pair around the K steps; per_shape ms_mean: a second pass of the "
                              "same steps with an event pair around each launch; ms_back_to_back: each shape alone, "
                              "launches back to back over rotating input copies (> 256 MB between reuses)",
-                   "pct_of_dense_peak": round(100.0 * value / world / peaks["bf16_tflops"], 2)},
+                   "pct_of_dense_peak": round(100.0 * value / world / burst, 2)},
         "roofline": roofline,
         "gpu_launches": launches,
         "per_shape": per_shape,
@@ -476,7 +500,18 @@ def run_cublas_compare(args, mats, stream, call):
     step by step with this library so both see the same clocks and power."""
     import torch
 
+    one = torch.ones((), dtype=torch.float32, device="cuda")
+    colmajor = {}
+
     def cublas(m):
+        if args.ab != "bf16":
+            # cuBLAS's 8-bit GEMM (torch._scaled_mm, unit scales) wants B column-major
+            if id(m["Bd"]) not in colmajor:
+                colmajor[id(m["Bd"])] = (m["Bd"].t().contiguous().t() if args.b_layout == "kn" else m["Bd"].t())
+            out = torch._scaled_mm(m["Ad"], colmajor[id(m["Bd"])], scale_a=one, scale_b=one,
+                                   out_dtype=m["C"].dtype)
+            m["C"].copy_(out)
+            return
         Bd = m["Bd"].t() if args.b_layout == "nk" else m["Bd"]
         if m["C"].dtype == torch.bfloat16:
             torch.matmul(m["Ad"], Bd, out=m["C"])
@@ -485,9 +520,12 @@ def run_cublas_compare(args, mats, stream, call):
 
     steps = max(3, min(args.steps, 50))
     t = [[0.0, 0.0] for _ in mats]
-    for _ in range(2):
-        for m in mats:
-            cublas(m)
+    try:
+        for _ in range(2):
+            for m in mats:
+                cublas(m)
+    except Exception as e:  # e.g. a shape cuBLAS's 8-bit GEMM does not take
+        return {"unavailable": "cuBLAS comparison failed: %s" % str(e).splitlines()[0][:200]}
     for k in range(steps):
         for which in (0, 1):
             ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in mats]
@@ -578,10 +616,19 @@ def oracle_sample(mats_cpu, rows):
         M, K = A.shape
         N = B.shape[1]
         r = np.linspace(0, M - 1, min(rows, M)).astype(np.int64)
-        A_rows = A[r].contiguous()
-        Bc = B.contiguous()
+        fmt = {"torch.float8_e4m3fn": "e4m3", "torch.float8_e5m2": "e5m2"}.get(str(A.dtype))
+        if fmt:  # 8-bit tensors are sampled through their byte view
+            import torch
+            A_rows = A.view(torch.uint8)[r].contiguous().numpy()
+            Bc = B.view(torch.uint8).contiguous().numpy()
+        else:
+            A_rows = A[r].contiguous()
+            Bc = B.contiguous()
         t0 = time.perf_counter()
-        oracle.gemm_f64(A_rows, Bc)
+        if fmt:
+            oracle.gemm_f8_f64(A_rows, Bc, fmt)
+        else:
+            oracle.gemm_f64(A_rows, Bc)
         t += time.perf_counter() - t0
         flops += 2.0 * r.size * N * K
     return flops, t
@@ -598,7 +645,7 @@ def run_cpu_baseline(mats):
     flops, secs = oracle_sample(mats_cpu, rows)
     return {"value": round(flops / secs / 1e12, 6), "unit": "TFLOP/s",
             "cores": int(os.environ["OMP_NUM_THREADS"]), "kind": "oracle", "seconds": round(secs, 2),
-            "sample": "%d evenly spaced rows of C for each shape (fp64 i-k-j triple loop, OpenMP over rows)"
+            "sample": "%d evenly spaced rows of C for each shape (fp64 triple loop, OpenMP over rows)"
                       % rows}
 
 
@@ -614,7 +661,10 @@ def run_reference(args, rank, world):
     shapes = workload_shapes(args)
     mats_cpu = []
     for s in shapes:
-        A, B = synth.gemm_inputs(s["M"], s["N"], s["K"], s["kind"], seed=0)
+        if args.ab == "bf16":
+            A, B = synth.gemm_inputs(s["M"], s["N"], s["K"], s["kind"], seed=0)
+        else:
+            A, B = synth.gemm_inputs_f8(s["M"], s["N"], s["K"], args.ab, s["kind"], seed=0)
         mats_cpu.append((A, B))
     rows = 16
     for _ in range(args.warmup):
@@ -631,7 +681,8 @@ def run_reference(args, rank, world):
     return {"impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": "TFLOP/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(1e3 * secs / args.steps, 2),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic (seeded bf16)", "config": {"workload": desc, "sample": sample},
+            "data": "synthetic (seeded %s)" % args.ab, "config": {"workload": desc, "sample": sample,
+                                                                  "inputs": args.ab},
             "cpu_baseline": {"value": round(value, 6), "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": round(value, 6), "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},

@@ -83,12 +83,16 @@ def f8_dtype(fmt: str):
 
 def gemm_inputs_f8(M: int, N: int, K: int, fmt: str = "e4m3", kind: str = "uniform", seed: int = 0):
     """(A, B) as CPU 8-bit float tensors of format ``fmt``: A is M x K, B is
-    K x N.  Values are drawn in fp32 exactly as for ``gemm_inputs`` (uniform in
-    [-1, 1], or integers in {-2, ..., 2}) and rounded to the format by torch."""
+    K x N.  Values are drawn in fp32 with the distributions of ``gemm_inputs``
+    (uniform in [-1, 1]; prefill N(0, 1) x N(0, 0.02); integers in {-2, ..., 2})
+    and rounded to the format by torch."""
     g = _gen(seed)
     if kind == "uniform":
         A = torch.rand((M, K), generator=g, dtype=torch.float32) * 2.0 - 1.0
         B = torch.rand((K, N), generator=g, dtype=torch.float32) * 2.0 - 1.0
+    elif kind == "prefill":
+        A = torch.randn((M, K), generator=g, dtype=torch.float32)
+        B = torch.randn((K, N), generator=g, dtype=torch.float32) * 0.02
     elif kind == "int":
         A = torch.randint(-2, 3, (M, K), generator=g, dtype=torch.int32).float()
         B = torch.randint(-2, 3, (K, N), generator=g, dtype=torch.int32).float()
@@ -96,6 +100,10 @@ def gemm_inputs_f8(M: int, N: int, K: int, fmt: str = "e4m3", kind: str = "unifo
         raise ValueError("unknown input kind %r" % kind)
     dt = f8_dtype(fmt)
     return A.to(dt), B.to(dt)
+
+
+def uniform_f8(shape, fmt: str = "e4m3", seed: int = 0) -> torch.Tensor:
+    return (torch.rand(shape, generator=_gen(seed), dtype=torch.float32) * 2.0 - 1.0).to(f8_dtype(fmt))
 
 
 def pad8(n: int) -> int:
