@@ -95,7 +95,7 @@ def parse_args():
     ap.add_argument("--impl", choices=("ours", "reference"), default="ours")
     ap.add_argument("--workload", choices=sorted(WORKLOADS), default="square")
     ap.add_argument("--order", choices=("sfc", "raster"), default="sfc")
-    ap.add_argument("--assign", choices=("auto", "wave", "segment"), default="auto")
+    ap.add_argument("--assign", choices=("auto", "wave", "wave_static", "segment"), default="auto")
     ap.add_argument("--sizes", type=str, default=None,
                     help="square workload only: comma-separated sizes instead of the full sweep")
     ap.add_argument("--ca-c", type=int, default=None, help="force one K-layer count for every shape")
