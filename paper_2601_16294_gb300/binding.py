@@ -262,9 +262,20 @@ def matmul_host(A_host, B_host, C_host=None, *, ca_c: int = 1, out_dtype=None, s
     given).  Returns C_host after the stream has synchronised."""
     import torch
     s = stream or torch.cuda.current_stream()
+
+    def to_device(t):
+        # rows whose byte length is not a multiple of 16 get a padded row stride on the device
+        align = 16 // t.element_size()
+        ld = (t.shape[1] + align - 1) // align * align
+        if ld == t.shape[1]:
+            return t.to("cuda", non_blocking=True)
+        d = torch.empty((t.shape[0], ld), dtype=t.dtype, device="cuda")[:, : t.shape[1]]
+        d.copy_(t, non_blocking=True)
+        return d
+
     with torch.cuda.stream(s):
-        A = A_host.to("cuda", non_blocking=True)
-        B = B_host.to("cuda", non_blocking=True)
+        A = to_device(A_host)
+        B = to_device(B_host)
         C = gemm(A, B, ca_c=ca_c, out_dtype=out_dtype, stream=s, **kw)
         if C_host is None:
             C_host = torch.empty(C.shape, dtype=C.dtype, pin_memory=True)
