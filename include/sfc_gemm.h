@@ -45,7 +45,7 @@ extern "C" {
 typedef enum {
     SFC_OK = 0,
     SFC_ERR_INVALID_ARG = -1,  /* bad size, null pointer, bad enum, ca_c out of range  */
-    SFC_ERR_UNALIGNED = -2,    /* A/B base not 16-byte aligned or lda/ldb not a multiple of 8 */
+    SFC_ERR_UNALIGNED = -2,    /* an element, bias or workspace misaligned (see each call)    */
     SFC_ERR_WORKSPACE = -3,    /* workspace smaller than sfc_gemm_workspace_size(...)  */
     SFC_ERR_CUDA = -4,         /* a CUDA runtime call failed (see sfc_last_cuda_error) */
     SFC_ERR_TIMEOUT = -5,      /* a device-side wait gave up (reported by sfc_get_device_status) */
@@ -149,8 +149,13 @@ size_t sfc_gemm_workspace_size(int64_t M, int64_t N, int64_t K, int ca_c);
  *         more than one layer (the replication factor choice of Sec. II-D,
  *         made per call); sfc_gemm_plan reports the choice.
  *   stream: a cudaStream_t passed as void*.
- * Requirements: A and B 16-byte aligned, lda and ldb multiples of 8 (the tile
- * loads use the Tensor Memory Accelerator).  C may have any alignment.
+ * Alignment: the tile loads (Tensor Memory Accelerator) read 16-byte-aligned
+ * rows.  When A or B is not 16-byte aligned, or lda / ldb is not a multiple of
+ * 8, the call first copies that operand into a padded buffer taken from the
+ * stream-ordered pool (one extra read and write of the operand; no counterpart
+ * in the paper, whose blocked layouts are always aligned).  A and B must be
+ * aligned to their element size (else SFC_ERR_UNALIGNED).  C may have any
+ * alignment.
  * Accuracy: products are exact and summed in fp32; the tensor core's running
  * sum is restarted every 4096 values of k and the partial sums are added with
  * round-to-nearest fp32 adds, which bounds the error growth of very long K.
@@ -187,8 +192,8 @@ int sfc_gemm_ex(int64_t M, int64_t N, int64_t K,
  * operand layout and epilogue of a BLAS-style GEMM (no counterpart in the
  * paper, which computes C = A B with C zeroed first, Listing 1):
  *     C = A B + beta * C + bias[j]     (fp32 arithmetic, then rounded to c_dtype)
- *   ab_dtype: sfc_ab_t of both A and B.  For the 8-bit kinds lda and ldb are
- *             multiples of 16 elements, K layers split ceil(K/128) slabs of
+ *   ab_dtype: sfc_ab_t of both A and B.  For the 8-bit kinds rows are repacked
+ *             unless lda and ldb are multiples of 16, K layers split ceil(K/128) slabs of
  *             128 values of k, and the N-major (SFC_B_KN) layout is not served
  *             by SFC_TILE_PAIR_N128 (SFC_TILE_N128 is used instead).
  *   b_layout: SFC_B_KN (B is K x N, ldb >= N) or SFC_B_NK (B is stored as its
@@ -263,7 +268,9 @@ int sfc_num_workers(void);
  *   Arguments as sfc_gemm_ex with order = SFC, assign and tile = AUTO.
  *   Errors: SFC_ERR_WORKSPACE (nothing launched) when
  *           sfc_gemm_workspace_size(M, N, K, ca_c) > SFC_NOALLOC_SCRATCH_BYTES;
- *           otherwise as sfc_gemm_ex.
+ *           SFC_ERR_UNALIGNED when A or B would need repacking (a base not
+ *           16-byte aligned or lda / ldb not a multiple of 8), since that
+ *           takes memory; otherwise as sfc_gemm_ex.
  * The first call on each device looks up the scratch area's device address
  * (once per device, with that device current); make that first call before
  * any stream capture.  All calls share the one scratch area and leave their

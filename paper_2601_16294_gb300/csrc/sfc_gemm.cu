@@ -367,9 +367,10 @@ int validate(int64_t M, int64_t N, int64_t K, const void* A, const void* B, cons
     if (ca_c < 0 || ca_c > Kt || ca_c > kMaxLayers) return SFC_ERR_INVALID_ARG;  // 0: chosen per call
     const int64_t layers = ca_c > 0 ? ca_c : auto_layer_cap(M, N, K, ab);
     if (ceil_div(M, kBM) * ceil_div(N, 128) * layers > (int64_t(1) << 31) - 1) return SFC_ERR_INVALID_ARG;
-    // the tile loads use the Tensor Memory Accelerator: 16-byte rows and bases
-    const int64_t row_align = 16 / in_bytes(ab);
-    if (!aligned16(A) || !aligned16(B) || (lda % row_align) != 0 || (ldb % row_align) != 0) return SFC_ERR_UNALIGNED;
+    // elements must be naturally aligned; rows that are not 16-byte aligned are
+    // repacked before the tile loads (run_gemm)
+    const uintptr_t ea = static_cast<uintptr_t>(in_bytes(ab)) - 1u;
+    if ((reinterpret_cast<uintptr_t>(A) & ea) || (reinterpret_cast<uintptr_t>(B) & ea)) return SFC_ERR_UNALIGNED;
     if (lda >= (int64_t(1) << 39) || ldb >= (int64_t(1) << 39)) return SFC_ERR_INVALID_ARG;
     return SFC_OK;
 }
@@ -389,11 +390,18 @@ cudaError_t launch_gemm(int v, bool f8, const CUtensorMap& ta, const CUtensorMap
 int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void* C, int64_t lda, int64_t ldb,
              int64_t ldc, int ca_c, int c_dtype, int order, int assign, int tile, void* workspace,
              size_t workspace_bytes, cudaStream_t stream, int debug_never, uint64_t timeout_ns,
-             int b_layout = SFC_B_KN, float beta = 0.0f, const float* bias = nullptr, int ab = SFC_AB_BF16) {
+             int b_layout = SFC_B_KN, float beta = 0.0f, const float* bias = nullptr, int ab = SFC_AB_BF16,
+             bool allow_pack = true) {
     int rc = validate(M, N, K, A, B, C, lda, ldb, ldc, ca_c, c_dtype, order, assign, tile, b_layout, ab);
     if (rc != SFC_OK) return rc;
     const bool f8 = (ab != SFC_AB_BF16);
     const int sk = slab_k(ab), eb = in_bytes(ab);
+    // operands whose rows (or base) are not 16-byte aligned are repacked into pool memory
+    const int64_t row_align = 16 / eb;
+    const int64_t b_rows = (b_layout == SFC_B_NK) ? N : K, b_cols = (b_layout == SFC_B_NK) ? K : N;
+    const bool pack_a = !aligned16(A) || (lda % row_align) != 0;
+    const bool pack_b = !aligned16(B) || (ldb % row_align) != 0;
+    if ((pack_a || pack_b) && !allow_pack) return SFC_ERR_UNALIGNED;
     if (bias && (reinterpret_cast<uintptr_t>(bias) & 3u) != 0) return SFC_ERR_UNALIGNED;
     const bool b_kmajor = (b_layout == SFC_B_NK);
     if (ca_c > 0 && workspace && workspace_bytes < sfc_gemm_workspace_size(M, N, K, ca_c)) return SFC_ERR_WORKSPACE;
@@ -413,18 +421,55 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     const size_t ws_need = sfc_gemm_workspace_size(M, N, K, ca_c);
     const int bn = variant_bn(v);
     const int bm = variant_bm(v);
+    void* packed[2] = {nullptr, nullptr};
+    auto release_packed = [&]() {
+        for (void* ptr : packed)
+            if (ptr) cudaFreeAsync(ptr, stream);
+    };
+    for (int which = 0; which < 2; ++which) {
+        if (!(which == 0 ? pack_a : pack_b)) continue;
+        const int64_t rows = which == 0 ? M : b_rows, cols = which == 0 ? K : b_cols;
+        const int64_t ld_src = which == 0 ? lda : ldb;
+        const int64_t ld_dst = (cols + row_align - 1) / row_align * row_align;
+        cudaError_t e = cudaMallocAsync(&packed[which], static_cast<size_t>(rows * ld_dst * eb), stream);
+        if (e != cudaSuccess) {
+            release_packed();
+            return cuda_fail(e);
+        }
+        int64_t blocks = ceil_div(rows * cols, 256);
+        if (blocks > static_cast<int64_t>(dev->num_sms) * 16) blocks = static_cast<int64_t>(dev->num_sms) * 16;
+        pack_rows_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(
+            static_cast<const uint8_t*>(which == 0 ? A : B), ld_src, rows, cols, eb,
+            static_cast<uint8_t*>(packed[which]), ld_dst);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) {
+            release_packed();
+            return cuda_fail(e);
+        }
+        if (which == 0) {
+            A = packed[0];
+            lda = ld_dst;
+        } else {
+            B = packed[1];
+            ldb = ld_dst;
+        }
+    }
     CUtensorMap ta, tb;
     rc = make_in_map(&ta, A, M, K, lda, eb, kBM, sk);  // each CTA loads 128 rows of A, one slab of k
-    if (rc != SFC_OK) return rc;
-    if (b_kmajor) {
-        // B given as N x K: boxes of (this CTA's share of the tile's N rows) x one slab of k, like A
-        rc = make_in_map(&tb, B, N, K, ldb, eb, variant_pair(v) ? bn / 2 : bn, sk);
-    } else {
-        // N-major B boxes: one slab of k rows x 128 bytes of columns; with two pairs
-        // sharing B each CTA loads half the slab's rows
-        rc = make_in_map(&tb, B, K, N, ldb, eb, v == kQuad256 ? sk / 2 : sk, 128 / eb);
+    if (rc == SFC_OK) {
+        if (b_kmajor) {
+            // B given as N x K: boxes of (this CTA's share of the tile's N rows) x one slab of k, like A
+            rc = make_in_map(&tb, B, N, K, ldb, eb, variant_pair(v) ? bn / 2 : bn, sk);
+        } else {
+            // N-major B boxes: one slab of k rows x 128 bytes of columns; with two pairs
+            // sharing B each CTA loads half the slab's rows
+            rc = make_in_map(&tb, B, K, N, ldb, eb, v == kQuad256 ? sk / 2 : sk, 128 / eb);
+        }
     }
-    if (rc != SFC_OK) return rc;
+    if (rc != SFC_OK) {
+        release_packed();
+        return rc;
+    }
 
     GemmParams p;
     p.M = M;
@@ -460,7 +505,10 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     bool pooled = false;
     if (ca_c > 1 && !ws) {
         cudaError_t e = cudaMallocAsync(&ws, ws_need, stream);
-        if (e != cudaSuccess) return cuda_fail(e);
+        if (e != cudaSuccess) {
+            release_packed();
+            return cuda_fail(e);
+        }
         pooled = true;
     }
 
@@ -513,6 +561,7 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
         cudaError_t f = cudaFreeAsync(ws, stream);
         if (e == cudaSuccess) e = f;
     }
+    release_packed();  // stream-ordered: after the kernels that read the packed copies
     if (e != cudaSuccess) return cuda_fail(e);
     return SFC_OK;
 }
@@ -689,7 +738,8 @@ SFC_API int sfc_gemm_noalloc(int64_t M, int64_t N, int64_t K, const void* A, con
     void* scratch = nullptr;
     int rc = noalloc_scratch(&scratch);
     if (rc != SFC_OK) return rc;
-    return sfc_gemm_ex(M, N, K, A, B, C, lda, ldb, ldc, ca_c, c_dtype, SFC_ORDER_SFC, SFC_ASSIGN_AUTO,
-                       SFC_TILE_AUTO, scratch, SFC_NOALLOC_SCRATCH_BYTES, stream);
+    return run_gemm(M, N, K, A, B, C, lda, ldb, ldc, ca_c, c_dtype, SFC_ORDER_SFC, SFC_ASSIGN_AUTO, SFC_TILE_AUTO,
+                    scratch, SFC_NOALLOC_SCRATCH_BYTES, static_cast<cudaStream_t>(stream), 0, kDefaultTimeoutNs,
+                    SFC_B_KN, 0.0f, nullptr, SFC_AB_BF16, /*allow_pack=*/false);
 }
 

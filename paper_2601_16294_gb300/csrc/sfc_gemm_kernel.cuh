@@ -818,6 +818,24 @@ ca_reduce_kernel(const float* __restrict__ ws, int64_t ldw, int64_t layer_stride
     }
 }
 
+// Row-major copy of a rows x cols matrix of `elem`-byte values (2 or 1) into a
+// buffer whose rows are 16-byte aligned (row stride ld_dst), for inputs whose
+// own rows or base are not: the tile loads need 16-byte-aligned rows.
+__global__ void __launch_bounds__(256)
+pack_rows_kernel(const uint8_t* __restrict__ src, int64_t ld_src, int64_t rows, int64_t cols, int elem,
+                 uint8_t* __restrict__ dst, int64_t ld_dst) {
+    const int64_t total = rows * cols;
+    for (int64_t idx = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; idx < total;
+         idx += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const int64_t r = idx / cols;
+        const int64_t c = idx - r * cols;
+        if (elem == 2)
+            reinterpret_cast<uint16_t*>(dst)[r * ld_dst + c] = reinterpret_cast<const uint16_t*>(src)[r * ld_src + c];
+        else
+            dst[r * ld_dst + c] = src[r * ld_src + c];
+    }
+}
+
 // out[s] = tm * Nt + tn for every curve position s, with the kernels' decoder.
 __global__ void tile_order_kernel(int Mt, int Nt, int32_t* __restrict__ out) {
     const int64_t n = static_cast<int64_t>(Mt) * Nt;

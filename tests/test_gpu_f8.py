@@ -112,3 +112,14 @@ def test_layer_count_choice_and_beta_bias(sfc, oracle):
     sfc.gemm(A.cuda(), B.cuda(), C, ca_c=0, beta=0.5, bias=bias.cuda())
     torch.cuda.synchronize()
     assert np.array_equal(C.cpu().numpy().astype(np.float64), ref)
+
+
+def test_unaligned_rows_are_repacked(sfc, oracle):
+    # 8-bit rows of 1000 and 300 values (not multiples of 16 bytes) go through the repacking copy
+    M, N, K = 200, 300, 1000
+    A, B = synth.gemm_inputs_f8(M, N, K, "e4m3", "int", seed=77)
+    ref = oracle.gemm_f8_f64(A, B, "e4m3")
+    C = sfc.gemm(A.cuda(), B.cuda(), ca_c=2)
+    torch.cuda.synchronize()
+    assert sfc.device_status() == 0
+    assert np.array_equal(C.cpu().numpy().astype(np.float64), ref)

@@ -176,8 +176,9 @@ def test_error_codes_on_device(sfc):
     from paper_2601_16294_gb300 import binding
     A = torch.zeros(256, 264, dtype=torch.bfloat16, device="cuda")
     B = torch.zeros(256, 256, dtype=torch.bfloat16, device="cuda")
+    C = torch.empty(256, 256, dtype=torch.float32, device="cuda")
     with pytest.raises(binding.SfcError) as e:
-        sfc.gemm(A[:, 1:257], B)                                # base misaligned by 2 bytes
+        binding.gemm_noalloc(A[:, 1:257], B, C)                 # would need repacking: no memory to do it in
     assert e.value.code == binding.SFC_ERR_UNALIGNED
     with pytest.raises(binding.SfcError) as e:
         sfc.gemm(A[:, :256], B, ca_c=5)                         # more layers than K tiles
@@ -200,3 +201,29 @@ def test_bounded_wait_reports_timeout_and_context_survives(sfc, oracle):
     A2, B2 = synth.gemm_inputs(256, 256, 256, "int", seed=4)
     ref = oracle.gemm_f64(A2, B2)
     assert np.array_equal(run(sfc, A2, B2), ref)
+
+
+@pytest.mark.parametrize("M,N,K,off_a,off_b", [(300, 260, 1001, 1, 0), (129, 517, 2500, 0, 3), (256, 256, 130, 5, 7),
+                                               (1000, 1200, 2500, 0, 0)])
+def test_unaligned_operands_are_repacked(sfc, oracle, M, N, K, off_a, off_b):
+    # rows of K and N bf16 values that are not multiples of 8, at bases off by a few elements
+    A, B = synth.gemm_inputs(M, N, K, "uniform", seed=M + K)
+    ref = oracle.gemm_f64(A, B)
+    Abuf = torch.zeros(M * K + off_a, dtype=torch.bfloat16, device="cuda")
+    Bbuf = torch.zeros(K * N + off_b, dtype=torch.bfloat16, device="cuda")
+    Ad = Abuf[off_a:].view(M, K)
+    Bd = Bbuf[off_b:].view(K, N)
+    Ad.copy_(A)
+    Bd.copy_(B)
+    for c in (1, 3):
+        for tile in ("auto", 128, "pair256"):
+            C = sfc.gemm(Ad, Bd, ca_c=c, tile=tile)
+            torch.cuda.synchronize()
+            assert sfc.device_status() == 0
+            check_fp32(C.cpu().numpy().astype(np.float64), ref, K)
+    # transposed B with odd rows
+    Btbuf = torch.zeros(N * K + off_b, dtype=torch.bfloat16, device="cuda")
+    Btd = Btbuf[off_b:].view(N, K)
+    Btd.copy_(B.t())
+    C = sfc.gemm(Ad, Btd, b_layout="nk")
+    check_fp32(C.cpu().numpy().astype(np.float64), ref, K)
