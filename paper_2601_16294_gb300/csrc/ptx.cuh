@@ -103,9 +103,6 @@ __device__ __forceinline__ void bulk_wait_read_all() { asm volatile("cp.async.bu
 // store group has been read.
 __device__ __forceinline__ void bulk_wait_read_1() { asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory"); }
 
-// Wait until all committed bulk stores have completed.
-__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
-
 // Order this thread's generic-proxy shared-memory writes before later async-proxy (TMA) reads.
 __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -186,17 +183,6 @@ __device__ __forceinline__ void tmem_ld_32x32b_x32(uint32_t taddr, uint32_t (&r)
         : "memory");
 }
 
-// 32 lanes x 16 columns: thread t gets lane (base_lane + t), register j holds column (base_col + j).
-__device__ __forceinline__ void tmem_ld_32x32b_x16(uint32_t taddr, uint32_t (&r)[16]) {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-        : "r"(taddr)
-        : "memory");
-}
-
 __device__ __forceinline__ void tmem_ld_wait() {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
@@ -214,18 +200,6 @@ __device__ __forceinline__ uint32_t map_to_cta(uint32_t addr, uint32_t rank) {
     uint32_t r;
     asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
     return r;
-}
-
-// 32-bit store into shared memory of another CTA of the cluster.
-__device__ __forceinline__ void st_shared_cluster(uint32_t cluster_addr, int v) {
-    asm volatile("st.shared::cluster.s32 [%0], %1;" ::"r"(cluster_addr), "r"(v) : "memory");
-}
-
-// Arrive on an mbarrier that may live in another CTA of the cluster, releasing
-// this thread's earlier writes at cluster scope: for publishing data that the
-// waiting side reads (e.g. after st.shared::cluster into the peer's memory).
-__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
-    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
 
 // Send 16 bytes into a peer CTA's shared memory; the peer's mbarrier counts
@@ -246,8 +220,9 @@ __device__ __forceinline__ void mbar_expect_tx_remote(uint32_t cluster_bar, uint
 
 // Arrive on an mbarrier that may live in another CTA of the cluster with the
 // default (CTA-scope) release: for a consumer handing a buffer back after its
-// reads have completed (queue slots, tensor-memory accumulators).  The
-// cluster-scope release above costs several hundred nanoseconds on each call.
+// reads have completed (queue slots, tensor-memory accumulators).  A
+// cluster-scope release (.release.cluster) costs several hundred nanoseconds
+// per call; data published to a peer goes by st_async_v4 instead.
 __device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
     asm volatile("mbarrier.arrive.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
 }
