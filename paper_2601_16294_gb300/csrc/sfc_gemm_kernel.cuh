@@ -150,12 +150,30 @@ __device__ __forceinline__ WorkItem decode_item(int64_t i64, const GemmParams& p
 // Chunks of an item's K range: n = ceil(len / kc), boundaries balanced.
 __device__ __forceinline__ int num_chunks(const WorkItem& w, int kc) {
     const int len = w.k1 - w.k0;
-    return (len + kc - 1) / kc;
+    return len <= kc ? 1 : (len + kc - 1) / kc;
 }
 // Position (0-based, in processing order) where chunk j of n starts.
-__device__ __forceinline__ int chunk_begin(const WorkItem& w, int j, int n) {
-    return static_cast<int>((static_cast<int64_t>(j) * (w.k1 - w.k0)) / n);
-}
+// Chunk j of n starts at position floor(j * len / n) of the item's K range;
+// the walk steps through j = 0, 1, ..., n with one 32-bit division per item
+// (the MMA issuer does this between its MMAs).
+struct ChunkWalk {
+    int q, r, n, begin, rem;
+    __device__ __forceinline__ ChunkWalk(const WorkItem& w, int n_) : n(n_), begin(0), rem(0) {
+        const int len = w.k1 - w.k0;
+        q = (n_ == 1) ? len : len / n_;
+        r = len - q * n_;
+    }
+    // end of the current chunk = begin of the next; advances
+    __device__ __forceinline__ int next() {
+        rem += r;
+        begin += q;
+        if (rem >= n) {
+            rem -= n;
+            ++begin;
+        }
+        return begin;
+    }
+};
 
 // Items of worker `worker` out of `workers`: [first, end) with stride `step`.
 __device__ __forceinline__ void worker_items(const GemmParams& p, int64_t worker, int64_t workers,
@@ -316,8 +334,8 @@ __device__ __forceinline__ int64_t src_take(const ItemSource& S, int j, const Ge
     w.tn = S.q_entry[4 * q + 2];
     w.layer = S.q_entry[4 * q + 3];
     ptx::mbar_arrive_remote(S.q_empty0 + 8u * q);  // slot free once every consumer has read it
-    w.k0 = layer_k0(w.layer, p);
-    w.k1 = layer_k0(w.layer + 1, p);
+    w.k0 = (p.ca_c == 1) ? 0 : layer_k0(w.layer, p);
+    w.k1 = (p.ca_c == 1) ? p.Kt : layer_k0(w.layer + 1, p);
     w.rev = p.serpentine ? (j & 1) : 0;
     return item;
 }
@@ -705,8 +723,9 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
                     break;
                 }
                 const int nch = num_chunks(w, p.kc);
+                ChunkWalk cw(w, nch);
                 for (int ck = 0; ok && ck < nch; ++ck) {
-                    const int kb = chunk_begin(w, ck, nch), ke = chunk_begin(w, ck + 1, nch);
+                    const int kb = cw.begin, ke = cw.next();
                     if (!wait_bounded(B.acc_empty(acc), acc_phase ^ 1u, abort_flag, p.timeout_ns, kWaitMmaAccEmpty)) {
                         ok = false;
                         break;
@@ -721,17 +740,19 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
                         ptx::tc_fence_after();
                         const uint32_t sa = ring + stage * kStageBytes;
                         const uint32_t sb = sa + kABytes;
+                        // A: K-major, 128-byte rows, 8-row atoms 1024 B apart; 32 B per instruction.
+                        // B N-major: 128-byte-wide boxes one box apart, 8-row atoms 1 KB apart, kMmaK
+                        // rows per instruction; B K-major: as A.  Later instructions of the slab step
+                        // the start-address field (16-byte units, bits 0-13; the ring lies below
+                        // 256 KB, so the field never carries).
+                        const uint64_t adesc = ptx::smem_desc_sw128(sa, 16, 1024);
+                        const uint64_t bdesc = p.b_kmajor ? ptx::smem_desc_sw128(sb, 16, 1024)
+                                                          : ptx::smem_desc_sw128(sb, I::kBBoxBytes, 1024);
+                        const uint32_t bstep = p.b_kmajor ? 2u : (I::kMmaK * 128) / 16;
 #pragma unroll
-                        for (int kk = 0; kk < I::kSlabK / I::kMmaK; ++kk) {
-                            // A: K-major, 128-byte rows, 8-row atoms 1024 B apart; 32 B per instruction
-                            const uint64_t adesc = ptx::smem_desc_sw128(sa + kk * 32, 16, 1024);
-                            // B N-major: 128-byte-wide boxes one box apart, 8-row atoms 1 KB apart,
-                            // kMmaK rows per instruction; B K-major: as A
-                            const uint64_t bdesc = p.b_kmajor
-                                ? ptx::smem_desc_sw128(sb + kk * 32, 16, 1024)
-                                : ptx::smem_desc_sw128(sb + kk * (I::kMmaK * 128), I::kBBoxBytes, 1024);
-                            ptx::tc_mma<F8>(d_tmem, adesc, bdesc, idesc, (q > kb || kk > 0) ? 1u : 0u);
-                        }
+                        for (int kk = 0; kk < I::kSlabK / I::kMmaK; ++kk)
+                            ptx::tc_mma<F8>(d_tmem, adesc + 2u * kk, bdesc + bstep * kk, idesc,
+                                            (q > kb || kk > 0) ? 1u : 0u);
                         ptx::tc_commit(B.empty(stage));  // frees the stage once these MMAs finish
                         if (++stage == STAGES) {
                             stage = 0;

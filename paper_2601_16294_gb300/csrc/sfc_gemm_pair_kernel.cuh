@@ -214,8 +214,9 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
                     break;
                 }
                 const int nch = num_chunks(w, p.kc);
+                ChunkWalk cw(w, nch);
                 for (int ck = 0; ok && ck < nch; ++ck) {
-                    const int kb = chunk_begin(w, ck, nch), ke = chunk_begin(w, ck + 1, nch);
+                    const int kb = cw.begin, ke = cw.next();
                     if (!wait_bounded(B.acc_empty(acc), acc_phase ^ 1u, abort_flag, p.timeout_ns, kWaitMmaAccEmpty)) {
                         ok = false;
                         break;
@@ -230,17 +231,18 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
                         ptx::tc_fence_after();
                         const uint32_t sa = ring + stage * S::kBytes;
                         const uint32_t sb = sa + S::kABytes;
+                        // A half: K-major, 128-byte rows, 8-row atoms 1 KB apart; 32 B per instruction.
+                        // B half N-major: 128-byte-wide boxes one box apart, kMmaK rows per
+                        // instruction; K-major: as A.  Later instructions step the start-address
+                        // field (16-byte units, bits 0-13; the ring lies below 256 KB: no carry).
+                        const uint64_t adesc = ptx::smem_desc_sw128(sa, 16, 1024);
+                        const uint64_t bdesc = bk ? ptx::smem_desc_sw128(sb, 16, 1024)
+                                                  : ptx::smem_desc_sw128(sb, I::kBBoxBytes, 1024);
+                        const uint32_t bstep = bk ? 2u : (I::kMmaK * 128) / 16;
 #pragma unroll
-                        for (int kk = 0; kk < I::kSlabK / I::kMmaK; ++kk) {
-                            // A half: K-major, 128-byte rows, 8-row atoms 1 KB apart; 32 B per instruction
-                            const uint64_t adesc = ptx::smem_desc_sw128(sa + kk * 32, 16, 1024);
-                            // B half N-major: 128-byte-wide boxes one box apart, kMmaK rows per
-                            // instruction; K-major: as A
-                            const uint64_t bdesc = bk
-                                ? ptx::smem_desc_sw128(sb + kk * 32, 16, 1024)
-                                : ptx::smem_desc_sw128(sb + kk * (I::kMmaK * 128), I::kBBoxBytes, 1024);
-                            ptx::tc_mma_pair<F8>(d_tmem, adesc, bdesc, idesc, (q > kb || kk > 0) ? 1u : 0u);
-                        }
+                        for (int kk = 0; kk < I::kSlabK / I::kMmaK; ++kk)
+                            ptx::tc_mma_pair<F8>(d_tmem, adesc + 2u * kk, bdesc + bstep * kk, idesc,
+                                                 (q > kb || kk > 0) ? 1u : 0u);
                         // the stage is free in every CTA whose smem this pair read (and, with
                         // QUAD, whose producer also wrote into this pair's smem)
                         ptx::tc_commit_pair_multicast(B.empty(stage), stage_mask);
