@@ -264,9 +264,10 @@ int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
 constexpr double kSlabClockGhz = 1.9;        // SM clock the slab times assume
 constexpr double kReduceLaunchNs = 3000.0;   // reduction kernel launch and ramp
 constexpr double kPartialBytesPerNs = 6000.0;
-// relative tensor-pipe efficiency measured on GB300 (256-wide tiles feed the
-// tensor core with fewer shared-memory bytes per flop)
-constexpr double kEff[kNumVariants] = {0.50, 0.85, 0.55, 0.95, 0.90};
+// relative tensor-pipe efficiency measured on GB300, back to back at 8192 x
+// 8192 x 4096 and 6144^2 x 4096 (256-wide tiles feed the tensor core with fewer
+// shared-memory bytes per flop; the quad variant is kept just below the pair)
+constexpr double kEff[kNumVariants] = {0.60, 0.82, 0.62, 0.95, 0.92};
 
 // Layers ca_c = 0 may choose: enough to give about 320 items of 128 x 128,
 // never more than 64 or the number of K slabs (host-only, so the workspace
