@@ -284,6 +284,61 @@ int sfc_gemm_noalloc(int64_t M, int64_t N, int64_t K,
                      int ca_c, sfc_dtype_t c_dtype, void *stream);
 
 /*
+ * sfc_gemm_host -- C = A * B with A, B and C in HOST memory: the library
+ * uploads the operands, runs the GEMM and downloads C, with the copies
+ * overlapped against the tile contraction.  No counterpart in the paper,
+ * whose operands already sit in the memory the cores compute from.
+ *
+ * The output is cut into `panels` slices along the dimension of the larger
+ * operand (rows of C when M >= N, else columns).  The smaller operand goes up
+ * whole, then each slice of the larger one; the GEMM of a slice starts when
+ * its slice has arrived, and its part of C goes back while the next slice
+ * computes.  Slice edges fall on multiples of 512 rows or 256 columns (the
+ * largest output tiles), so the result is bit-identical to sfc_gemm_ex2 over
+ * the whole problem with the tile and ca_c that sfc_gemm_plan(M, N, K, ca_c,
+ * c_dtype, tile, ab_dtype, b_layout, ...) reports, which every slice uses.
+ *
+ *   A, B, C: HOST pointers, row-major with row strides lda, ldb, ldc in
+ *            elements (any stride; the device copies get 16-byte rows).  A and
+ *            B are ab_dtype (sfc_ab_t), B laid out per b_layout
+ *            (sfc_b_layout_t); C is c_dtype (written, never read).  Use
+ *            page-locked memory (cudaHostAlloc / cudaHostRegister): with
+ *            pageable memory the result is the same but the copies do not
+ *            overlap the GEMM.
+ *   ca_c, tile: as sfc_gemm_ex2 (0 / SFC_TILE_AUTO: chosen for the whole
+ *            problem).  Order is the curve, assignment automatic, beta = 0,
+ *            no bias.
+ *   panels:  number of slices; 0 picks about one per 2048 rows or columns,
+ *            at most 8.  Clamped to the number of 512-row (256-column) units.
+ *   stream:  the GEMMs run on it; the copies run on two library streams that
+ *            it waits for, so `stream` has finished with C once it has
+ *            reached the end of this call's work.
+ * The call is asynchronous: it returns once everything is enqueued.  A and B
+ * are read after it returns: they must hold their values when the call is
+ * made (their uploads are NOT ordered after work already on `stream`) and
+ * stay unchanged until `stream` is synchronized; C is complete then.
+ * Device memory: staging slots owned by the library, each holding one call's
+ * device copies of A, B and C; a slot is reused once the call that used it
+ * has completed, so calls issued back to back overlap (the next call's
+ * uploads run while this one computes).  New slots are allocated while the
+ * slots held stay under half of the device memory that was free at the first
+ * call; past that, the call waits for the slots in use and frees them first.
+ * sfc_release frees every slot.  Calls from several host threads are
+ * serialized per device.
+ * Errors (nothing is enqueued): SFC_ERR_INVALID_ARG for sizes, strides
+ * (lda < K, ldb < N or K, ldc < N), enums or panels < 0 as sfc_gemm_ex2;
+ * SFC_ERR_UNALIGNED when a pointer is not aligned to its element size;
+ * SFC_ERR_CUDA when staging memory cannot be allocated; SFC_ERR_UNSUPPORTED.
+ * A CUDA error after enqueueing began returns SFC_ERR_CUDA; the call then
+ * still orders the staging slot's reuse after whatever it enqueued.
+ */
+int sfc_gemm_host(int64_t M, int64_t N, int64_t K,
+                  const void *A, const void *B, void *C,
+                  int64_t lda, int64_t ldb, int64_t ldc,
+                  int ab_dtype, int b_layout, int ca_c, sfc_dtype_t c_dtype,
+                  sfc_tile_t tile, int panels, void *stream);
+
+/*
  * sfc_debug_force_timeout -- test hook for the failure path: launches one GEMM
  * worker on a tiny problem whose MMA stage waits on a barrier that nothing
  * arrives at, with a wait limit of `limit_ms` milliseconds (1..1000).  The

@@ -44,7 +44,7 @@ def _ab_code(dtype) -> int:
 
 EXPORTS = ("sfc_tile_order", "sfc_tile_order_device", "sfc_gemm_workspace_size", "sfc_gemm", "sfc_gemm_ex",
            "sfc_get_device_status", "sfc_last_cuda_error", "sfc_num_workers", "sfc_debug_force_timeout",
-           "sfc_gemm_noalloc", "sfc_gemm_plan", "sfc_release", "sfc_gemm_ex2")
+           "sfc_gemm_noalloc", "sfc_gemm_plan", "sfc_release", "sfc_gemm_ex2", "sfc_gemm_host")
 NOALLOC_SCRATCH_BYTES = 32 << 20
 
 
@@ -97,6 +97,7 @@ def load():
         lib.sfc_gemm_ex2.argtypes = [i64, i64, i64, vp, vp, vp, i64, i64, i64, i32, i32, ctypes.c_float, vp, i32,
                                      i32, i32, i32, i32, vp, sz, vp]
         lib.sfc_release.argtypes = []
+        lib.sfc_gemm_host.argtypes = [i64, i64, i64, vp, vp, vp, i64, i64, i64, i32, i32, i32, i32, i32, i32, vp]
         for name in EXPORTS:
             if name != "sfc_gemm_workspace_size":
                 getattr(lib, name).restype = ctypes.c_int
@@ -256,29 +257,50 @@ def debug_force_timeout(A, B, C, limit_ms: int = 20, stream=None) -> int:
                                           ctypes.c_void_p(C.data_ptr()), int(limit_ms), _stream_ptr(stream))
 
 
-def matmul_host(A_host, B_host, C_host=None, *, ca_c: int = 1, out_dtype=None, stream=None, **kw):
-    """End-to-end call from HOST tensors: copy A and B (pinned for speed) to the
-    device, run the GEMM, copy C back into ``C_host`` (allocated pinned if not
-    given).  Returns C_host after the stream has synchronised."""
+def gemm_host(A_host, B_host, C_host=None, *, ca_c: int = 0, out_dtype=None, tile=0, b_layout: str = "kn",
+              panels: int = 0, stream=None):
+    """C = A @ B from HOST tensors through ``sfc_gemm_host``: the library
+    uploads A and B, runs the GEMM and downloads C, overlapping the copies
+    with the contraction (slices of ``panels`` rows or columns; 0 = automatic).
+    A, B: CPU tensors (bf16 or an 8-bit float), row-major with any row stride,
+    ideally pinned; B is (K, N) for ``b_layout="kn"`` or (N, K) for ``"nk"``.
+    C_host: (M, N) fp32 or bf16 CPU tensor, allocated pinned if not given.
+    Asynchronous on ``stream``: C_host is complete once the stream has been
+    synchronised, and A and B must not change before then."""
+    import torch
+    M, K = A_host.shape
+    if b_layout == "kn":
+        K2, N = B_host.shape
+    elif b_layout == "nk":
+        N, K2 = B_host.shape
+    else:
+        raise ValueError("b_layout must be 'kn' or 'nk'")
+    if K != K2:
+        raise ValueError("inner dimensions differ: %d vs %d" % (K, K2))
+    if A_host.dtype != B_host.dtype:
+        raise TypeError("A and B must have the same dtype")
+    for name, t in (("A", A_host), ("B", B_host)):
+        if t.device.type != "cpu":
+            raise ValueError("%s must be a host (CPU) tensor" % name)
+    if C_host is None:
+        C_host = torch.empty((M, N), dtype=out_dtype or torch.float32, pin_memory=True)
+    if C_host.device.type != "cpu" or C_host.dtype not in (torch.float32, torch.bfloat16) or \
+            tuple(C_host.shape) != (M, N):
+        raise ValueError("C_host must be an (M, N) float32 or bfloat16 CPU tensor")
+    rc = load().sfc_gemm_host(M, N, K, ctypes.c_void_p(A_host.data_ptr()), ctypes.c_void_p(B_host.data_ptr()),
+                              ctypes.c_void_p(C_host.data_ptr()), _row_major_2d(A_host, "A"),
+                              _row_major_2d(B_host, "B"), _row_major_2d(C_host, "C"), _ab_code(A_host.dtype),
+                              B_LAYOUTS[b_layout], int(ca_c), SFC_F32 if C_host.dtype == torch.float32 else SFC_BF16,
+                              TILES[tile], int(panels), _stream_ptr(stream))
+    _check(rc, "sfc_gemm_host")
+    return C_host
+
+
+def matmul_host(A_host, B_host, C_host=None, *, ca_c: int = 0, out_dtype=None, stream=None, **kw):
+    """End-to-end call from HOST tensors: :func:`gemm_host`, then a
+    synchronisation of the stream.  Returns C_host, complete."""
     import torch
     s = stream or torch.cuda.current_stream()
-
-    def to_device(t):
-        # rows whose byte length is not a multiple of 16 get a padded row stride on the device
-        align = 16 // t.element_size()
-        ld = (t.shape[1] + align - 1) // align * align
-        if ld == t.shape[1]:
-            return t.to("cuda", non_blocking=True)
-        d = torch.empty((t.shape[0], ld), dtype=t.dtype, device="cuda")[:, : t.shape[1]]
-        d.copy_(t, non_blocking=True)
-        return d
-
-    with torch.cuda.stream(s):
-        A = to_device(A_host)
-        B = to_device(B_host)
-        C = gemm(A, B, ca_c=ca_c, out_dtype=out_dtype, stream=s, **kw)
-        if C_host is None:
-            C_host = torch.empty(C.shape, dtype=C.dtype, pin_memory=True)
-        C_host.copy_(C, non_blocking=True)
+    C_host = gemm_host(A_host, B_host, C_host, ca_c=ca_c, out_dtype=out_dtype, stream=s, **kw)
     s.synchronize()
     return C_host

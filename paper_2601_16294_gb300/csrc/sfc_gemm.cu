@@ -13,23 +13,26 @@
 #include "sfc_gemm.h"
 #include "sfc_gemm_kernel.cuh"
 #include "sfc_gemm_pair_kernel.cuh"
+#include "sfc_internal.h"
 
 #define SFC_API extern "C" __attribute__((visibility("default")))
 
 namespace sfc {
+
+thread_local int t_last_cuda_error = 0;
+
+int cuda_fail(cudaError_t e) {
+    t_last_cuda_error = static_cast<int>(e);
+    return SFC_ERR_CUDA;
+}
+
 namespace {
 
 constexpr int kMaxDevices = 64;
 constexpr int kMaxLayers = 4096;  // keeps the kernels' layer arithmetic in 32 bits
 constexpr uint64_t kDefaultTimeoutNs = 2000000000ull;  // 2 s per wait
 
-thread_local int t_last_cuda_error = 0;
 std::atomic<uint64_t> g_launch_seq{0};  // picks each launch's scheduler counter slot
-
-int cuda_fail(cudaError_t e) {
-    t_last_cuda_error = static_cast<int>(e);
-    return SFC_ERR_CUDA;
-}
 
 // ---------------------------------------------------------- per-device state
 
@@ -627,10 +630,13 @@ SFC_API int sfc_gemm_plan(int64_t M, int64_t N, int64_t K, int ca_c, int c_dtype
 }
 
 SFC_API int sfc_release(void) {
-    // The only memory the library holds between calls is what the device's
-    // default stream-ordered pool keeps after K-layer workspaces were freed.
+    // The library holds device memory between calls in two places: the staging
+    // slots of sfc_gemm_host, and what the device's default stream-ordered
+    // pool keeps after K-layer workspaces and repacked operands were freed.
     int dev;
     int rc = current_device(&dev);
+    if (rc != SFC_OK) return rc;
+    rc = host_release_staging();
     if (rc != SFC_OK) return rc;
     cudaMemPool_t pool;
     cudaError_t e = cudaDeviceGetDefaultMemPool(&pool, dev);

@@ -174,3 +174,29 @@ def test_gemm_ex2_validation_codes(lib):
     assert call_ex2(lib, bias=0x50002) == E.SFC_ERR_UNALIGNED                           # bias not 4-byte aligned
     assert call_ex2(lib, ab=3) == E.SFC_ERR_INVALID_ARG                                 # unknown input type
     assert call_ex2(lib, ab=1, K=256 * 129, ca_c=259) == E.SFC_ERR_INVALID_ARG          # 258 slabs of 128 k
+
+
+def call_host(lib, M=256, N=256, K=256, lda=None, ldb=None, ldc=None, ab=0, b_layout=0, c_dtype=0, panels=0,
+              a=0x10000, b=0x20000, c=0x30000):
+    ldb = (N if b_layout == 0 else K) if ldb is None else ldb
+    return lib.sfc_gemm_host(M, N, K, ctypes.c_void_p(a), ctypes.c_void_p(b), ctypes.c_void_p(c), lda or K, ldb,
+                             ldc or N, ab, b_layout, 1, c_dtype, 0, panels, None)
+
+
+def test_gemm_host_validation_codes(lib):
+    # every case fails on the host before any staging memory or stream is touched
+    E = binding
+    assert call_host(lib, M=0) == E.SFC_ERR_INVALID_ARG
+    assert call_host(lib, K=-1) == E.SFC_ERR_INVALID_ARG
+    assert call_host(lib, a=0) == E.SFC_ERR_INVALID_ARG                       # null host pointer
+    assert call_host(lib, c=0) == E.SFC_ERR_INVALID_ARG
+    assert call_host(lib, lda=255) == E.SFC_ERR_INVALID_ARG                   # rows of A shorter than K
+    assert call_host(lib, N=512, ldb=256) == E.SFC_ERR_INVALID_ARG            # rows of B shorter than N
+    assert call_host(lib, N=512, K=256, b_layout=1, ldb=200) == E.SFC_ERR_INVALID_ARG
+    assert call_host(lib, ldc=100) == E.SFC_ERR_INVALID_ARG
+    assert call_host(lib, ab=7) == E.SFC_ERR_INVALID_ARG
+    assert call_host(lib, b_layout=3) == E.SFC_ERR_INVALID_ARG
+    assert call_host(lib, c_dtype=5) == E.SFC_ERR_INVALID_ARG
+    assert call_host(lib, panels=-1) == E.SFC_ERR_INVALID_ARG
+    assert call_host(lib, a=0x10001) == E.SFC_ERR_UNALIGNED                   # bf16 at an odd address
+    assert call_host(lib, c=0x30002) == E.SFC_ERR_UNALIGNED                   # fp32 C at a 2-byte offset
