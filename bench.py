@@ -104,6 +104,9 @@ def parse_args():
     ap.add_argument("--ab", choices=("bf16", "e4m3", "e5m2"), default="bf16",
                     help="element type of A and B (8-bit floats use the tensor cores' 8-bit path)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--e2e-order", choices=("given", "largest_first"), default="largest_first",
+                    help="order in which the end-to-end step issues its host-buffer calls (largest first: the "
+                         "smaller calls' copies then overlap the largest call's GEMMs)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
     ap.add_argument("--no-cublas", action="store_true",
@@ -576,6 +579,8 @@ def run_e2e(args, mats, stream, world):
     host = []
     for m in mats:
         host.append((m, pin(m["A"]), host_b(m["B"]), torch.empty(m["C"].shape, dtype=m["C"].dtype, pin_memory=True)))
+    if args.e2e_order == "largest_first":
+        host.sort(key=lambda h: -h[0]["s"]["M"] * h[0]["s"]["N"] * h[0]["s"]["K"])
     h2d = sum(Ah.numel() * 2 + Bh.numel() * 2 for _, Ah, Bh, _ in host)
     d2h = sum(Ch.numel() * Ch.element_size() for _, _, _, Ch in host)
 
@@ -599,7 +604,8 @@ def run_e2e(args, mats, stream, world):
     flops = sum(2.0 * m["s"]["M"] * m["s"]["N"] * m["s"]["K"] for m in mats) * steps * world
     return {"value": round(flops / el / 1e12, 1), "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": d2h, "steps": steps,
-            "api": "paper_2601_16294_gb300.gemm_host -> sfc_gemm_host (C ABI, host buffers)"}
+            "api": "paper_2601_16294_gb300.gemm_host -> sfc_gemm_host (C ABI, host buffers)",
+            "order": args.e2e_order}
 
 
 def cpu_cores():

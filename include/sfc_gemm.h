@@ -22,8 +22,9 @@
  *
  * Conventions for every entry point:
  *   - sizes and leading dimensions are in ELEMENTS; lda >= K, ldb >= N, ldc >= N;
- *   - A, B, C and workspace are DEVICE pointers owned by the caller; the
- *     library never frees them and keeps no reference after the call returns;
+ *   - A, B, C and workspace are DEVICE pointers owned by the caller (HOST
+ *     pointers for sfc_gemm_host); the library never frees them and keeps no
+ *     reference after the call's work has completed;
  *   - calls that take a stream are asynchronous on that stream (NULL = the
  *     legacy default stream); arguments are validated on the host first and a
  *     validation error launches nothing;
@@ -289,14 +290,16 @@ int sfc_gemm_noalloc(int64_t M, int64_t N, int64_t K,
  * overlapped against the tile contraction.  No counterpart in the paper,
  * whose operands already sit in the memory the cores compute from.
  *
- * The output is cut into `panels` slices along the dimension of the larger
- * operand (rows of C when M >= N, else columns).  The smaller operand goes up
- * whole, then each slice of the larger one; the GEMM of a slice starts when
- * its slice has arrived, and its part of C goes back while the next slice
- * computes.  Slice edges fall on multiples of 512 rows or 256 columns (the
- * largest output tiles), so the result is bit-identical to sfc_gemm_ex2 over
- * the whole problem with the tile and ca_c that sfc_gemm_plan(M, N, K, ca_c,
- * c_dtype, tile, ab_dtype, b_layout, ...) reports, which every slice uses.
+ * A is cut into row panels and B into column panels.  After the first panel
+ * of each, the uploads follow a staircase: the next panel is the one that
+ * keeps the rows and columns of C covered so far closest to equal, and each
+ * upload is followed by the GEMM of the strip of C it completes, so GEMMs
+ * start after two panels have arrived and finished strips of C go back while
+ * later strips compute.  Panel edges fall on multiples of 512 rows or 256
+ * columns (the largest output tiles), so the result is bit-identical to
+ * sfc_gemm_ex2 over the whole problem with the tile and ca_c that
+ * sfc_gemm_plan(M, N, K, ca_c, c_dtype, tile, ab_dtype, b_layout, ...)
+ * reports, which every strip uses.
  *
  *   A, B, C: HOST pointers, row-major with row strides lda, ldb, ldc in
  *            elements (any stride; the device copies get 16-byte rows).  A and
@@ -308,11 +311,18 @@ int sfc_gemm_noalloc(int64_t M, int64_t N, int64_t K,
  *   ca_c, tile: as sfc_gemm_ex2 (0 / SFC_TILE_AUTO: chosen for the whole
  *            problem).  Order is the curve, assignment automatic, beta = 0,
  *            no bias.
- *   panels:  number of slices; 0 picks about one per 2048 rows or columns,
- *            at most 8.  Clamped to the number of 512-row (256-column) units.
- *   stream:  the GEMMs run on it; the copies run on two library streams that
- *            it waits for, so `stream` has finished with C once it has
- *            reached the end of this call's work.
+ *   panels:  number of panels of each operand; 0 picks about one per 2048
+ *            rows of A and per 2048 columns of B (per 8 KB of a row of an
+ *            N-major B, whose column panels are pitched copies), at most 8
+ *            each.  Clamped to 64 and to the number of 512-row (256-column)
+ *            units.
+ *   stream:  the uploads, GEMMs and downloads run on three library streams
+ *            (one set per device, shared by all calls); `stream` is made to
+ *            wait for the call's last download, so C is complete once
+ *            `stream` has reached that point.  The GEMMs touch staging memory
+ *            only and are not ordered after earlier work on `stream`, and a
+ *            call's GEMMs do not wait for the previous call's downloads:
+ *            calls issued back to back overlap in all three streams.
  * The call is asynchronous: it returns once everything is enqueued.  A and B
  * are read after it returns: they must hold their values when the call is
  * made (their uploads are NOT ordered after work already on `stream`) and

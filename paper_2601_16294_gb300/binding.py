@@ -266,7 +266,9 @@ def gemm_host(A_host, B_host, C_host=None, *, ca_c: int = 0, out_dtype=None, til
     ideally pinned; B is (K, N) for ``b_layout="kn"`` or (N, K) for ``"nk"``.
     C_host: (M, N) fp32 or bf16 CPU tensor, allocated pinned if not given.
     Asynchronous on ``stream``: C_host is complete once the stream has been
-    synchronised, and A and B must not change before then."""
+    synchronised, and A and B are read until then, so the caller keeps all
+    three tensors alive and A and B unchanged until it synchronises (a
+    temporary passed here could be freed and its memory reused too early)."""
     import torch
     M, K = A_host.shape
     if b_layout == "kn":

@@ -2,21 +2,29 @@
 // A, B and C in host memory, the host<->device copies pipelined against the
 // tile contraction.
 //
-// The output is cut into panels along the dimension of the larger operand
-// (rows of C when A is at least as large as B, else columns).  The smaller
-// operand is uploaded whole, then each panel's slice of the larger one; the
-// GEMM of panel p starts as soon as its slice has arrived and its slice of C
-// is copied back while panel p + 1 computes.  Panel edges fall on multiples
-// of the largest output tile, so every output tile is contracted exactly as a
-// single sfc_gemm_ex2 call over the whole problem with the same tile and layer
-// count would contract it: the results are bit-identical.
+// A is cut into row panels and B into column panels.  The uploads follow a
+// staircase: after the first panel of each, the next upload is the panel that
+// keeps the rows and columns covered so far closest to equal, and each upload
+// is followed by the GEMM of the strip of C it completes (the new rows against
+// every column present, or the new columns against every row present).  The
+// GEMMs thus start after two panels instead of a whole operand, and C's
+// strips go back while later strips compute.  This is the idea of the curve
+// order one level up: the output is grown so that what is already resident
+// (here in device memory, behind the host link) is reused as much as possible
+// per byte moved.  Panel edges fall on multiples of the largest output tile,
+// so every output tile is contracted exactly as a single sfc_gemm_ex2 call
+// over the whole problem with the same tile and layer count would contract it:
+// the results are bit-identical.
 //
-// Streams: uploads run on a library stream `up`, downloads on `down`, the
-// GEMMs on the caller's stream, ordered by events.  Device memory comes from
-// staging slots owned by the library: a slot holds one call's device copies of
-// A, B and C and is reused once the event recorded at the end of that call has
-// completed, so calls issued back to back overlap (the next call's uploads
-// proceed while this call computes).  sfc_release frees the slots.
+// Streams: uploads run on a library stream `up`, GEMMs on `comp`, downloads
+// on `down`, ordered by events; the caller's stream only waits for the call's
+// last download.  The GEMMs read and write staging memory alone, so they need
+// no order against the caller's earlier work, and the next call's GEMMs do not
+// wait for this call's downloads: consecutive calls overlap their GEMMs, their
+// uploads and their downloads.  Device memory comes from staging slots owned
+// by the library: a slot holds one call's device copies of A, B and C and is
+// reused once the event recorded after that call's last download has
+// completed.  sfc_release frees the slots.
 #include <cuda_runtime.h>
 
 #include <cstdint>
@@ -32,18 +40,21 @@ namespace sfc_host {
 namespace {
 
 constexpr int kMaxDevices = 64;
-constexpr int kMaxPanels = 64;
+constexpr int64_t kMaxPanels = 64;
 constexpr int64_t kPanelRowsM = 512;    // rows of the largest output tile (two stacked 2-SM pairs)
 constexpr int64_t kPanelColsN = 256;    // columns of the widest output tile
 constexpr int64_t kAutoPanelSpan = 2048;  // automatic panels: about this many rows or columns each
-constexpr int kAutoMaxPanels = 8;
+constexpr int64_t kAutoMaxPanels = 8;
+// Pitched host<->device copies run below the link's rate for short rows
+// (measured on GB300: 4 KB rows 175 GB/s, 8 KB 188, 16 KB and up 211).
+constexpr int64_t kMinPitchedRowBytes = 8192;
 
 int fail(cudaError_t e) { return sfc::cuda_fail(e); }
 
 struct Slot {
     void* base = nullptr;
     size_t bytes = 0;
-    cudaEvent_t done = nullptr;  // recorded on the caller's stream after the call's last use
+    cudaEvent_t done = nullptr;  // recorded after the call's last download
     bool recorded = false;
     bool taken = false;          // reserved by a call that is still enqueueing
 };
@@ -51,7 +62,7 @@ struct Slot {
 struct Pipe {
     std::mutex mu;
     bool ready = false;
-    cudaStream_t up = nullptr, down = nullptr;
+    cudaStream_t up = nullptr, comp = nullptr, down = nullptr;
     std::vector<Slot> slots;
     size_t held = 0, cap = 0;
 };
@@ -64,6 +75,7 @@ int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
 int pipe_setup(Pipe& p) {
     if (p.ready) return SFC_OK;
     cudaError_t e = cudaStreamCreateWithFlags(&p.up, cudaStreamNonBlocking);
+    if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&p.comp, cudaStreamNonBlocking);
     if (e == cudaSuccess) e = cudaStreamCreateWithFlags(&p.down, cudaStreamNonBlocking);
     size_t free_b = 0, total_b = 0;
     if (e == cudaSuccess) e = cudaMemGetInfo(&free_b, &total_b);
@@ -131,6 +143,26 @@ int acquire(Pipe& p, size_t need, size_t* out) {
     p.slots[best].taken = true;
     *out = best;
     return SFC_OK;
+}
+
+// Output rows [r0, r1) x columns [c0, c1) computed by one GEMM.
+struct Region {
+    int64_t r0, r1, c0, c1;
+};
+
+// Span of a panel along a dimension of `extent` elements (`units` multiples of
+// `unit`): `panels` panels if given, else about one per `auto_span` elements,
+// at most kAutoMaxPanels; always a whole number of units.
+int64_t panel_span(int64_t extent, int64_t units, int64_t unit, int panels, int64_t auto_span) {
+    int64_t np = panels;
+    if (np == 0) {
+        np = (extent + auto_span - 1) / auto_span;
+        if (np > kAutoMaxPanels) np = kAutoMaxPanels;
+    }
+    if (np > kMaxPanels) np = kMaxPanels;
+    if (np > units) np = units;
+    if (np < 1) np = 1;
+    return (units + np - 1) / np * unit;
 }
 
 // Row-major copy of `rows` rows of `width` bytes between pitched buffers.
@@ -206,20 +238,16 @@ SFC_API int sfc_gemm_host(int64_t M, int64_t N, int64_t K, const void* A, const 
     const size_t b_bytes = static_cast<size_t>(round_up(b_rows * ldb_d * eb, 256));
     const size_t c_bytes = static_cast<size_t>(round_up(M * ldc_d * ob, 256));
 
-    // panels along M when A is at least as large as B, else along N
-    const bool by_rows = M >= N;
-    const int64_t extent = by_rows ? M : N, unit = by_rows ? kPanelRowsM : kPanelColsN;
-    const int64_t units = (extent + unit - 1) / unit;
-    int64_t np = panels;
-    if (np == 0) {
-        np = (extent + kAutoPanelSpan - 1) / kAutoPanelSpan;
-        if (np > kAutoMaxPanels) np = kAutoMaxPanels;
-    }
-    if (np > units) np = units;
-    if (np > kMaxPanels) np = kMaxPanels;
-    if (np < 1) np = 1;
-    const int64_t per = (units + np - 1) / np * unit;  // panel span, a multiple of the tile
-    np = (extent + per - 1) / per;
+    // row panels of A (multiples of 512 rows) and column panels of B (multiples of 256 columns)
+    const int64_t m_units = (M + kPanelRowsM - 1) / kPanelRowsM, n_units = (N + kPanelColsN - 1) / kPanelColsN;
+    // a column panel of an N-major B is a pitched copy: keep its rows at least 8 KB long
+    const int64_t col_span = b_nk ? kAutoPanelSpan : (kMinPitchedRowBytes / eb > kAutoPanelSpan
+                                                         ? kMinPitchedRowBytes / eb : kAutoPanelSpan);
+    const int64_t per_m = panel_span(M, m_units, kPanelRowsM, panels, kAutoPanelSpan);
+    const int64_t per_n = panel_span(N, n_units, kPanelColsN, panels, col_span);
+    const int64_t pm = (M + per_m - 1) / per_m, pn = (N + per_n - 1) / per_n;
+    auto row_end = [&](int64_t i) { return i * per_m < M ? i * per_m : M; };
+    auto col_end = [&](int64_t j) { return j * per_n < N ? j * per_n : N; };
 
     std::lock_guard<std::mutex> lock(p.mu);
     rc = pipe_setup(p);
@@ -235,64 +263,78 @@ SFC_API int sfc_gemm_host(int64_t M, int64_t N, int64_t K, const void* A, const 
     const char* Bh = static_cast<const char*>(B);
     char* Ch = static_cast<char*>(C);
 
+    auto upload_a = [&](int64_t i) {
+        const int64_t r0 = row_end(i), r1 = row_end(i + 1);
+        return copy_rows(Ad + r0 * lda_d * eb, lda_d * eb, Ah + r0 * lda * eb, lda * eb, K * eb, r1 - r0,
+                         cudaMemcpyHostToDevice, p.up);
+    };
+    auto upload_b = [&](int64_t j) {
+        const int64_t c0 = col_end(j), c1 = col_end(j + 1);
+        if (b_nk)
+            return copy_rows(Bd + c0 * ldb_d * eb, ldb_d * eb, Bh + c0 * ldb * eb, ldb * eb, K * eb, c1 - c0,
+                             cudaMemcpyHostToDevice, p.up);
+        return copy_rows(Bd + c0 * eb, ldb_d * eb, Bh + c0 * eb, ldb * eb, (c1 - c0) * eb, K,
+                         cudaMemcpyHostToDevice, p.up);
+    };
+
     Events evs;
+    std::vector<Region> regions;
     std::vector<cudaEvent_t> computed;
-    // the operand every panel needs goes up first
-    if (by_rows)
-        e = copy_rows(Bd, ldb_d * eb, Bh, ldb * eb, b_cols * eb, b_rows, cudaMemcpyHostToDevice, p.up);
-    else
-        e = copy_rows(Ad, lda_d * eb, Ah, lda * eb, K * eb, M, cudaMemcpyHostToDevice, p.up);
-    for (int64_t i = 0; i < np && e == cudaSuccess && rc == SFC_OK; ++i) {
-        const int64_t lo = i * per, hi = (lo + per < extent) ? lo + per : extent;
-        const void *a = Ad, *b = Bd;
-        void* c = Cd;
-        int64_t m = M, n = N;
-        if (by_rows) {
-            e = copy_rows(Ad + lo * lda_d * eb, lda_d * eb, Ah + lo * lda * eb, lda * eb, K * eb, hi - lo,
-                          cudaMemcpyHostToDevice, p.up);
-            a = Ad + lo * lda_d * eb;
-            c = Cd + lo * ldc_d * ob;
-            m = hi - lo;
-        } else if (b_nk) {
-            e = copy_rows(Bd + lo * ldb_d * eb, ldb_d * eb, Bh + lo * ldb * eb, ldb * eb, K * eb, hi - lo,
-                          cudaMemcpyHostToDevice, p.up);
-            b = Bd + lo * ldb_d * eb;
-            c = Cd + lo * ob;
-            n = hi - lo;
-        } else {
-            e = copy_rows(Bd + lo * eb, ldb_d * eb, Bh + lo * eb, ldb * eb, (hi - lo) * eb, K,
-                          cudaMemcpyHostToDevice, p.up);
-            b = Bd + lo * eb;
-            c = Cd + lo * ob;
-            n = hi - lo;
-        }
-        if (e == cudaSuccess) e = join(s, p.up, evs);
-        if (e != cudaSuccess) break;
-        rc = sfc_gemm_ex2(m, n, K, a, b, c, lda_d, ldb_d, ldc_d, ab_dtype, b_layout, 0.0f, nullptr, c_used,
-                          c_dtype, SFC_ORDER_SFC, SFC_ASSIGN_AUTO, static_cast<sfc_tile_t>(tile_used), nullptr, 0,
-                          stream);
-        if (rc != SFC_OK) break;
+    // GEMM of the block of C that the panels uploaded so far newly cover
+    auto compute = [&](Region g) -> cudaError_t {
+        cudaError_t r = join(p.comp, p.up, evs);
+        if (r != cudaSuccess) return r;
+        const char* a = Ad + g.r0 * lda_d * eb;
+        const char* b = b_nk ? Bd + g.c0 * ldb_d * eb : Bd + g.c0 * eb;
+        char* c = Cd + g.r0 * ldc_d * ob + g.c0 * ob;
+        rc = sfc_gemm_ex2(g.r1 - g.r0, g.c1 - g.c0, K, a, b, c, lda_d, ldb_d, ldc_d, ab_dtype, b_layout, 0.0f,
+                          nullptr, c_used, c_dtype, SFC_ORDER_SFC, SFC_ASSIGN_AUTO,
+                          static_cast<sfc_tile_t>(tile_used), nullptr, 0, p.comp);
+        if (rc != SFC_OK) return cudaSuccess;
         cudaEvent_t done;
-        e = evs.make(&done);
-        if (e == cudaSuccess) e = cudaEventRecord(done, s);
-        if (e == cudaSuccess) computed.push_back(done);
+        r = evs.make(&done);
+        if (r == cudaSuccess) r = cudaEventRecord(done, p.comp);
+        if (r == cudaSuccess) {
+            regions.push_back(g);
+            computed.push_back(done);
+        }
+        return r;
+    };
+
+    // Staircase walk: after the first row and column panel, upload whichever
+    // panel keeps the covered rows and columns closest to equal (most output
+    // per uploaded byte), and compute the strip of C it completes.
+    e = upload_a(0);
+    if (e == cudaSuccess) e = upload_b(0);
+    if (e == cudaSuccess) e = compute(Region{0, row_end(1), 0, col_end(1)});
+    int64_t a = 1, b = 1;
+    while (e == cudaSuccess && rc == SFC_OK && (a < pm || b < pn)) {
+        const bool take_a = b >= pn || (a < pm && row_end(a) <= col_end(b));
+        if (take_a) {
+            e = upload_a(a);
+            if (e == cudaSuccess) e = compute(Region{row_end(a), row_end(a + 1), 0, col_end(b)});
+            ++a;
+        } else {
+            e = upload_b(b);
+            if (e == cudaSuccess) e = compute(Region{0, row_end(a), col_end(b), col_end(b + 1)});
+            ++b;
+        }
     }
     // downloads are enqueued after every GEMM, so a blocking copy into pageable memory cannot hold one back
     for (size_t i = 0; i < computed.size() && e == cudaSuccess; ++i) {
-        const int64_t lo = static_cast<int64_t>(i) * per, hi = (lo + per < extent) ? lo + per : extent;
+        const Region& g = regions[i];
         e = cudaStreamWaitEvent(p.down, computed[i], 0);
-        if (e != cudaSuccess) break;
-        if (by_rows)
-            e = copy_rows(Ch + lo * ldc * ob, ldc * ob, Cd + lo * ldc_d * ob, ldc_d * ob, N * ob, hi - lo,
-                          cudaMemcpyDeviceToHost, p.down);
-        else
-            e = copy_rows(Ch + lo * ob, ldc * ob, Cd + lo * ob, ldc_d * ob, (hi - lo) * ob, M,
-                          cudaMemcpyDeviceToHost, p.down);
+        if (e == cudaSuccess)
+            e = copy_rows(Ch + g.r0 * ldc * ob + g.c0 * ob, ldc * ob, Cd + g.r0 * ldc_d * ob + g.c0 * ob, ldc_d * ob,
+                          (g.c1 - g.c0) * ob, g.r1 - g.r0, cudaMemcpyDeviceToHost, p.down);
     }
-    // the caller's stream ends after everything this call enqueued; the slot is free after that
-    cudaError_t j = join(s, p.up, evs);
-    if (j == cudaSuccess) j = join(s, p.down, evs);
-    if (j == cudaSuccess) j = cudaEventRecord(p.slots[si].done, s);
+    // the slot is free, and the caller's stream may go on, after everything
+    // this call enqueued (downloads wait for their GEMMs, GEMMs for their
+    // uploads; the joins also cover a call that stopped early)
+    cudaError_t j = join(p.down, p.up, evs);
+    if (j == cudaSuccess) j = join(p.down, p.comp, evs);
+    if (j == cudaSuccess) j = cudaEventRecord(p.slots[si].done, p.down);
+    if (j == cudaSuccess) j = cudaStreamWaitEvent(s, p.slots[si].done, 0);
     Slot& slot = p.slots[si];
     slot.taken = false;
     if (j == cudaSuccess) {

@@ -1,10 +1,11 @@
 """The host-buffer entry point (sfc_gemm_host): operands and result in host
-memory, copies pipelined against the GEMM in row or column slices.
+memory, copies pipelined against the GEMM along a staircase of row panels of
+A and column panels of B.
 
-Each slice is a GEMM over whole output tiles with the plan of the full
+Each strip of C is a GEMM over whole output tiles with the plan of the full
 problem, so the result must equal sfc_gemm_ex2 on device copies (same tile,
-same layer count) bit for bit, for every slicing; integer-valued inputs must
-equal the oracle exactly.
+same layer count) bit for bit, for every panel count; integer-valued inputs
+must equal the oracle exactly.
 """
 import numpy as np
 import pytest
@@ -50,12 +51,14 @@ def on_device(sfc, A, B, *, b_layout="kn", out_dtype=torch.float32, ca_c=0, tile
 
 
 CASES = [
-    # M, N, K, lda, ldb: column slices (M < N), odd K rows on the host
+    # M, N, K, lda, ldb: odd K rows on the host
     (1000, 1200, 2500, 2501, 1203),
-    # row slices (M >= N), K not a multiple of 64, padded host rows
+    # K not a multiple of 64, padded host rows, more row than column panels
     (3000, 700, 1001, 1001, 705),
-    # several 512-row units, aligned rows (one-piece copies)
+    # several 512-row units, aligned rows (one-piece copies), one column panel
     (2600, 512, 640, 640, 512),
+    # several column panels of 256 columns, one row panel
+    (300, 2900, 320, 320, 2900),
     # one tile
     (100, 60, 40, 40, 60),
 ]
@@ -114,7 +117,9 @@ def test_fp8_inputs(sfc, fmt):
 
 def test_calls_in_flight_overlap_and_stay_correct(sfc):
     # several calls enqueued back to back, one synchronisation at the end:
-    # each takes its own staging slot
+    # each takes its own staging slot.  The host operands are read after the
+    # calls return, so they are kept alive (and unchanged) until the stream
+    # has synchronised.
     shapes = [(2048, 2048, 1024), (700, 3000, 512), (4096, 1024, 2048), (512, 512, 4096)]
     jobs = []
     s = torch.cuda.current_stream()
@@ -122,21 +127,22 @@ def test_calls_in_flight_overlap_and_stay_correct(sfc):
         A, B = synth.gemm_inputs(M, N, K, "uniform", seed=40 + i)
         A, B = A.contiguous(), B.contiguous()
         Ch = torch.full((M, N), float("nan"), dtype=torch.bfloat16, pin_memory=True)
-        sfc.gemm_host(host(A), host(B), Ch, stream=s)
-        jobs.append((A, B, Ch))
+        jobs.append((A, B, host(A), host(B), Ch, on_device(sfc, A, B, out_dtype=torch.bfloat16)))
+    for _, _, Ah, Bh, Ch, _ in jobs:
+        sfc.gemm_host(Ah, Bh, Ch, stream=s)
     s.synchronize()
-    for A, B, Ch in jobs:
-        assert torch.equal(Ch, on_device(sfc, A, B, out_dtype=torch.bfloat16))
+    for _, _, _, _, Ch, ref in jobs:
+        assert torch.equal(Ch, ref)
     # the same slots serve the next round of calls
-    for A, B, Ch in jobs:
+    for _, _, Ah, Bh, Ch, _ in jobs:
         Ch.fill_(float("nan"))
-        sfc.gemm_host(host(A), host(B), Ch, stream=s)
+        sfc.gemm_host(Ah, Bh, Ch, stream=s)
     s.synchronize()
-    for A, B, Ch in jobs:
-        assert torch.equal(Ch, on_device(sfc, A, B, out_dtype=torch.bfloat16))
+    for _, _, _, _, Ch, ref in jobs:
+        assert torch.equal(Ch, ref)
     sfc.release()
-    A, B, Ch = jobs[0]
-    assert torch.equal(sfc.matmul_host(host(A), host(B), out_dtype=torch.bfloat16), Ch)
+    _, _, Ah, Bh, _, ref = jobs[0]
+    assert torch.equal(sfc.matmul_host(Ah, Bh, out_dtype=torch.bfloat16), ref)
 
 
 def test_pageable_memory_and_padded_c(sfc):
