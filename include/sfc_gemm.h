@@ -143,8 +143,9 @@ size_t sfc_gemm_workspace_size(int64_t M, int64_t N, int64_t K, int ca_c);
  *   ca_c: number of K layers, 1 <= ca_c <= min(ceil(K/64), 4096).  Layer l contracts K
  *         tiles [floor(l*Kt/ca_c), floor((l+1)*Kt/ca_c)) of the Kt = ceil(K/64)
  *         64-wide K tiles.  For ca_c > 1 the library takes its fp32 workspace
- *         from a stream-ordered pool (cudaMallocAsync / cudaFreeAsync on
- *         `stream`).  ca_c = 0 lets the library choose the count (and the
+ *         from its own stream-ordered pool (allocated and freed in order on
+ *         `stream`; freed memory stays in the pool for the next call until
+ *         sfc_release).  ca_c = 0 lets the library choose the count (and the
  *         tile) from a model of the call's time on this device: waves of
  *         items times the length of a layer, plus the reduction's cost for
  *         more than one layer (the replication factor choice of Sec. II-D,
@@ -230,10 +231,11 @@ int sfc_gemm_plan(int64_t M, int64_t N, int64_t K, int ca_c, int c_dtype, int ti
                   int ab_dtype, int b_layout, int *out_tile, int *out_ca_c);
 
 /*
- * sfc_release -- returns to the driver the device memory the library's
- * stream-ordered workspace allocations left cached in the current device's
- * default memory pool (synchronizes the device first).  The library keeps no
- * other allocation between calls.  SFC_OK, or SFC_ERR_CUDA.
+ * sfc_release -- returns to the driver the device memory the library holds
+ * between calls on the current device: the staging slots of sfc_gemm_host and
+ * what its stream-ordered pool keeps after K-layer workspaces and repacked
+ * operands were freed (synchronizes the device first).  SFC_OK, SFC_ERR_CUDA
+ * or SFC_ERR_UNSUPPORTED.
  */
 int sfc_release(void);
 

@@ -158,7 +158,8 @@ def plan(M: int, N: int, K: int, ca_c: int = 0, out_dtype=None, tile="auto", in_
 
 
 def release() -> None:
-    """Give the memory cached by the library's workspace allocations back to the driver."""
+    """Give the device memory the library keeps between calls (host-entry staging
+    slots, its workspace pool) back to the driver."""
     _check(load().sfc_release(), "sfc_release")
 
 

@@ -116,6 +116,9 @@ struct DeviceInfo {
     int serpentine = 0;
     int one_item_per_worker = 0;
     int workers[kNumVariants] = {0, 0, 0, 0, 0};  // co-resident workers (blocks or clusters) per variant
+    // the library's stream-ordered pool (layer workspaces, repacked operands): it keeps
+    // freed memory for reuse, so a call after a synchronisation does not map new pages
+    cudaMemPool_t pool = nullptr;
 };
 DeviceInfo g_devices[kMaxDevices];
 
@@ -164,6 +167,16 @@ int device_setup(DeviceInfo** info) {
         if (e == cudaSuccess) e = set_attrs<__nv_bfloat16, false>();
         if (e == cudaSuccess) e = set_attrs<float, true>();
         if (e == cudaSuccess) e = set_attrs<__nv_bfloat16, true>();
+        if (e != cudaSuccess) { d.status = cuda_fail(e); return; }
+        cudaMemPoolProps props;
+        std::memset(&props, 0, sizeof(props));
+        props.allocType = cudaMemAllocationTypePinned;
+        props.handleTypes = cudaMemHandleTypeNone;
+        props.location.type = cudaMemLocationTypeDevice;
+        props.location.id = dev;
+        e = cudaMemPoolCreate(&d.pool, &props);
+        uint64_t keep = UINT64_MAX;  // released only by sfc_release
+        if (e == cudaSuccess) e = cudaMemPoolSetAttribute(d.pool, cudaMemPoolAttrReleaseThreshold, &keep);
         if (e != cudaSuccess) { d.status = cuda_fail(e); return; }
         for (int v = 0; v < kNumVariants; ++v) {
             if (!variant_pair(v)) {
@@ -435,7 +448,8 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
         const int64_t rows = which == 0 ? M : b_rows, cols = which == 0 ? K : b_cols;
         const int64_t ld_src = which == 0 ? lda : ldb;
         const int64_t ld_dst = (cols + row_align - 1) / row_align * row_align;
-        cudaError_t e = cudaMallocAsync(&packed[which], static_cast<size_t>(rows * ld_dst * eb), stream);
+        cudaError_t e = cudaMallocFromPoolAsync(&packed[which], static_cast<size_t>(rows * ld_dst * eb), dev->pool,
+                                                stream);
         if (e != cudaSuccess) {
             release_packed();
             return cuda_fail(e);
@@ -508,7 +522,7 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     void* ws = workspace;
     bool pooled = false;
     if (ca_c > 1 && !ws) {
-        cudaError_t e = cudaMallocAsync(&ws, ws_need, stream);
+        cudaError_t e = cudaMallocFromPoolAsync(&ws, ws_need, dev->pool, stream);
         if (e != cudaSuccess) {
             release_packed();
             return cuda_fail(e);
@@ -631,17 +645,15 @@ SFC_API int sfc_gemm_plan(int64_t M, int64_t N, int64_t K, int ca_c, int c_dtype
 
 SFC_API int sfc_release(void) {
     // The library holds device memory between calls in two places: the staging
-    // slots of sfc_gemm_host, and what the device's default stream-ordered
-    // pool keeps after K-layer workspaces and repacked operands were freed.
-    int dev;
-    int rc = current_device(&dev);
+    // slots of sfc_gemm_host, and what its stream-ordered pool keeps after
+    // K-layer workspaces and repacked operands were freed.
+    DeviceInfo* dev = nullptr;
+    int rc = device_setup(&dev);
     if (rc != SFC_OK) return rc;
     rc = host_release_staging();
     if (rc != SFC_OK) return rc;
-    cudaMemPool_t pool;
-    cudaError_t e = cudaDeviceGetDefaultMemPool(&pool, dev);
-    if (e == cudaSuccess) e = cudaDeviceSynchronize();
-    if (e == cudaSuccess) e = cudaMemPoolTrimTo(pool, 0);
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e == cudaSuccess) e = cudaMemPoolTrimTo(dev->pool, 0);
     return e == cudaSuccess ? SFC_OK : cuda_fail(e);
 }
 
