@@ -104,6 +104,10 @@ def parse_args():
     ap.add_argument("--ab", choices=("bf16", "e4m3", "e5m2"), default="bf16",
                     help="element type of A and B (8-bit floats use the tensor cores' 8-bit path)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--out", choices=("workload", "f32", "bf16"), default="workload",
+                    help="output type of every shape (default: the workload's own)")
+    ap.add_argument("--k-block-factor", type=int, default=1,
+                    help="passes over each layer's K range (Listing 1's k_block_factor); 1 = one pass")
     ap.add_argument("--e2e-order", choices=("given", "largest_first"), default="largest_first",
                     help="order in which the end-to-end step issues its host-buffer calls (largest first: the "
                          "smaller calls' copies then overlap the largest call's GEMMs)")
@@ -123,6 +127,9 @@ def workload_shapes(args):
     if args.ca_c is not None:
         for s in shapes:
             s["cs"] = (args.ca_c,)
+    if args.out != "workload":
+        for s in shapes:
+            s["out"] = args.out
     return shapes
 
 
@@ -311,7 +318,7 @@ def run_ours(args, rank, local, world):
 
     def call(m, c):
         sfc.gemm(m["Ad"], m["Bd"], m["C"], ca_c=c, order=args.order, assign=args.assign, stream=stream,
-                 b_layout=args.b_layout)
+                 b_layout=args.b_layout, k_block_factor=args.k_block_factor)
 
     # pick the K-layer count per shape where several are listed (timed, warm)
     cs_report = {}
@@ -320,7 +327,7 @@ def run_ours(args, rank, local, world):
             continue
         Kt = (m["s"]["K"] + 63) // 64
         best = None
-        for c in [c for c in m["s"]["cs"] if c <= Kt]:
+        for c in [c for c in m["s"]["cs"] if c * args.k_block_factor <= Kt]:
             for _ in range(2):
                 call(m, c)
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -411,13 +418,13 @@ def run_ours(args, rank, local, world):
         reps = max(2 * copies, min(400, int(0.05 / max(roofline_time_s(s_, peaks, args.ab)[0], 1e-6))))
         for a, b in extra:
             sfc.gemm(a, b, m["C"], ca_c=m["c"], order=args.order, assign=args.assign, stream=stream,
-                     b_layout=args.b_layout)
+                     b_layout=args.b_layout, k_block_factor=args.k_block_factor)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
         for r in range(reps):
             a, b = extra[r % copies]
             sfc.gemm(a, b, m["C"], ca_c=m["c"], order=args.order, assign=args.assign, stream=stream,
-                     b_layout=args.b_layout)
+                     b_layout=args.b_layout, k_block_factor=args.k_block_factor)
         e1.record(stream)
         torch.cuda.synchronize()
         b2b_ms.append(e0.elapsed_time(e1) / reps)
@@ -468,7 +475,14 @@ def run_ours(args, rank, local, world):
                     peaks["source"], "sustained" if sustained else "burst", elapsed_ms,
                     "" if args.ab == "bf16" else " x %.1f, the nominal 8-bit / bf16 ratio" % ratio),
                 "frac_of_burst_peak": round(achieved / burst, 4)}
-    launches = args.steps * sum(1 if m["c"] == 1 else 2 for m in mats)
+    def launches_per_call(m):
+        # GEMM launches (one per K block) plus the reduction when partials go through the workspace
+        c = m["c"] if m["c"] else sfc.plan(m["s"]["M"], m["s"]["N"], m["s"]["K"], 0, out_dtype=m["C"].dtype,
+                                           in_dtype=m["Ad"].dtype, b_layout=args.b_layout)[1]
+        kbf = args.k_block_factor
+        return kbf + (1 if c > 1 or (kbf > 1 and m["C"].dtype != torch.float32) else 0)
+
+    launches = args.steps * sum(launches_per_call(m) for m in mats)
     desc = WORKLOADS[args.workload]["desc"] if not args.sizes else "square sweep sizes %s" % args.sizes
     result = {
         "metric": METRIC, "value": round(value, 1), "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
@@ -476,7 +490,7 @@ def run_ours(args, rank, local, world):
         "scaling": "weak", "vs_baseline": None, "dtype": args.ab,
         "data": "synthetic (seeded %s %s)" % (",".join(sorted({m["s"]["kind"] for m in mats})), args.ab),
         "config": {"workload": desc, "order": args.order, "assign": args.assign, "b_layout": args.b_layout,
-                   "inputs": args.ab,
+                   "inputs": args.ab, "k_block_factor": args.k_block_factor,
                    "parallelism": "replicas" if world > 1 else "single GPU",
                    "l2": "inputs larger than L2 between reuses: one step runs every shape once, so a shape's "
                          "operands are re-read only after the other shapes' traffic has passed through L2",

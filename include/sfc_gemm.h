@@ -219,6 +219,45 @@ int sfc_gemm_ex2(int64_t M, int64_t N, int64_t K,
                  void *workspace, size_t workspace_bytes, void *stream);
 
 /*
+ * sfc_gemm_ex3 -- sfc_gemm_ex2 with Listing 1's K-block loop: k_block_factor
+ * passes over K (Sec. II-D; the loop over ik, whose blocks set the A and B
+ * panel depth k' of Sec. II-E).  Pass ik contracts block ik of every layer's
+ * K slabs -- layer l's slabs [L_l, L_(l+1)) split as
+ * [L_l + floor(ik * n_l / kbf), L_l + floor((ik + 1) * n_l / kbf)), n_l =
+ * L_(l+1) - L_l -- for every output tile (one launch per pass), and adds it
+ * into that layer's copy of C, which stays where it is between passes: an fp32
+ * C with one layer is accumulated in place (pass 0 also applies beta and
+ * bias), otherwise the copies are fp32 workspace and the final reduction
+ * applies beta, bias and the output rounding.  Sums are fp32, pass by pass in
+ * order, so the rounding differs from k_block_factor = 1 but not between
+ * orders, assignments or runs.
+ *   k_block_factor: 1..64, and every layer must hold at least that many
+ *     slabs (a slab is 64 values of k for bf16, 128 for the 8-bit kinds):
+ *     ca_c * k_block_factor <= ceil(K / slab) for ca_c > 0; with ca_c = 0 the
+ *     planner keeps to it.  1 is exactly sfc_gemm_ex2.
+ *   workspace: at least sfc_gemm_workspace_size2(M, N, K, ca_c,
+ *     k_block_factor, c_dtype) bytes, or NULL to use the library's pool.
+ * Errors: as sfc_gemm_ex2.
+ */
+int sfc_gemm_ex3(int64_t M, int64_t N, int64_t K,
+                 const void *A, const void *B, void *C,
+                 int64_t lda, int64_t ldb, int64_t ldc,
+                 int ab_dtype, int b_layout, float beta, const float *bias,
+                 int ca_c, int k_block_factor, sfc_dtype_t c_dtype,
+                 sfc_order_t order, sfc_assign_t assign, sfc_tile_t tile,
+                 void *workspace, size_t workspace_bytes, void *stream);
+
+/*
+ * sfc_gemm_workspace_size2 -- bytes of fp32 workspace sfc_gemm_ex3 needs:
+ * ca_c copies of C (M * round_up(N, 4) * 4 bytes each) when ca_c > 1; one copy
+ * when ca_c == 1, k_block_factor > 1 and c_dtype is SFC_BF16; else 0.  For
+ * ca_c == 0 the size for the most layers the planner may choose, at most
+ * ceil(K/64) / k_block_factor.  0 for invalid arguments.  Needs no GPU.
+ */
+size_t sfc_gemm_workspace_size2(int64_t M, int64_t N, int64_t K, int ca_c, int k_block_factor,
+                                sfc_dtype_t c_dtype);
+
+/*
  * sfc_gemm_plan -- the tile and K-layer count sfc_gemm_ex2 would use for these
  * arguments on the current device (ca_c = 0: the library's choice; ca_c >= 1:
  * that count with the tile AUTO or `tile` picks).  No kernel runs.

@@ -44,7 +44,8 @@ def _ab_code(dtype) -> int:
 
 EXPORTS = ("sfc_tile_order", "sfc_tile_order_device", "sfc_gemm_workspace_size", "sfc_gemm", "sfc_gemm_ex",
            "sfc_get_device_status", "sfc_last_cuda_error", "sfc_num_workers", "sfc_debug_force_timeout",
-           "sfc_gemm_noalloc", "sfc_gemm_plan", "sfc_release", "sfc_gemm_ex2", "sfc_gemm_host")
+           "sfc_gemm_noalloc", "sfc_gemm_plan", "sfc_release", "sfc_gemm_ex2", "sfc_gemm_host", "sfc_gemm_ex3",
+           "sfc_gemm_workspace_size2")
 NOALLOC_SCRATCH_BYTES = 32 << 20
 
 
@@ -98,8 +99,12 @@ def load():
                                      i32, i32, i32, i32, vp, sz, vp]
         lib.sfc_release.argtypes = []
         lib.sfc_gemm_host.argtypes = [i64, i64, i64, vp, vp, vp, i64, i64, i64, i32, i32, i32, i32, i32, i32, vp]
+        lib.sfc_gemm_ex3.argtypes = [i64, i64, i64, vp, vp, vp, i64, i64, i64, i32, i32, ctypes.c_float, vp, i32,
+                                     i32, i32, i32, i32, i32, vp, sz, vp]
+        lib.sfc_gemm_workspace_size2.argtypes = [i64, i64, i64, i32, i32, i32]
+        lib.sfc_gemm_workspace_size2.restype = sz
         for name in EXPORTS:
-            if name != "sfc_gemm_workspace_size":
+            if name not in ("sfc_gemm_workspace_size", "sfc_gemm_workspace_size2"):
                 getattr(lib, name).restype = ctypes.c_int
         _lib = lib
         return lib
@@ -137,8 +142,11 @@ def tile_order_device(Mt: int, Nt: int, stream=None):
 
 # ------------------------------------------------------------------- GEMM
 
-def workspace_size(M: int, N: int, K: int, ca_c: int) -> int:
-    return int(load().sfc_gemm_workspace_size(int(M), int(N), int(K), int(ca_c)))
+def workspace_size(M: int, N: int, K: int, ca_c: int, k_block_factor: int = 1, out_dtype=None) -> int:
+    """Bytes of workspace a call needs (``sfc_gemm_workspace_size2``)."""
+    import torch
+    dt = SFC_BF16 if out_dtype == torch.bfloat16 else SFC_F32
+    return int(load().sfc_gemm_workspace_size2(int(M), int(N), int(K), int(ca_c), int(k_block_factor), dt))
 
 
 def plan(M: int, N: int, K: int, ca_c: int = 0, out_dtype=None, tile="auto", in_dtype=None,
@@ -177,15 +185,18 @@ def _row_major_2d(t, name):
 
 
 def gemm(A, B, C=None, *, ca_c: int = 1, out_dtype=None, order: str = "sfc", assign: str = "auto",
-         tile=0, workspace=None, stream=None, b_layout: str = "kn", beta: float = 0.0, bias=None):
+         tile=0, workspace=None, stream=None, b_layout: str = "kn", beta: float = 0.0, bias=None,
+         k_block_factor: int = 1):
     """C = A @ B (+ beta * C + bias) on the GPU.  A: (M, K) CUDA tensor, bf16
     or an 8-bit float (float8_e4m3fn, float8_e5m2), row-major (row stride may
     be padded).  B: the same dtype, (K, N) for ``b_layout="kn"`` or its
     transpose (N, K) for ``"nk"`` (a linear layer's weight).  C: (M, N)
     fp32 or bf16 CUDA tensor, allocated if not given (then ``beta`` must be 0).
     ``bias``: optional fp32 CUDA tensor of N values.  ``ca_c``: K layers (0: the
-    library chooses).  ``workspace``: optional CUDA tensor of at least
-    ``workspace_size(M, N, K, ca_c)`` bytes."""
+    library chooses).  ``k_block_factor``: passes over each layer's K range,
+    summed into C (or the layer copies) in place.  ``workspace``: optional CUDA
+    tensor of at least ``workspace_size(M, N, K, ca_c, k_block_factor,
+    out_dtype)`` bytes."""
     import torch
     lib = load()
     M, K = A.shape
@@ -217,11 +228,11 @@ def gemm(A, B, C=None, *, ca_c: int = 1, out_dtype=None, order: str = "sfc", ass
     ws_ptr, ws_bytes = None, 0
     if workspace is not None:
         ws_ptr, ws_bytes = ctypes.c_void_p(workspace.data_ptr()), workspace.numel() * workspace.element_size()
-    rc = lib.sfc_gemm_ex2(M, N, K, ctypes.c_void_p(A.data_ptr()), ctypes.c_void_p(B.data_ptr()),
+    rc = lib.sfc_gemm_ex3(M, N, K, ctypes.c_void_p(A.data_ptr()), ctypes.c_void_p(B.data_ptr()),
                           ctypes.c_void_p(C.data_ptr()), lda, ldb, ldc, ab, B_LAYOUTS[b_layout], float(beta), bias_ptr,
-                          int(ca_c), SFC_F32 if C.dtype == torch.float32 else SFC_BF16, ORDERS[order],
-                          ASSIGNS[assign], TILES[tile], ws_ptr, ws_bytes, _stream_ptr(stream))
-    _check(rc, "sfc_gemm_ex2")
+                          int(ca_c), int(k_block_factor), SFC_F32 if C.dtype == torch.float32 else SFC_BF16,
+                          ORDERS[order], ASSIGNS[assign], TILES[tile], ws_ptr, ws_bytes, _stream_ptr(stream))
+    _check(rc, "sfc_gemm_ex3")
     return C
 
 

@@ -30,6 +30,7 @@ namespace {
 
 constexpr int kMaxDevices = 64;
 constexpr int kMaxLayers = 4096;  // keeps the kernels' layer arithmetic in 32 bits
+constexpr int kMaxKBlocks = 64;   // k_block_factor bound (keeps the kernels' pass arithmetic in 32 bits)
 constexpr uint64_t kDefaultTimeoutNs = 2000000000ull;  // 2 s per wait
 
 std::atomic<uint64_t> g_launch_seq{0};  // picks each launch's scheduler counter slot
@@ -394,6 +395,14 @@ int validate(int64_t M, int64_t N, int64_t K, const void* A, const void* B, cons
 
 int64_t ws_ld(int64_t N) { return (N + 3) / 4 * 4; }
 
+// fp32 workspace of a call: one copy of C per K layer when there is more than
+// one layer, and one copy when K blocks are summed for a bf16 C (an fp32 C
+// sums them in place).
+size_t workspace_bytes_for(int64_t M, int64_t N, int c, int kbf, int c_dtype) {
+    const int copies = (c > 1) ? c : ((kbf > 1 && c_dtype != SFC_F32) ? 1 : 0);
+    return static_cast<size_t>(copies) * static_cast<size_t>(M) * static_cast<size_t>(ws_ld(N)) * 4u;
+}
+
 template <typename OutT>
 cudaError_t launch_gemm(int v, bool f8, const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc,
                         const GemmParams& p, int grid, cudaStream_t s) {
@@ -404,24 +413,91 @@ cudaError_t launch_gemm(int v, bool f8, const CUtensorMap& ta, const CUtensorMap
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
+// Operands whose rows (or base) are not 16-byte aligned are copied into
+// padded pool buffers (packed[0] for A, packed[1] for B), and the pointer and
+// row stride are redirected to the copy.
+int pack_operands(const DeviceInfo* dev, int ab, int b_layout, int64_t M, int64_t N, int64_t K, const void** A,
+                  int64_t* lda, const void** B, int64_t* ldb, void* packed[2], cudaStream_t stream) {
+    const int eb = in_bytes(ab);
+    const int64_t row_align = 16 / eb;
+    const int64_t b_rows = (b_layout == SFC_B_NK) ? N : K, b_cols = (b_layout == SFC_B_NK) ? K : N;
+    for (int which = 0; which < 2; ++which) {
+        const void** ptr = which == 0 ? A : B;
+        int64_t* ld = which == 0 ? lda : ldb;
+        if (aligned16(*ptr) && (*ld % row_align) == 0) continue;
+        const int64_t rows = which == 0 ? M : b_rows, cols = which == 0 ? K : b_cols;
+        const int64_t ld_dst = (cols + row_align - 1) / row_align * row_align;
+        cudaError_t e = cudaMallocFromPoolAsync(&packed[which], static_cast<size_t>(rows * ld_dst * eb), dev->pool,
+                                                stream);
+        if (e != cudaSuccess) return cuda_fail(e);
+        int64_t blocks = ceil_div(rows * cols, 256);
+        if (blocks > static_cast<int64_t>(dev->num_sms) * 16) blocks = static_cast<int64_t>(dev->num_sms) * 16;
+        pack_rows_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(
+            static_cast<const uint8_t*>(*ptr), *ld, rows, cols, eb, static_cast<uint8_t*>(packed[which]), ld_dst);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return cuda_fail(e);
+        *ptr = packed[which];
+        *ld = ld_dst;
+    }
+    return SFC_OK;
+}
+
+void free_packed(void* packed[2], cudaStream_t stream) {
+    for (int i = 0; i < 2; ++i)
+        if (packed[i]) cudaFreeAsync(packed[i], stream);  // stream-ordered: after the kernels that read them
+}
+
+// C = cvt(sum over layers of the fp32 copies in ws [+ beta * C + bias]), Listing 1's final reduction.
+cudaError_t launch_reduce(const DeviceInfo* dev, const float* ws, int64_t ldo, int64_t layer_stride, int layers,
+                          int64_t M, int64_t N, void* C, int64_t ldc, int c_dtype, float beta, const float* bias,
+                          cudaStream_t stream) {
+    const int64_t work = M * ((N + 3) / 4);
+    int64_t blocks = ceil_div(work, 256);
+    const int64_t cap = static_cast<int64_t>(dev->num_sms) * 8;
+    if (blocks > cap) blocks = cap;
+    const int vec = (c_dtype == SFC_F32) ? (aligned16(C) && (ldc % 4) == 0)
+                                         : (((reinterpret_cast<uintptr_t>(C) & 7u) == 0) && (ldc % 4) == 0);
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr.val.programmaticStreamSerializationAllowed = 1;
+    cfg.gridDim = dim3(static_cast<unsigned>(blocks), 1, 1);
+    cfg.blockDim = dim3(256, 1, 1);
+    cfg.stream = stream;
+    cfg.attrs = &attr;
+    cfg.numAttrs = 1;
+    cudaError_t e;
+    if (c_dtype == SFC_F32)
+        e = cudaLaunchKernelEx(&cfg, ca_reduce_kernel<float>, ws, ldo, layer_stride, layers, M, N,
+                               static_cast<float*>(C), ldc, vec, beta, bias);
+    else
+        e = cudaLaunchKernelEx(&cfg, ca_reduce_kernel<__nv_bfloat16>, ws, ldo, layer_stride, layers, M, N,
+                               static_cast<__nv_bfloat16*>(C), ldc, vec, beta, bias);
+    return e == cudaSuccess ? cudaGetLastError() : e;
+}
+
 int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void* C, int64_t lda, int64_t ldb,
              int64_t ldc, int ca_c, int c_dtype, int order, int assign, int tile, void* workspace,
              size_t workspace_bytes, cudaStream_t stream, int debug_never, uint64_t timeout_ns,
              int b_layout = SFC_B_KN, float beta = 0.0f, const float* bias = nullptr, int ab = SFC_AB_BF16,
-             bool allow_pack = true) {
+             bool allow_pack = true, int kbf = 1) {
     int rc = validate(M, N, K, A, B, C, lda, ldb, ldc, ca_c, c_dtype, order, assign, tile, b_layout, ab);
     if (rc != SFC_OK) return rc;
+    // K blocks per layer (Listing 1's k_block_factor): every layer needs at least kbf slabs
+    if (kbf < 1 || kbf > kMaxKBlocks) return SFC_ERR_INVALID_ARG;
+    const int64_t Kt_all = ceil_div(K, slab_k(ab));
+    if (kbf > Kt_all || (ca_c > 0 && Kt_all / ca_c < kbf)) return SFC_ERR_INVALID_ARG;
     const bool f8 = (ab != SFC_AB_BF16);
     const int sk = slab_k(ab), eb = in_bytes(ab);
     // operands whose rows (or base) are not 16-byte aligned are repacked into pool memory
     const int64_t row_align = 16 / eb;
-    const int64_t b_rows = (b_layout == SFC_B_NK) ? N : K, b_cols = (b_layout == SFC_B_NK) ? K : N;
     const bool pack_a = !aligned16(A) || (lda % row_align) != 0;
     const bool pack_b = !aligned16(B) || (ldb % row_align) != 0;
     if ((pack_a || pack_b) && !allow_pack) return SFC_ERR_UNALIGNED;
     if (bias && (reinterpret_cast<uintptr_t>(bias) & 3u) != 0) return SFC_ERR_UNALIGNED;
     const bool b_kmajor = (b_layout == SFC_B_NK);
-    if (ca_c > 0 && workspace && workspace_bytes < sfc_gemm_workspace_size(M, N, K, ca_c)) return SFC_ERR_WORKSPACE;
+    if (ca_c > 0 && workspace && workspace_bytes < workspace_bytes_for(M, N, ca_c, kbf, c_dtype))
+        return SFC_ERR_WORKSPACE;
     if (workspace && !aligned16(workspace)) return SFC_ERR_UNALIGNED;
 
     DeviceInfo* dev = nullptr;
@@ -430,47 +506,22 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
 
     // ca_c = 0: the planner's layer count, within the caller's workspace if one is given
     int max_c = static_cast<int>(auto_layer_cap(M, N, K, ab));
-    while (ca_c == 0 && workspace && max_c > 1 && workspace_bytes < sfc_gemm_workspace_size(M, N, K, max_c)) --max_c;
+    if (max_c > Kt_all / kbf) max_c = static_cast<int>(Kt_all / kbf);
+    while (ca_c == 0 && workspace && max_c > 1 && workspace_bytes < workspace_bytes_for(M, N, max_c, kbf, c_dtype))
+        --max_c;
     const Plan plan = make_plan(M, N, K, ca_c, max_c, *dev, static_cast<sfc_tile_t>(tile), c_dtype == SFC_F32 ? 4 : 2,
                                 b_kmajor, ab);
     const int v = plan.v;
     ca_c = plan.c;
-    const size_t ws_need = sfc_gemm_workspace_size(M, N, K, ca_c);
+    const size_t ws_need = workspace_bytes_for(M, N, ca_c, kbf, c_dtype);
     const int bn = variant_bn(v);
     const int bm = variant_bm(v);
     void* packed[2] = {nullptr, nullptr};
-    auto release_packed = [&]() {
-        for (void* ptr : packed)
-            if (ptr) cudaFreeAsync(ptr, stream);
-    };
-    for (int which = 0; which < 2; ++which) {
-        if (!(which == 0 ? pack_a : pack_b)) continue;
-        const int64_t rows = which == 0 ? M : b_rows, cols = which == 0 ? K : b_cols;
-        const int64_t ld_src = which == 0 ? lda : ldb;
-        const int64_t ld_dst = (cols + row_align - 1) / row_align * row_align;
-        cudaError_t e = cudaMallocFromPoolAsync(&packed[which], static_cast<size_t>(rows * ld_dst * eb), dev->pool,
-                                                stream);
-        if (e != cudaSuccess) {
-            release_packed();
-            return cuda_fail(e);
-        }
-        int64_t blocks = ceil_div(rows * cols, 256);
-        if (blocks > static_cast<int64_t>(dev->num_sms) * 16) blocks = static_cast<int64_t>(dev->num_sms) * 16;
-        pack_rows_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(
-            static_cast<const uint8_t*>(which == 0 ? A : B), ld_src, rows, cols, eb,
-            static_cast<uint8_t*>(packed[which]), ld_dst);
-        e = cudaGetLastError();
-        if (e != cudaSuccess) {
-            release_packed();
-            return cuda_fail(e);
-        }
-        if (which == 0) {
-            A = packed[0];
-            lda = ld_dst;
-        } else {
-            B = packed[1];
-            ldb = ld_dst;
-        }
+    auto release_packed = [&]() { free_packed(packed, stream); };
+    rc = pack_operands(dev, ab, b_layout, M, N, K, &A, &lda, &B, &ldb, packed, stream);
+    if (rc != SFC_OK) {
+        release_packed();
+        return rc;
     }
     CUtensorMap ta, tb;
     rc = make_in_map(&ta, A, M, K, lda, eb, kBM, sk);  // each CTA loads 128 rows of A, one slab of k
@@ -513,15 +564,19 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     p.beta = beta;
     p.c_in = C;
     p.ldc_in = ldc;
+    p.c_in_layer_stride = 0;
     p.bias = bias;
     p.ab_fmt = (ab == SFC_AB_E4M3) ? 0 : 1;  // bf16 (kind::f16) and e5m2 (kind::f8f6f4) are both code 1
+    p.kbf = 1;
+    p.pass = 0;
+    p.accumulate = 0;
     const int64_t workers = dev->one_item_per_worker ? p.num_items : dev->workers[v];
     const int64_t used = p.num_items < workers ? p.num_items : workers;
     const int grid = static_cast<int>(variant_cluster(v) * used);
 
     void* ws = workspace;
     bool pooled = false;
-    if (ca_c > 1 && !ws) {
+    if (ws_need > 0 && !ws) {
         cudaError_t e = cudaMallocFromPoolAsync(&ws, ws_need, dev->pool, stream);
         if (e != cudaSuccess) {
             release_packed();
@@ -530,50 +585,56 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
         pooled = true;
     }
 
-    cudaError_t e;
+    cudaError_t e = cudaSuccess;
     CUtensorMap tc;
     std::memset(&tc, 0, sizeof(tc));
-    if (ca_c == 1) {
+    if (ws_need == 0) {
+        // one pass straight into C, or K blocks added into an fp32 C in place
         p.out = C;
         p.ldo = ldc;
         p.layer_stride = 0;
         const int esz = (c_dtype == SFC_F32) ? 4 : 2;
         p.vec_store = aligned16(C) && ((ldc * esz) % 16 == 0);
         p.tma_store = p.vec_store && make_out_map(&tc, C, M, N, ldc, esz, 1) == SFC_OK;
-        e = (c_dtype == SFC_F32) ? launch_gemm<float>(v, f8, ta, tb, tc, p, grid, stream)
-                                 : launch_gemm<__nv_bfloat16>(v, f8, ta, tb, tc, p, grid, stream);
+        for (int pass = 0; pass < kbf && e == cudaSuccess; ++pass) {
+            if (pass > 0) {
+                // C holds the earlier K blocks' sum (and beta C + bias): the stores add into it
+                // (TMA reduction in L2), or, for rows the TMA cannot store, the epilogue reads it
+                p.accumulate = p.tma_store;
+                p.beta = p.tma_store ? 0.0f : 1.0f;
+                p.bias = nullptr;
+                p.sched_slot = static_cast<int>(g_launch_seq.fetch_add(1, std::memory_order_relaxed) % kSchedSlots);
+            }
+            p.kbf = kbf;
+            p.pass = pass;
+            e = (c_dtype == SFC_F32) ? launch_gemm<float>(v, f8, ta, tb, tc, p, grid, stream)
+                                     : launch_gemm<__nv_bfloat16>(v, f8, ta, tb, tc, p, grid, stream);
+        }
     } else {
+        // fp32 copies of C, one per K layer (K blocks added in place), then the reduction
         p.out = ws;
         p.ldo = ws_ld(N);
         p.layer_stride = M * p.ldo;
         p.vec_store = 1;
         p.tma_store = make_out_map(&tc, ws, M, N, p.ldo, 4, ca_c) == SFC_OK;
-        e = launch_gemm<float>(v, f8, ta, tb, tc, p, grid, stream);
-        if (e == cudaSuccess) {
-            const int64_t work = M * ((N + 3) / 4);
-            int64_t blocks = ceil_div(work, 256);
-            const int64_t cap = static_cast<int64_t>(dev->num_sms) * 8;
-            if (blocks > cap) blocks = cap;
-            const int vec = (c_dtype == SFC_F32) ? (aligned16(C) && (ldc % 4) == 0)
-                                                 : (((reinterpret_cast<uintptr_t>(C) & 7u) == 0) && (ldc % 4) == 0);
-            cudaLaunchConfig_t cfg = {};
-            cudaLaunchAttribute attr;
-            attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
-            attr.val.programmaticStreamSerializationAllowed = 1;
-            cfg.gridDim = dim3(static_cast<unsigned>(blocks), 1, 1);
-            cfg.blockDim = dim3(256, 1, 1);
-            cfg.stream = stream;
-            cfg.attrs = &attr;
-            cfg.numAttrs = 1;
-            const float* wsf = static_cast<const float*>(ws);
-            if (c_dtype == SFC_F32)
-                e = cudaLaunchKernelEx(&cfg, ca_reduce_kernel<float>, wsf, p.ldo, p.layer_stride, ca_c, M, N,
-                                       static_cast<float*>(C), ldc, vec, beta, bias);
-            else
-                e = cudaLaunchKernelEx(&cfg, ca_reduce_kernel<__nv_bfloat16>, wsf, p.ldo, p.layer_stride, ca_c, M,
-                                       N, static_cast<__nv_bfloat16*>(C), ldc, vec, beta, bias);
-            if (e == cudaSuccess) e = cudaGetLastError();
+        p.beta = 0.0f;
+        p.bias = nullptr;
+        for (int pass = 0; pass < kbf && e == cudaSuccess; ++pass) {
+            if (pass > 0) {
+                p.accumulate = p.tma_store;
+                p.beta = p.tma_store ? 0.0f : 1.0f;
+                p.c_in = ws;
+                p.ldc_in = p.ldo;
+                p.c_in_layer_stride = p.layer_stride;
+                p.sched_slot = static_cast<int>(g_launch_seq.fetch_add(1, std::memory_order_relaxed) % kSchedSlots);
+            }
+            p.kbf = kbf;
+            p.pass = pass;
+            e = launch_gemm<float>(v, f8, ta, tb, tc, p, grid, stream);
         }
+        if (e == cudaSuccess)
+            e = launch_reduce(dev, static_cast<const float*>(ws), p.ldo, p.layer_stride, ca_c, M, N, C, ldc, c_dtype,
+                              beta, bias, stream);
     }
     if (pooled) {
         cudaError_t f = cudaFreeAsync(ws, stream);
@@ -678,6 +739,29 @@ SFC_API int sfc_gemm_ex2(int64_t M, int64_t N, int64_t K, const void* A, const v
     return run_gemm(M, N, K, A, B, C, lda, ldb, ldc, ca_c, c_dtype, order, assign, tile, workspace,
                     workspace_bytes, static_cast<cudaStream_t>(stream), 0, kDefaultTimeoutNs, b_layout, beta, bias,
                     ab_dtype);
+}
+
+SFC_API int sfc_gemm_ex3(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void* C, int64_t lda,
+                         int64_t ldb, int64_t ldc, int ab_dtype, int b_layout, float beta, const float* bias,
+                         int ca_c, int k_block_factor, sfc_dtype_t c_dtype, sfc_order_t order, sfc_assign_t assign,
+                         sfc_tile_t tile, void* workspace, size_t workspace_bytes, void* stream) {
+    return run_gemm(M, N, K, A, B, C, lda, ldb, ldc, ca_c, c_dtype, order, assign, tile, workspace,
+                    workspace_bytes, static_cast<cudaStream_t>(stream), 0, kDefaultTimeoutNs, b_layout, beta, bias,
+                    ab_dtype, true, k_block_factor);
+}
+
+SFC_API size_t sfc_gemm_workspace_size2(int64_t M, int64_t N, int64_t K, int ca_c, int k_block_factor,
+                                        sfc_dtype_t c_dtype) {
+    if (M <= 0 || N <= 0 || K <= 0 || ca_c < 0 || k_block_factor < 1 || k_block_factor > kMaxKBlocks) return 0;
+    if (c_dtype != SFC_F32 && c_dtype != SFC_BF16) return 0;
+    int64_t layers = ca_c;
+    if (layers == 0) {  // the most the planner may choose
+        layers = auto_layer_cap(M, N, K);
+        const int64_t per = ceil_div(K, kBK) / k_block_factor;
+        if (layers > per) layers = per;
+        if (layers < 1) layers = 1;
+    }
+    return workspace_bytes_for(M, N, static_cast<int>(layers), k_block_factor, c_dtype);
 }
 
 SFC_API int sfc_get_device_status(void* stream) {

@@ -115,8 +115,11 @@ struct GemmParams {
     float beta;            // C = A B + beta C_in + bias (ca_c == 1: applied by the epilogue)
     const void* c_in;      // C_in (the output array, read before it is written) when beta != 0
     int64_t ldc_in;        // its row stride in elements
+    int64_t c_in_layer_stride;  // != 0: C_in is `out` itself, K-layer copy by copy (beta applied per layer)
     const float* bias;     // N fp32 values or null
     int ab_fmt;            // A/B format code of the instruction descriptor (bf16: 1; e4m3: 0, e5m2: 1)
+    int kbf, pass;         // k_block_factor > 1: this launch contracts K block `pass` of every layer
+    int accumulate;        // 1: the TMA stores add into `out` (fp32, in L2) instead of overwriting it
 };
 
 struct WorkItem {
@@ -131,6 +134,20 @@ __device__ __forceinline__ int slab_at(const WorkItem& w, int q) { return w.rev 
 // in 32-bit arithmetic (c <= 4096 keeps l * (Kt % c) below 2^24).
 __device__ __forceinline__ int layer_k0(int l, const GemmParams& p) { return l * p.kq + (l * p.kr) / p.ca_c; }
 
+// With k_block_factor > 1 (the outer K-block loop of Listing 1) a launch
+// contracts block `pass` of each layer's slabs: [k0 + floor(pass * len / kbf),
+// k0 + floor((pass + 1) * len / kbf)).  kbf <= 64 and len < 2^25 keep the
+// products in 32 bits.
+__device__ __forceinline__ void narrow_to_pass(WorkItem& w, const GemmParams& p) {
+    if (p.kbf > 1) {
+        const unsigned len = static_cast<unsigned>(w.k1 - w.k0), kbf = static_cast<unsigned>(p.kbf);
+        const unsigned pass = static_cast<unsigned>(p.pass);
+        const int base = w.k0;
+        w.k0 = base + static_cast<int>(pass * len / kbf);
+        w.k1 = base + static_cast<int>((pass + 1u) * len / kbf);
+    }
+}
+
 // Item index i < 2^31 (validated on the host) -> tile, K layer and K range.
 __device__ __forceinline__ WorkItem decode_item(int64_t i64, const GemmParams& p) {
     const int i = static_cast<int>(i64);
@@ -144,6 +161,7 @@ __device__ __forceinline__ WorkItem decode_item(int64_t i64, const GemmParams& p
     w.k0 = layer_k0(layer, p);
     w.k1 = layer_k0(layer + 1, p);
     w.rev = 0;
+    narrow_to_pass(w, p);
     return w;
 }
 
@@ -261,12 +279,13 @@ __device__ __forceinline__ void store_chunk(OutT* row_ptr, int64_t col0, int64_t
     }
 }
 
-// beta * C_in + bias for columns [col0, col0 + n) of one row, added into v
-// (fp32, before rounding to the output type).  Columns >= N are left alone.
+// beta * C_in + bias for columns [col0, col0 + n) of one row of K layer
+// `layer`, added into v (fp32, before rounding to the output type).  Columns
+// >= N are left alone.
 template <typename OutT, int n>
-__device__ __forceinline__ void apply_affine(const GemmParams& p, int64_t row, int64_t col0, float* v) {
+__device__ __forceinline__ void apply_affine(const GemmParams& p, int64_t row, int64_t col0, int layer, float* v) {
     if (p.beta != 0.0f && row < p.M) {
-        const OutT* src = static_cast<const OutT*>(p.c_in) + row * p.ldc_in + col0;
+        const OutT* src = static_cast<const OutT*>(p.c_in) + layer * p.c_in_layer_stride + row * p.ldc_in + col0;
 #pragma unroll
         for (int j = 0; j < n; ++j)
             if (col0 + j < p.N) v[j] = __fmaf_rn(p.beta, static_cast<float>(src[j]), v[j]);
@@ -337,6 +356,7 @@ __device__ __forceinline__ int64_t src_take(const ItemSource& S, int j, const Ge
     w.k0 = (p.ca_c == 1) ? 0 : layer_k0(w.layer, p);
     w.k1 = (p.ca_c == 1) ? p.Kt : layer_k0(w.layer + 1, p);
     w.rev = p.serpentine ? (j & 1) : 0;
+    narrow_to_pass(w, p);
     return item;
 }
 
@@ -497,8 +517,9 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
     const uint32_t acce_target = PAIR ? ptx::map_to_cta(B.acc_empty(0), pair_leader) : B.acc_empty(0);
     float run[kEpiCols];
     int nbox = 0;  // boxes this warp has stored (selects the staging half)
-    // beta C_in + bias in this epilogue only without K layers (else the reduction applies it)
-    const bool affine = p.ca_c == 1 && (p.beta != 0.0f || p.bias != nullptr);
+    // beta C_in + bias in this epilogue only without K layers (else the reduction applies
+    // it), or when a later K block adds into the layer copies (k_block_factor > 1)
+    const bool affine = (p.ca_c == 1 || p.c_in_layer_stride != 0) && (p.beta != 0.0f || p.bias != nullptr);
     for (int j = 0;; ++j) {
         // lane 0 takes the item, the warp follows (tcgen05.ld needs the whole warp)
         int64_t it = 0;
@@ -557,7 +578,8 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
             for (int g = 0; g < kEpiCols / kCols; ++g) {
                 if (col_base + g * kCols >= p.N) break;  // warp-uniform
                 uint8_t* box = staging + ew * kStageBufBytes + (nbox & 1) * kBoxBytes;
-                if (affine) apply_affine<OutT, kCols>(p, warp_row + lane, col_base + g * kCols, run + g * kCols);
+                if (affine)
+                    apply_affine<OutT, kCols>(p, warp_row + lane, col_base + g * kCols, w.layer, run + g * kCols);
                 if (lane == 0) ptx::bulk_wait_read_1();  // the store that last used this box has read it
                 __syncwarp();
                 stage_row<OutT>(box, lane, run + g * kCols);
@@ -565,12 +587,14 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
                 __syncwarp();
                 if (lane == 0) {
                     const uint32_t box_addr = ptx::smem_addr(box);
-                    if (p.ca_c > 1)
-                        ptx::tma_store_3d(tmap_c, box_addr, static_cast<int32_t>(col_base + g * kCols),
-                                          static_cast<int32_t>(warp_row), w.layer);
-                    else
-                        ptx::tma_store_2d(tmap_c, box_addr, static_cast<int32_t>(col_base + g * kCols),
-                                          static_cast<int32_t>(warp_row));
+                    const int32_t x = static_cast<int32_t>(col_base + g * kCols), y = static_cast<int32_t>(warp_row);
+                    if (p.ca_c > 1) {
+                        if (p.accumulate) ptx::tma_reduce_add_3d(tmap_c, box_addr, x, y, w.layer);
+                        else ptx::tma_store_3d(tmap_c, box_addr, x, y, w.layer);
+                    } else {
+                        if (p.accumulate) ptx::tma_reduce_add_2d(tmap_c, box_addr, x, y);
+                        else ptx::tma_store_2d(tmap_c, box_addr, x, y);
+                    }
                     ptx::bulk_commit();
                 }
                 ++nbox;
@@ -581,7 +605,7 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
                 OutT* row_ptr = out + static_cast<int64_t>(w.layer) * p.layer_stride + row * p.ldo;
 #pragma unroll
                 for (int g = 0; g < kEpiCols / 32; ++g) {
-                    if (affine) apply_affine<OutT, 32>(p, row, col_base + g * 32, run + g * 32);
+                    if (affine) apply_affine<OutT, 32>(p, row, col_base + g * 32, w.layer, run + g * 32);
                     store_chunk<OutT>(row_ptr, col_base + g * 32, p.N, run + g * 32, p.vec_store != 0);
                 }
             }

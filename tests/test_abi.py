@@ -200,3 +200,33 @@ def test_gemm_host_validation_codes(lib):
     assert call_host(lib, panels=-1) == E.SFC_ERR_INVALID_ARG
     assert call_host(lib, a=0x10001) == E.SFC_ERR_UNALIGNED                   # bf16 at an odd address
     assert call_host(lib, c=0x30002) == E.SFC_ERR_UNALIGNED                   # fp32 C at a 2-byte offset
+
+
+def test_workspace_size_with_k_blocks(lib):
+    import torch
+    ws = sfc.workspace_size
+    assert ws(512, 512, 4096, 1, k_block_factor=4) == 0                                  # fp32 C: in place
+    assert ws(512, 512, 4096, 1, k_block_factor=4, out_dtype=torch.bfloat16) == 512 * 512 * 4   # one fp32 copy
+    assert ws(512, 512, 4096, 1, k_block_factor=1, out_dtype=torch.bfloat16) == 0
+    assert ws(512, 512, 4096, 3, k_block_factor=2) == 3 * 512 * 512 * 4
+    # ca_c = 0: the planner's bound, at most ceil(K/64) / k_block_factor layers
+    assert ws(512, 512, 32768, 0, k_block_factor=1) == 20 * 512 * 512 * 4
+    assert ws(512, 512, 1024, 0, k_block_factor=4) == 4 * 512 * 512 * 4                 # 16 slabs / 4
+    assert ws(512, 512, 4096, 1, k_block_factor=0) == 0                                  # invalid
+    assert ws(512, 512, 4096, 1, k_block_factor=65) == 0
+
+
+def call_ex3(lib, M=256, N=256, K=1024, ca_c=1, kbf=2, ab=0):
+    return lib.sfc_gemm_ex3(M, N, K, ctypes.c_void_p(PA), ctypes.c_void_p(PB), ctypes.c_void_p(PC), K, N, N, ab, 0,
+                            0.0, None, ca_c, kbf, 0, 0, 2, 0, None, 0, None)
+
+
+def test_gemm_ex3_validation_codes(lib):
+    # every case is rejected on the host, before the device is touched
+    E = binding
+    assert call_ex3(lib, kbf=0) == E.SFC_ERR_INVALID_ARG
+    assert call_ex3(lib, kbf=65) == E.SFC_ERR_INVALID_ARG
+    assert call_ex3(lib, K=256, kbf=5) == E.SFC_ERR_INVALID_ARG                # 4 slabs of 64
+    assert call_ex3(lib, K=1024, ca_c=4, kbf=5) == E.SFC_ERR_INVALID_ARG       # 16 slabs: 4 per layer < 5
+    assert call_ex3(lib, K=1024, ab=1, ca_c=2, kbf=5) == E.SFC_ERR_INVALID_ARG  # 8 slabs of 128: 4 per layer
+    assert call_ex3(lib, M=0) == E.SFC_ERR_INVALID_ARG

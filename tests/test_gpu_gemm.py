@@ -98,12 +98,14 @@ def test_integer_inputs_bit_exact_every_variant(sfc, oracle):
     assert sfc.device_status() == 0
 
 
-def test_order_and_assignment_do_not_change_bits(sfc):
-    # The per-tile K order is fixed, so curve vs raster and segment vs wave
-    # must give bit-identical results for a fixed number of K layers.
+def test_order_assignment_and_tile_do_not_change_bits(sfc):
+    # The per-tile K order and its accumulation chains are fixed, so curve vs
+    # raster, segment vs wave and every tile shape must give bit-identical
+    # results for a fixed number of K layers.
     A, B = synth.gemm_inputs(1000, 1200, 2500, "uniform", seed=5, lda=synth.pad8(2500))
     Ad, Bd = to_dev(A, B)
     for c in (1, 3):
+        first = None
         for tile in TILES:
             outs = [sfc.gemm(Ad, Bd, ca_c=c, order=o, assign=a, tile=tile)
                     for o in ("sfc", "raster") for a in ("segment", "wave")]
@@ -111,6 +113,8 @@ def test_order_and_assignment_do_not_change_bits(sfc):
                 assert torch.equal(outs[0], other)
             again = sfc.gemm(Ad, Bd, ca_c=c, order="sfc", assign="segment", tile=tile)
             assert torch.equal(outs[0], again)                 # repeatable
+            first = outs[0] if first is None else first
+            assert torch.equal(first, outs[0]), tile           # the tile shape does not matter either
 
 
 def test_k_layers_agree_within_tolerance(sfc, oracle):
