@@ -596,6 +596,11 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
         const int esz = (c_dtype == SFC_F32) ? 4 : 2;
         p.vec_store = aligned16(C) && ((ldc * esz) % 16 == 0);
         p.tma_store = p.vec_store && make_out_map(&tc, C, M, N, ldc, esz, 1) == SFC_OK;
+        if (beta == 1.0f && !bias && c_dtype == SFC_F32 && p.tma_store) {
+            // C += A B: the stores add into C in L2 (the same rounding as reading C and adding)
+            p.accumulate = 1;
+            p.beta = 0.0f;
+        }
         for (int pass = 0; pass < kbf && e == cudaSuccess; ++pass) {
             if (pass > 0) {
                 // C holds the earlier K blocks' sum (and beta C + bias): the stores add into it

@@ -118,3 +118,29 @@ def test_beta_zero_never_reads_c(sfc, oracle):
         sfc.gemm(A.cuda(), B.cuda(), C, beta=0.0, ca_c=c)
         torch.cuda.synchronize()
         assert np.array_equal(C.cpu().numpy().astype(np.float64), ref)
+
+
+@pytest.mark.parametrize("tile", ["auto", 128, "pair256", "quad256"])
+def test_accumulate_into_c(sfc, oracle, tile):
+    # C += A B (beta = 1, no bias, fp32 C with 16-byte rows) adds in L2 instead of
+    # reading C; it must equal the path that reads C (rows the TMA cannot store)
+    # bit for bit, and the oracle exactly on integer data.
+    M, N, K = 520, 392, 2000
+    A, B = synth.gemm_inputs(M, N, K, "uniform", seed=81)
+    C_in = synth.uniform_bf16((M, N), seed=82).float()
+    Ad, Bd = padded(A, 2000), padded(B, 392)
+    C = C_in.cuda()
+    sfc.gemm(Ad, Bd, C, beta=1.0, tile=tile)
+    big = torch.zeros(M, N + 1, dtype=torch.float32, device="cuda")
+    Cr = big[:, :N]
+    Cr.copy_(C_in)
+    sfc.gemm(Ad, Bd, Cr, beta=1.0, tile=tile)                   # ldc = N + 1: read, add, store
+    assert torch.equal(C, Cr)
+    check_fp32(C.cpu().numpy().astype(np.float64),
+               oracle.gemm_affine_f64(A, B, beta=1.0, C_in=C_in.numpy()), K)
+    Ai, Bi = synth.gemm_inputs(M, N, K, "int", seed=83)
+    Ci = torch.randint(-8, 9, (M, N), dtype=torch.float32)
+    ref = oracle.gemm_affine_f64(Ai, Bi, beta=1.0, C_in=Ci.numpy())
+    C = Ci.cuda()
+    sfc.gemm(padded(Ai, 2000), padded(Bi, 392), C, beta=1.0, tile=tile)
+    assert np.array_equal(C.cpu().numpy().astype(np.float64), ref)
