@@ -44,9 +44,9 @@ constexpr int64_t kMaxPanels = 64;
 constexpr int64_t kPanelRowsM = 512;    // rows of the largest output tile (two stacked 2-SM pairs)
 constexpr int64_t kPanelColsN = 256;    // columns of the widest output tile
 constexpr int64_t kAutoPanelSpan = 2048;  // automatic panels: about this many rows or columns each
-constexpr int64_t kAutoMaxPanels = 8;
+constexpr int64_t kAutoMaxPanels = 8;  // panels of the automatic span before the span grows
 // Pitched host<->device copies run below the link's rate for short rows
-// (measured on GB300: 4 KB rows 175 GB/s, 8 KB 188, 16 KB and up 211).
+// (measured on GB300: 2 KB rows 128 GB/s, 4 KB 175, 8 KB 188, 16 KB and up 211).
 constexpr int64_t kMinPitchedRowBytes = 8192;
 
 int fail(cudaError_t e) { return sfc::cuda_fail(e); }
@@ -150,19 +150,53 @@ struct Region {
     int64_t r0, r1, c0, c1;
 };
 
-// Span of a panel along a dimension of `extent` elements (`units` multiples of
-// `unit`): `panels` panels if given, else about one per `auto_span` elements,
-// at most kAutoMaxPanels; always a whole number of units.
-int64_t panel_span(int64_t extent, int64_t units, int64_t unit, int panels, int64_t auto_span) {
-    int64_t np = panels;
-    if (np == 0) {
-        np = (extent + auto_span - 1) / auto_span;
-        if (np > kAutoMaxPanels) np = kAutoMaxPanels;
+// Panel edges [0, e_1, ..., extent] along a dimension, every inner edge a
+// multiple of `unit`.  `panels` > 0: that many equal panels (at most
+// kMaxPanels, at most one per unit).  0: panels of about `auto_span` elements
+// (more when that would make over kAutoMaxPanels of them); with `ramp`, the
+// first two and the last two are a quarter and a half of that, so that the
+// first GEMM starts after little data has arrived and the last leaves little
+// to do after the final upload (not for pitched copies, whose short rows
+// would slow the link down).
+std::vector<int64_t> panel_edges(int64_t extent, int64_t unit, int panels, int64_t auto_span, bool ramp_ok) {
+    const int64_t units = (extent + unit - 1) / unit;
+    std::vector<int64_t> sizes;  // in units
+    if (panels > 0) {
+        int64_t np = panels;
+        if (np > kMaxPanels) np = kMaxPanels;
+        if (np > units) np = units;
+        const int64_t per = (units + np - 1) / np;
+        for (int64_t done = 0; done < units; done += per) sizes.push_back(per < units - done ? per : units - done);
+    } else {
+        int64_t mid = auto_span / unit;
+        if (mid < 1) mid = 1;
+        const int64_t spread = (units + kAutoMaxPanels - 1) / kAutoMaxPanels;
+        if (mid < spread) mid = spread;
+        const int64_t q = mid / 4 > 0 ? mid / 4 : 1, h = mid / 2 > 0 ? mid / 2 : 1;
+        int64_t rest = units;
+        const bool ramp = ramp_ok && units > 2 * (q + h) + 2 * mid;
+        if (ramp) {
+            sizes.push_back(q);
+            sizes.push_back(h);
+            rest -= 2 * (q + h);
+        }
+        while (rest > 0) {
+            const int64_t sz = mid < rest ? mid : rest;
+            sizes.push_back(sz);
+            rest -= sz;
+        }
+        if (ramp) {
+            sizes.push_back(h);
+            sizes.push_back(q);
+        }
     }
-    if (np > kMaxPanels) np = kMaxPanels;
-    if (np > units) np = units;
-    if (np < 1) np = 1;
-    return (units + np - 1) / np * unit;
+    std::vector<int64_t> edges{0};
+    int64_t at = 0;
+    for (int64_t sz : sizes) {
+        at += sz;
+        edges.push_back(at * unit < extent ? at * unit : extent);
+    }
+    return edges;
 }
 
 // Row-major copy of `rows` rows of `width` bytes between pitched buffers.
@@ -239,15 +273,19 @@ SFC_API int sfc_gemm_host(int64_t M, int64_t N, int64_t K, const void* A, const 
     const size_t c_bytes = static_cast<size_t>(round_up(M * ldc_d * ob, 256));
 
     // row panels of A (multiples of 512 rows) and column panels of B (multiples of 256 columns)
-    const int64_t m_units = (M + kPanelRowsM - 1) / kPanelRowsM, n_units = (N + kPanelColsN - 1) / kPanelColsN;
     // a column panel of an N-major B is a pitched copy: keep its rows at least 8 KB long
     const int64_t col_span = b_nk ? kAutoPanelSpan : (kMinPitchedRowBytes / eb > kAutoPanelSpan
                                                          ? kMinPitchedRowBytes / eb : kAutoPanelSpan);
-    const int64_t per_m = panel_span(M, m_units, kPanelRowsM, panels, kAutoPanelSpan);
-    const int64_t per_n = panel_span(N, n_units, kPanelColsN, panels, col_span);
-    const int64_t pm = (M + per_m - 1) / per_m, pn = (N + per_n - 1) / per_n;
-    auto row_end = [&](int64_t i) { return i * per_m < M ? i * per_m : M; };
-    auto col_end = [&](int64_t j) { return j * per_n < N ? j * per_n : N; };
+    // row panels of A (and of a K-major B) copy rows of K values: ramp them when those rows are
+    // contiguous or long
+    const bool k_rows_fast = K * eb >= kMinPitchedRowBytes;
+    const std::vector<int64_t> em =
+        panel_edges(M, kPanelRowsM, panels, kAutoPanelSpan, k_rows_fast || (lda == K && lda_d == K));
+    const std::vector<int64_t> en =
+        panel_edges(N, kPanelColsN, panels, col_span, b_nk && (k_rows_fast || (ldb == K && ldb_d == K)));
+    const int64_t pm = static_cast<int64_t>(em.size()) - 1, pn = static_cast<int64_t>(en.size()) - 1;
+    auto row_end = [&](int64_t i) { return em[static_cast<size_t>(i)]; };
+    auto col_end = [&](int64_t j) { return en[static_cast<size_t>(j)]; };
 
     std::lock_guard<std::mutex> lock(p.mu);
     rc = pipe_setup(p);
