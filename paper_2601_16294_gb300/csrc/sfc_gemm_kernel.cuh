@@ -546,14 +546,26 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
             ptx::tc_fence_after();
             const uint32_t taddr = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) +
                                    static_cast<uint32_t>(acc * BN + half * kEpiCols);
+            if (ck == 0) {
+                // the chain's first chunk becomes the running sum as loaded
 #pragma unroll
-            for (int g = 0; g < kEpiCols / 32; ++g) {
-                uint32_t r[32];
-                ptx::tmem_ld_32x32b_x32(taddr + g * 32, r);
-                ptx::tmem_ld_wait();
+                for (int g = 0; g < kEpiCols / 32; ++g) {
+                    uint32_t r[32];
+                    ptx::tmem_ld_32x32b_x32(taddr + g * 32, r);
+                    ptx::tmem_ld_wait();
 #pragma unroll
-                for (int j = 0; j < 32; ++j)
-                    run[g * 32 + j] = (ck == 0) ? __uint_as_float(r[j]) : __fadd_rn(run[g * 32 + j], __uint_as_float(r[j]));
+                    for (int j = 0; j < 32; ++j) run[g * 32 + j] = __uint_as_float(r[j]);
+                }
+            } else {
+                // later chunks are added in 16-column pieces (fewer registers live beside run[])
+#pragma unroll
+                for (int g = 0; g < kEpiCols / 16; ++g) {
+                    uint32_t r[16];
+                    ptx::tmem_ld_32x32b_x16(taddr + g * 16, r);
+                    ptx::tmem_ld_wait();
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) run[g * 16 + j] = __fadd_rn(run[g * 16 + j], __uint_as_float(r[j]));
+                }
             }
             ptx::tc_fence_before();
             __syncwarp();
