@@ -106,6 +106,11 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--out", choices=("workload", "f32", "bf16"), default="workload",
                     help="output type of every shape (default: the workload's own)")
+    ap.add_argument("--sustained", action="store_true",
+                    help="instead of the step timing: run each configuration back to back for --phase-seconds under "
+                         "the power cap (ours by order / dealing / tile / K blocks, then cuBLAS) at each --sizes "
+                         "(default 16384,8192), sampling SM clock and power, and print one JSON line of phases")
+    ap.add_argument("--phase-seconds", type=float, default=2.5)
     ap.add_argument("--k-block-factor", type=int, default=1,
                     help="passes over each layer's K range (Listing 1's k_block_factor); 1 = one pass")
     ap.add_argument("--e2e-order", choices=("given", "largest_first"), default="largest_first",
@@ -714,8 +719,71 @@ def run_reference(args, rank, world):
             "gpu_launches": 0}
 
 
+def run_sustained(args):
+    """Sustained, power-capped phases: each configuration runs back to back for
+    --phase-seconds while nvidia-smi samples the SM clock and board power every
+    50 ms; medians over the second half of each phase (steady state)."""
+    import torch
+    import paper_2601_16294_gb300 as sfc
+
+    torch.cuda.set_device(0)
+    sfc.load()
+    sizes = [int(x) for x in (args.sizes or "16384,8192").split(",")]
+    phases = []
+
+    def phase(name, n, fn):
+        for _ in range(2):
+            fn()
+        torch.cuda.synchronize()
+        smi = subprocess.Popen(["nvidia-smi", "--query-gpu=clocks.sm,power.draw", "--format=csv,noheader,nounits",
+                                "-lms", "50"], stdout=subprocess.PIPE, text=True)
+        time.sleep(0.3)
+        calls = 0
+        t0 = time.time()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        while time.time() - t0 < args.phase_seconds:
+            for _ in range(5):
+                fn()
+            calls += 5
+            torch.cuda.synchronize()
+        e1.record()
+        torch.cuda.synchronize()
+        smi.terminate()
+        out = smi.communicate()[0]
+        rows = [line.split(",") for line in out.strip().splitlines() if line.strip()]
+        half = rows[len(rows) // 2:] or rows
+        clk = statistics.median(float(r[0]) for r in half) if half else None
+        pw = statistics.median(float(r[1]) for r in half) if half else None
+        tf = 2.0 * n ** 3 * calls / (e0.elapsed_time(e1) * 1e-3) / 1e12
+        phases.append({"phase": name, "size": n, "tflops": round(tf, 1), "sm_mhz": clk, "power_w": pw,
+                       "tflops_per_ghz": round(tf / clk * 1e3, 1) if clk else None, "calls": calls})
+        print(json.dumps(phases[-1]), file=sys.stderr, flush=True)
+
+    for n in sizes:
+        A = torch.empty(n, n, dtype=torch.bfloat16, device="cuda").uniform_(-1, 1)
+        B = torch.empty(n, n, dtype=torch.bfloat16, device="cuda").uniform_(-1, 1)
+        C = torch.empty(n, n, dtype=torch.bfloat16, device="cuda")
+        ours = [("curve, dynamic dealing", dict(tile="pair256", assign="wave")),
+                ("curve, static waves", dict(tile="pair256", assign="wave_static")),
+                ("raster, dynamic dealing", dict(tile="pair256", assign="wave", order="raster")),
+                ("curve, dynamic, quad256 (B multicast)", dict(tile="quad256", assign="wave")),
+                ("curve, dynamic, k_block_factor 2", dict(tile="pair256", assign="wave", k_block_factor=2))]
+        for name, kw in ours:
+            phase("ours " + name, n, lambda kw=kw: sfc.gemm(A, B, C, **kw))
+        phase("cuBLAS (torch.matmul)", n, lambda: torch.matmul(A, B, out=C))
+        phase("ours curve, dynamic dealing (again)", n, lambda: sfc.gemm(A, B, C, tile="pair256", assign="wave"))
+        del A, B, C
+        torch.cuda.empty_cache()
+    return {"mode": "sustained", "phase_seconds": args.phase_seconds, "out": "bf16", "inputs": "U[-1,1] bf16",
+            "phases": phases}
+
+
 def main():
     args = parse_args()
+    if args.sustained:
+        print(json.dumps(run_sustained(args)), flush=True)
+        return
     if args.impl == "reference":
         rank = int(os.environ.get("RANK", "0"))
         world = int(os.environ.get("WORLD_SIZE", "1"))
