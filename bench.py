@@ -106,6 +106,9 @@ def parse_args():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--out", choices=("workload", "f32", "bf16"), default="workload",
                     help="output type of every shape (default: the workload's own)")
+    ap.add_argument("--no-tune", action="store_true",
+                    help="skip measuring each shape's configurations (sfc_gemm_tune) before timing; the tile then "
+                         "comes from the library's time model")
     ap.add_argument("--sustained", action="store_true",
                     help="instead of the step timing: run each configuration back to back for --phase-seconds under "
                          "the power cap (ours by order / dealing / tile / K blocks, then cuBLAS) at each --sizes "
@@ -325,6 +328,16 @@ def run_ours(args, rank, local, world):
         sfc.gemm(m["Ad"], m["Bd"], m["C"], ca_c=c, order=args.order, assign=args.assign, stream=stream,
                  b_layout=args.b_layout, k_block_factor=args.k_block_factor)
 
+    # measure each shape's tiles (and layer counts where several are listed) once, untimed; the
+    # timed calls below keep tile="auto", which then uses the measured choice (the tile never
+    # changes the result's bits)
+    tuned = {}
+    if not args.no_tune and args.k_block_factor == 1:
+        for i, m in enumerate(mats):
+            tuned[i] = sfc.tune(m["Ad"], m["Bd"], m["C"], max_layers=max(m["s"]["cs"]), max_kbf=1,
+                                b_layout=args.b_layout, stream=stream)
+        torch.cuda.synchronize()
+
     # pick the K-layer count per shape where several are listed (timed, warm)
     cs_report = {}
     for i, m in enumerate(mats):
@@ -454,6 +467,8 @@ def run_ours(args, rank, local, world):
                "frac_of_roofline_back_to_back": round(t_roof / (b2b_ms[i] * 1e-3), 4)}
         if i in cs_report:
             row["ms_by_ca_c"] = cs_report[i]
+        row["tile"] = sfc.plan(s["M"], s["N"], s["K"], m["c"], out_dtype=m["C"].dtype, in_dtype=m["Ad"].dtype,
+                               b_layout=args.b_layout)[0]
         per_shape.append(row)
 
     # roofline of the dominant kernel (the GEMM kernel; the K-layer reduction,
@@ -496,6 +511,8 @@ def run_ours(args, rank, local, world):
         "data": "synthetic (seeded %s %s)" % (",".join(sorted({m["s"]["kind"] for m in mats})), args.ab),
         "config": {"workload": desc, "order": args.order, "assign": args.assign, "b_layout": args.b_layout,
                    "inputs": args.ab, "k_block_factor": args.k_block_factor,
+                   "tile": "measured per shape before timing (sfc_gemm_tune, untimed)" if tuned
+                           else "the library's time model",
                    "parallelism": "replicas" if world > 1 else "single GPU",
                    "l2": "inputs larger than L2 between reuses: one step runs every shape once, so a shape's "
                          "operands are re-read only after the other shapes' traffic has passed through L2",

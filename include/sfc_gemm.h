@@ -258,6 +258,40 @@ size_t sfc_gemm_workspace_size2(int64_t M, int64_t N, int64_t K, int ca_c, int k
                                 sfc_dtype_t c_dtype);
 
 /*
+ * sfc_gemm_tune -- measures the configurations of one shape and remembers the
+ * fastest (the paper's first way to configure a shape: benchmark the small
+ * space of knobs exhaustively, Sec. III-C).  For each layer count in 1, 2, 4,
+ * ... up to max_layers (and the time model's own choice) every tile shape is
+ * timed (one warm-up call, then the mean of three, CUDA events on `stream`);
+ * then K blocks 2, 4, ... up to max_kbf are timed on the fastest (tile,
+ * layers).  The results go into a per-device table for this (M, N, K,
+ * ab_dtype, b_layout, c_dtype): afterwards calls with tile = SFC_TILE_AUTO and
+ * k_block_factor = 1 use the fastest tile measured for their layer count, and
+ * with ca_c = 0 also the fastest layer count (sfc_gemm_plan reports the
+ * same).  The tile never changes the result's bits; the layer count does, so
+ * callers that need the same bits on every machine pass ca_c explicitly.
+ *   A, B, C, strides, ab_dtype, b_layout, c_dtype: as sfc_gemm_ex2; C is
+ *     overwritten, and holds the chosen configuration's result on return.
+ *   max_layers: 1..64 (1 tunes the tile only); max_kbf: 1..64.
+ *   out_tile, out_ca_c, out_kbf: the fastest configuration (tile as sfc_tile_t).
+ * Synchronizes `stream` (it times on the host), so it cannot be captured:
+ * SFC_ERR_UNSUPPORTED while `stream` is capturing.  Errors: as sfc_gemm_ex2,
+ * SFC_ERR_INVALID_ARG for a null output pointer or bounds out of range.
+ * Thread safety: the table is guarded; tuning the same shape from two
+ * threads at once times each candidate with the other's launches beside it.
+ */
+int sfc_gemm_tune(int64_t M, int64_t N, int64_t K,
+                  const void *A, const void *B, void *C,
+                  int64_t lda, int64_t ldb, int64_t ldc,
+                  int ab_dtype, int b_layout, sfc_dtype_t c_dtype,
+                  int max_layers, int max_kbf, void *stream,
+                  int *out_tile, int *out_ca_c, int *out_kbf);
+
+/* sfc_gemm_tune_forget -- empties the current device's table of tuned
+ * shapes (calls go back to the time model).  SFC_OK or a CUDA error. */
+int sfc_gemm_tune_forget(void);
+
+/*
  * sfc_gemm_plan -- the tile and K-layer count sfc_gemm_ex2 would use for these
  * arguments on the current device (ca_c = 0: the library's choice; ca_c >= 1:
  * that count with the tile AUTO or `tile` picks).  No kernel runs.

@@ -45,7 +45,7 @@ def _ab_code(dtype) -> int:
 EXPORTS = ("sfc_tile_order", "sfc_tile_order_device", "sfc_gemm_workspace_size", "sfc_gemm", "sfc_gemm_ex",
            "sfc_get_device_status", "sfc_last_cuda_error", "sfc_num_workers", "sfc_debug_force_timeout",
            "sfc_gemm_noalloc", "sfc_gemm_plan", "sfc_release", "sfc_gemm_ex2", "sfc_gemm_host", "sfc_gemm_ex3",
-           "sfc_gemm_workspace_size2")
+           "sfc_gemm_workspace_size2", "sfc_gemm_tune", "sfc_gemm_tune_forget")
 NOALLOC_SCRATCH_BYTES = 32 << 20
 
 
@@ -102,6 +102,8 @@ def load():
         lib.sfc_gemm_ex3.argtypes = [i64, i64, i64, vp, vp, vp, i64, i64, i64, i32, i32, ctypes.c_float, vp, i32,
                                      i32, i32, i32, i32, i32, vp, sz, vp]
         lib.sfc_gemm_workspace_size2.argtypes = [i64, i64, i64, i32, i32, i32]
+        lib.sfc_gemm_tune.argtypes = [i64, i64, i64, vp, vp, vp, i64, i64, i64, i32, i32, i32, i32, i32, vp, vp, vp, vp]
+        lib.sfc_gemm_tune_forget.argtypes = []
         lib.sfc_gemm_workspace_size2.restype = sz
         for name in EXPORTS:
             if name not in ("sfc_gemm_workspace_size", "sfc_gemm_workspace_size2"):
@@ -163,6 +165,33 @@ def plan(M: int, N: int, K: int, ca_c: int = 0, out_dtype=None, tile="auto", in_
                                 ctypes.byref(t), ctypes.byref(c)), "sfc_gemm_plan")
     name = {v: k for k, v in TILES.items() if k not in (0, "auto")}[t.value]
     return name, c.value
+
+
+def tune(A, B, C=None, *, out_dtype=None, b_layout: str = "kn", max_layers: int = 8, max_kbf: int = 4,
+         stream=None):
+    """Measure the configurations of this shape (``sfc_gemm_tune``) and remember
+    the fastest for later calls with ``tile="auto"``.  A, B: CUDA tensors as
+    for :func:`gemm`; C is overwritten (allocated if not given).  Returns
+    ``(tile, ca_c, k_block_factor)`` of the fastest configuration."""
+    import torch
+    M, K = A.shape
+    N = B.shape[1] if b_layout == "kn" else B.shape[0]
+    if C is None:
+        C = torch.empty((M, N), dtype=out_dtype or torch.float32, device=A.device)
+    t, c, kbf = ctypes.c_int(0), ctypes.c_int(0), ctypes.c_int(0)
+    rc = load().sfc_gemm_tune(M, N, K, ctypes.c_void_p(A.data_ptr()), ctypes.c_void_p(B.data_ptr()),
+                              ctypes.c_void_p(C.data_ptr()), _row_major_2d(A, "A"), _row_major_2d(B, "B"),
+                              _row_major_2d(C, "C"), _ab_code(A.dtype), B_LAYOUTS[b_layout],
+                              SFC_F32 if C.dtype == torch.float32 else SFC_BF16, int(max_layers), int(max_kbf),
+                              _stream_ptr(stream), ctypes.byref(t), ctypes.byref(c), ctypes.byref(kbf))
+    _check(rc, "sfc_gemm_tune")
+    name = {v: k for k, v in TILES.items() if k not in (0, "auto")}[t.value]
+    return name, c.value, kbf.value
+
+
+def tune_forget() -> None:
+    """Forget every tuned shape on the current device."""
+    _check(load().sfc_gemm_tune_forget(), "sfc_gemm_tune_forget")
 
 
 def release() -> None:

@@ -8,7 +8,11 @@
 #include <cstdint>
 #include <cstdlib>
 #include <cstring>
+#include <algorithm>
+#include <map>
 #include <mutex>
+#include <tuple>
+#include <vector>
 
 #include "sfc_gemm.h"
 #include "sfc_gemm_kernel.cuh"
@@ -413,6 +417,59 @@ cudaError_t launch_gemm(int v, bool f8, const CUtensorMap& ta, const CUtensorMap
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
+// ------------------------------------------------------------ tuning table
+// Shapes measured by sfc_gemm_tune (the paper's a-priori autotuning of a
+// shape, Sec. III-C): per layer count the fastest tile, and the fastest
+// (tile, layers, K blocks) overall.  Calls with tile = AUTO (and one K block)
+// use them; everything else uses the time model.
+constexpr int kTuneMaxLayers = 64;
+
+struct TuneKey {
+    int64_t M, N, K;
+    int ab, b_layout, c_dtype;
+    bool operator<(const TuneKey& o) const {
+        return std::tie(M, N, K, ab, b_layout, c_dtype) < std::tie(o.M, o.N, o.K, o.ab, o.b_layout, o.c_dtype);
+    }
+};
+
+struct TuneEntry {
+    int tile_for_c[kTuneMaxLayers + 1];  // SFC_TILE_* per layer count, 0 = not measured
+    int tile, c, kbf;                    // fastest overall
+};
+
+struct TuneTable {
+    std::mutex mu;
+    std::map<TuneKey, TuneEntry> map;
+};
+TuneTable g_tune[kMaxDevices];
+
+constexpr int kTileOf[kNumVariants] = {SFC_TILE_N128, SFC_TILE_N256, SFC_TILE_PAIR_N128, SFC_TILE_PAIR_N256,
+                                       SFC_TILE_QUAD_N256};
+
+// Tuned (tile, layers) for a call that lets the library choose the tile:
+// with ca_c > 0 the fastest tile for that layer count, with ca_c = 0 the
+// fastest pair.  False when the shape was not tuned (or not at that count).
+bool tuned_choice(int64_t M, int64_t N, int64_t K, int ab, int b_layout, int c_dtype, int ca_c, int* tile,
+                  int* layers) {
+    int dev;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return false;
+    TuneTable& t = g_tune[dev];
+    std::lock_guard<std::mutex> lock(t.mu);
+    if (t.map.empty()) return false;
+    auto it = t.map.find(TuneKey{M, N, K, ab, b_layout, c_dtype});
+    if (it == t.map.end()) return false;
+    const TuneEntry& e = it->second;
+    if (ca_c == 0) {
+        *tile = e.tile;
+        *layers = e.c;
+        return true;
+    }
+    if (ca_c > kTuneMaxLayers || e.tile_for_c[ca_c] == 0) return false;
+    *tile = e.tile_for_c[ca_c];
+    *layers = ca_c;
+    return true;
+}
+
 // Operands whose rows (or base) are not 16-byte aligned are copied into
 // padded pool buffers (packed[0] for A, packed[1] for B), and the pointer and
 // row stride are redirected to the copy.
@@ -503,6 +560,16 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     DeviceInfo* dev = nullptr;
     rc = device_setup(&dev);
     if (rc != SFC_OK) return rc;
+
+    // a tuned shape: its measured tile (and, for ca_c = 0, layer count) replace the time model's
+    if (tile == SFC_TILE_AUTO && kbf == 1) {
+        int t_tile = 0, t_c = 0;
+        if (tuned_choice(M, N, K, ab, b_layout, c_dtype, ca_c, &t_tile, &t_c) &&
+            (ca_c > 0 || !workspace || workspace_bytes >= workspace_bytes_for(M, N, t_c, 1, c_dtype))) {
+            tile = t_tile;
+            ca_c = t_c;
+        }
+    }
 
     // ca_c = 0: the planner's layer count, within the caller's workspace if one is given
     int max_c = static_cast<int>(auto_layer_cap(M, N, K, ab));
@@ -699,11 +766,16 @@ SFC_API int sfc_gemm_plan(int64_t M, int64_t N, int64_t K, int ca_c, int c_dtype
     DeviceInfo* dev = nullptr;
     rc = device_setup(&dev);
     if (rc != SFC_OK) return rc;
+    if (tile == SFC_TILE_AUTO) {
+        int t_tile = 0, t_c = 0;
+        if (tuned_choice(M, N, K, ab_dtype, b_layout, c_dtype, ca_c, &t_tile, &t_c)) {
+            tile = t_tile;
+            ca_c = t_c;
+        }
+    }
     const Plan plan = make_plan(M, N, K, ca_c, static_cast<int>(auto_layer_cap(M, N, K, ab_dtype)), *dev,
                                 static_cast<sfc_tile_t>(tile), c_dtype == SFC_F32 ? 4 : 2, b_layout == SFC_B_NK,
                                 ab_dtype);
-    static const int kTileOf[kNumVariants] = {SFC_TILE_N128, SFC_TILE_N256, SFC_TILE_PAIR_N128, SFC_TILE_PAIR_N256,
-                                              SFC_TILE_QUAD_N256};
     *out_tile = kTileOf[plan.v];
     *out_ca_c = plan.c;
     return SFC_OK;
@@ -767,6 +839,120 @@ SFC_API size_t sfc_gemm_workspace_size2(int64_t M, int64_t N, int64_t K, int ca_
         if (layers < 1) layers = 1;
     }
     return workspace_bytes_for(M, N, static_cast<int>(layers), k_block_factor, c_dtype);
+}
+
+SFC_API int sfc_gemm_tune(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void* C, int64_t lda,
+                          int64_t ldb, int64_t ldc, int ab_dtype, int b_layout, sfc_dtype_t c_dtype, int max_layers,
+                          int max_kbf, void* stream, int* out_tile, int* out_ca_c, int* out_kbf) {
+    if (!out_tile || !out_ca_c || !out_kbf) return SFC_ERR_INVALID_ARG;
+    if (max_layers < 1 || max_layers > kTuneMaxLayers || max_kbf < 1 || max_kbf > kMaxKBlocks)
+        return SFC_ERR_INVALID_ARG;
+    int rc = validate(M, N, K, A, B, C, lda, ldb, ldc, 1, c_dtype, SFC_ORDER_SFC, SFC_ASSIGN_AUTO, SFC_TILE_AUTO,
+                      b_layout, ab_dtype);
+    if (rc != SFC_OK) return rc;
+    DeviceInfo* dev = nullptr;
+    rc = device_setup(&dev);
+    if (rc != SFC_OK) return rc;
+    int devi = 0;
+    rc = current_device(&devi);
+    if (rc != SFC_OK) return rc;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaStreamCaptureStatus capturing = cudaStreamCaptureStatusNone;
+    cudaError_t e = cudaStreamIsCapturing(s, &capturing);
+    if (e != cudaSuccess) return cuda_fail(e);
+    if (capturing != cudaStreamCaptureStatusNone) return SFC_ERR_UNSUPPORTED;  // it times on the host
+
+    const int64_t Kt = ceil_div(K, slab_k(ab_dtype));
+    const bool b_kmajor = (b_layout == SFC_B_NK);
+    // layer counts 1, 2, 4, ... and the time model's own choice
+    std::vector<int> counts;
+    for (int c = 1; c <= max_layers && c <= Kt; c *= 2) counts.push_back(c);
+    const Plan model = make_plan(M, N, K, 0, static_cast<int>(auto_layer_cap(M, N, K, ab_dtype)), *dev,
+                                 SFC_TILE_AUTO, c_dtype == SFC_F32 ? 4 : 2, b_kmajor, ab_dtype);
+    if (model.c <= max_layers && std::find(counts.begin(), counts.end(), model.c) == counts.end())
+        counts.push_back(model.c);
+
+    cudaEvent_t e0 = nullptr, e1 = nullptr;
+    e = cudaEventCreate(&e0);
+    if (e == cudaSuccess) e = cudaEventCreate(&e1);
+    if (e != cudaSuccess) {
+        if (e0) cudaEventDestroy(e0);
+        return cuda_fail(e);
+    }
+    auto call = [&](int c, int tile, int kbf) {
+        return run_gemm(M, N, K, A, B, C, lda, ldb, ldc, c, c_dtype, SFC_ORDER_SFC, SFC_ASSIGN_AUTO, tile, nullptr,
+                        0, s, 0, kDefaultTimeoutNs, b_layout, 0.0f, nullptr, ab_dtype, true, kbf);
+    };
+    // one call to warm up, then the mean of three
+    auto measure = [&](int c, int tile, int kbf, float* us) {
+        int r = call(c, tile, kbf);
+        cudaError_t ce = cudaSuccess;
+        if (r == SFC_OK) ce = cudaEventRecord(e0, s);
+        for (int i = 0; i < 3 && r == SFC_OK && ce == cudaSuccess; ++i) r = call(c, tile, kbf);
+        if (r == SFC_OK && ce == cudaSuccess) ce = cudaEventRecord(e1, s);
+        if (r == SFC_OK && ce == cudaSuccess) ce = cudaEventSynchronize(e1);
+        float ms = 0.0f;
+        if (r == SFC_OK && ce == cudaSuccess) ce = cudaEventElapsedTime(&ms, e0, e1);
+        if (r == SFC_OK && ce != cudaSuccess) r = cuda_fail(ce);
+        *us = ms * 1000.0f / 3.0f;
+        return r;
+    };
+
+    TuneEntry entry;
+    std::memset(&entry, 0, sizeof(entry));
+    float best = -1.0f;
+    for (int c : counts) {
+        float best_c = -1.0f;
+        for (int v = 0; v < kNumVariants && rc == SFC_OK; ++v) {
+            if (dev->workers[v] <= 0 || !variant_allowed(v, b_kmajor, ab_dtype)) continue;
+            float us = 0.0f;
+            rc = measure(c, kTileOf[v], 1, &us);
+            if (rc != SFC_OK) break;
+            if (best_c < 0.0f || us < best_c) {
+                best_c = us;
+                entry.tile_for_c[c] = kTileOf[v];
+            }
+            if (best < 0.0f || us < best) {
+                best = us;
+                entry.tile = kTileOf[v];
+                entry.c = c;
+                entry.kbf = 1;
+            }
+        }
+        if (rc != SFC_OK) break;
+    }
+    // K blocks on the fastest (tile, layers)
+    for (int kbf = 2; rc == SFC_OK && kbf <= max_kbf && Kt / entry.c >= kbf; kbf *= 2) {
+        float us = 0.0f;
+        rc = measure(entry.c, entry.tile, kbf, &us);
+        if (rc == SFC_OK && us < best) {
+            best = us;
+            entry.kbf = kbf;
+        }
+    }
+    if (rc == SFC_OK) rc = call(entry.c, entry.tile, entry.kbf);  // C holds the chosen configuration's result
+    cudaEventDestroy(e0);
+    cudaEventDestroy(e1);
+    if (rc != SFC_OK) return rc;
+    {
+        TuneTable& t = g_tune[devi];
+        std::lock_guard<std::mutex> lock(t.mu);
+        t.map[TuneKey{M, N, K, ab_dtype, b_layout, c_dtype}] = entry;
+    }
+    *out_tile = entry.tile;
+    *out_ca_c = entry.c;
+    *out_kbf = entry.kbf;
+    return SFC_OK;
+}
+
+SFC_API int sfc_gemm_tune_forget(void) {
+    int dev;
+    int rc = current_device(&dev);
+    if (rc != SFC_OK) return rc;
+    TuneTable& t = g_tune[dev];
+    std::lock_guard<std::mutex> lock(t.mu);
+    t.map.clear();
+    return SFC_OK;
 }
 
 SFC_API int sfc_get_device_status(void* stream) {

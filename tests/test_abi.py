@@ -230,3 +230,20 @@ def test_gemm_ex3_validation_codes(lib):
     assert call_ex3(lib, K=1024, ca_c=4, kbf=5) == E.SFC_ERR_INVALID_ARG       # 16 slabs: 4 per layer < 5
     assert call_ex3(lib, K=1024, ab=1, ca_c=2, kbf=5) == E.SFC_ERR_INVALID_ARG  # 8 slabs of 128: 4 per layer
     assert call_ex3(lib, M=0) == E.SFC_ERR_INVALID_ARG
+
+
+def test_gemm_tune_validation_codes(lib):
+    # rejected on the host before the device is touched
+    E = binding
+    t, c, k = ctypes.c_int(0), ctypes.c_int(0), ctypes.c_int(0)
+
+    def tune(M=256, N=256, K=256, max_layers=8, max_kbf=4, outs=True):
+        args = (ctypes.byref(t), ctypes.byref(c), ctypes.byref(k)) if outs else (None, None, None)
+        return lib.sfc_gemm_tune(M, N, K, ctypes.c_void_p(PA), ctypes.c_void_p(PB), ctypes.c_void_p(PC), K, N, N,
+                                 0, 0, 0, max_layers, max_kbf, None, *args)
+    assert tune(outs=False) == E.SFC_ERR_INVALID_ARG
+    assert tune(max_layers=0) == E.SFC_ERR_INVALID_ARG
+    assert tune(max_layers=65) == E.SFC_ERR_INVALID_ARG
+    assert tune(max_kbf=0) == E.SFC_ERR_INVALID_ARG
+    assert tune(max_kbf=65) == E.SFC_ERR_INVALID_ARG
+    assert tune(M=0) == E.SFC_ERR_INVALID_ARG
