@@ -291,6 +291,16 @@ int sfc_gemm_tune(int64_t M, int64_t N, int64_t K,
  * shapes (calls go back to the time model).  SFC_OK or a CUDA error. */
 int sfc_gemm_tune_forget(void);
 
+/* sfc_gemm_tune_lookup -- how AUTO calls consult the table (process-wide):
+ * 1 (default) only a shape tuned exactly; 2 otherwise the nearest tuned shape
+ * with the same input type, B layout and output type, by distance in
+ * (log M, log N, log K), that was measured at the call's layer count (for
+ * ca_c = 0: whose layer count fits the call's K) -- the paper's
+ * nearest-neighbour prediction of a shape's knobs (Sec. III-C).  With 2 the
+ * layer count of a ca_c = 0 call can come from another shape.
+ * SFC_ERR_INVALID_ARG for another mode. */
+int sfc_gemm_tune_lookup(int mode);
+
 /*
  * sfc_gemm_plan -- the tile and K-layer count sfc_gemm_ex2 would use for these
  * arguments on the current device (ca_c = 0: the library's choice; ca_c >= 1:

@@ -45,7 +45,8 @@ def _ab_code(dtype) -> int:
 EXPORTS = ("sfc_tile_order", "sfc_tile_order_device", "sfc_gemm_workspace_size", "sfc_gemm", "sfc_gemm_ex",
            "sfc_get_device_status", "sfc_last_cuda_error", "sfc_num_workers", "sfc_debug_force_timeout",
            "sfc_gemm_noalloc", "sfc_gemm_plan", "sfc_release", "sfc_gemm_ex2", "sfc_gemm_host", "sfc_gemm_ex3",
-           "sfc_gemm_workspace_size2", "sfc_gemm_tune", "sfc_gemm_tune_forget")
+           "sfc_gemm_workspace_size2", "sfc_gemm_tune", "sfc_gemm_tune_forget",
+           "sfc_gemm_tune_lookup")
 NOALLOC_SCRATCH_BYTES = 32 << 20
 
 
@@ -104,6 +105,7 @@ def load():
         lib.sfc_gemm_workspace_size2.argtypes = [i64, i64, i64, i32, i32, i32]
         lib.sfc_gemm_tune.argtypes = [i64, i64, i64, vp, vp, vp, i64, i64, i64, i32, i32, i32, i32, i32, vp, vp, vp, vp]
         lib.sfc_gemm_tune_forget.argtypes = []
+        lib.sfc_gemm_tune_lookup.argtypes = [i32]
         lib.sfc_gemm_workspace_size2.restype = sz
         for name in EXPORTS:
             if name not in ("sfc_gemm_workspace_size", "sfc_gemm_workspace_size2"):
@@ -187,6 +189,12 @@ def tune(A, B, C=None, *, out_dtype=None, b_layout: str = "kn", max_layers: int 
     _check(rc, "sfc_gemm_tune")
     name = {v: k for k, v in TILES.items() if k not in (0, "auto")}[t.value]
     return name, c.value, kbf.value
+
+
+def tune_lookup(nearest: bool) -> None:
+    """AUTO calls use tuned shapes exactly (False, the default) or also the
+    nearest tuned shape (True; ``sfc_gemm_tune_lookup``)."""
+    _check(load().sfc_gemm_tune_lookup(2 if nearest else 1), "sfc_gemm_tune_lookup")
 
 
 def tune_forget() -> None:

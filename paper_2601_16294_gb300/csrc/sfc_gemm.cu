@@ -9,6 +9,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <algorithm>
+#include <cmath>
 #include <map>
 #include <mutex>
 #include <tuple>
@@ -442,6 +443,7 @@ struct TuneTable {
     std::map<TuneKey, TuneEntry> map;
 };
 TuneTable g_tune[kMaxDevices];
+std::atomic<int> g_tune_lookup{1};  // 1: exact shape only; 2: else the nearest tuned shape (Sec. III-C, third way)
 
 constexpr int kTileOf[kNumVariants] = {SFC_TILE_N128, SFC_TILE_N256, SFC_TILE_PAIR_N128, SFC_TILE_PAIR_N256,
                                        SFC_TILE_QUAD_N256};
@@ -457,6 +459,24 @@ bool tuned_choice(int64_t M, int64_t N, int64_t K, int ab, int b_layout, int c_d
     std::lock_guard<std::mutex> lock(t.mu);
     if (t.map.empty()) return false;
     auto it = t.map.find(TuneKey{M, N, K, ab, b_layout, c_dtype});
+    if (it == t.map.end() && g_tune_lookup.load(std::memory_order_relaxed) == 2) {
+        // nearest tuned shape of the same types and layout, by distance in log M, log N, log K;
+        // it must have been measured at the asked layer count, and its layer count must fit K
+        const int64_t Kt = ceil_div(K, slab_k(ab));
+        double best = -1.0;
+        for (auto cand = t.map.begin(); cand != t.map.end(); ++cand) {
+            const TuneKey& k = cand->first;
+            if (k.ab != ab || k.b_layout != b_layout || k.c_dtype != c_dtype) continue;
+            if (ca_c > 0 ? (ca_c > kTuneMaxLayers || cand->second.tile_for_c[ca_c] == 0) : cand->second.c > Kt)
+                continue;
+            const double dm = std::log(double(M) / k.M), dn = std::log(double(N) / k.N), dk = std::log(double(K) / k.K);
+            const double d = dm * dm + dn * dn + dk * dk;
+            if (best < 0.0 || d < best) {
+                best = d;
+                it = cand;
+            }
+        }
+    }
     if (it == t.map.end()) return false;
     const TuneEntry& e = it->second;
     if (ca_c == 0) {
@@ -942,6 +962,12 @@ SFC_API int sfc_gemm_tune(int64_t M, int64_t N, int64_t K, const void* A, const 
     *out_tile = entry.tile;
     *out_ca_c = entry.c;
     *out_kbf = entry.kbf;
+    return SFC_OK;
+}
+
+SFC_API int sfc_gemm_tune_lookup(int mode) {
+    if (mode != 1 && mode != 2) return SFC_ERR_INVALID_ARG;
+    g_tune_lookup.store(mode, std::memory_order_relaxed);
     return SFC_OK;
 }
 

@@ -247,3 +247,10 @@ def test_gemm_tune_validation_codes(lib):
     assert tune(max_kbf=0) == E.SFC_ERR_INVALID_ARG
     assert tune(max_kbf=65) == E.SFC_ERR_INVALID_ARG
     assert tune(M=0) == E.SFC_ERR_INVALID_ARG
+
+
+def test_tune_lookup_modes(lib):
+    assert lib.sfc_gemm_tune_lookup(3) == binding.SFC_ERR_INVALID_ARG
+    assert lib.sfc_gemm_tune_lookup(0) == binding.SFC_ERR_INVALID_ARG
+    assert lib.sfc_gemm_tune_lookup(2) == binding.SFC_OK
+    assert lib.sfc_gemm_tune_lookup(1) == binding.SFC_OK

@@ -67,3 +67,28 @@ def test_tuning_is_refused_during_capture(sfc):
         with torch.cuda.graph(g, stream=s):
             sfc.tune(A, B, C, stream=s)
     assert e.value.code == binding.SFC_ERR_UNSUPPORTED
+
+
+def test_nearest_tuned_shape(sfc):
+    sfc.tune_forget()
+    M, N, K = 3000, 5000, 7000
+    A, B = inputs(M, N, K, 11)
+    tile, c, _ = sfc.tune(A, B, out_dtype=torch.bfloat16, max_layers=1, max_kbf=1)
+    near = (3100, 4900, 7000)                                          # never tuned
+    model = sfc.plan(*near, ca_c=1, out_dtype=torch.bfloat16)
+    try:
+        sfc.tune_lookup(True)
+        assert sfc.plan(*near, ca_c=1, out_dtype=torch.bfloat16) == (tile, 1)
+        # other output types are other tables
+        f32 = sfc.plan(*near, ca_c=1)
+        sfc.tune_lookup(False)
+        assert sfc.plan(*near, ca_c=1) == f32
+        Anear, Bnear = inputs(*near, 12)
+        sfc.tune_lookup(True)
+        got = sfc.gemm(Anear, Bnear, ca_c=1, out_dtype=torch.bfloat16)
+        sfc.tune_lookup(False)
+        assert torch.equal(got, sfc.gemm(Anear, Bnear, ca_c=1, out_dtype=torch.bfloat16))   # the tile keeps the bits
+    finally:
+        sfc.tune_lookup(False)
+    assert sfc.plan(*near, ca_c=1, out_dtype=torch.bfloat16) == model   # exact lookup again
+    sfc.tune_forget()
