@@ -1,0 +1,46 @@
+"""bench.py's output contract on a GPU: one JSON line with the metric, the
+whole-job value, the roofline of the dominant kernel, the end-to-end rate from
+host buffers, the clocks seen during the timed region, the launch count and
+the oracle's CPU rate (small sizes, a few steps).  The reference arm's line is
+checked on CPU (test_bench_dist.py)."""
+import json
+import os
+import subprocess
+import sys
+
+import pytest
+
+pytestmark = pytest.mark.gpu
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def run_bench(*args):
+    out = subprocess.run([sys.executable, "bench.py", *args], cwd=ROOT, capture_output=True, text=True, timeout=600)
+    assert out.returncode == 0, out.stderr[-2000:]
+    lines = [line for line in out.stdout.splitlines() if line.strip()]
+    assert len(lines) == 1, out.stdout
+    return json.loads(lines[0])
+
+
+def test_default_line_keys():
+    d = run_bench("--sizes", "2048,4096", "--steps", "3", "--warmup", "3", "--no-cublas")
+    for key in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step", "higher_is_better", "scaling",
+                "vs_baseline", "dtype", "data", "config", "roofline", "gpu_launches", "e2e", "cpu_baseline",
+                "clocks", "per_shape"):
+        assert key in d, key
+    assert d["n_gpus"] == 1 and d["steps"] == 3 and d["warmup"] == 3 and d["higher_is_better"] is True
+    assert d["value"] > 0 and d["unit"] == "TFLOP/s" and d["dtype"] == "bf16"
+    assert "workload" in d["config"]
+    r = d["roofline"]
+    assert r["bound"] == "tensor" and r["unit"] == "TFLOP/s" and r["peak"] > 0
+    assert abs(r["frac"] - r["achieved"] / r["peak"]) < 1e-3
+    e = d["e2e"]
+    assert e["value"] > 0 and e["h2d_bytes_per_step"] == 2 * 2 * (2048 ** 2 + 4096 ** 2)   # A and B, bf16
+    assert e["d2h_bytes_per_step"] == 2 * (2048 ** 2 + 4096 ** 2)
+    assert d["gpu_launches"] == 3 * 2                                    # one GEMM launch per shape per step
+    c = d["cpu_baseline"]
+    assert c["kind"] == "oracle" and c["cores"] >= 1 and c["value"] > 0
+    assert {"sm_mhz", "sm_max_mhz", "reasons"} <= set(d["clocks"])
+    assert len(d["per_shape"]) == 2 and all(p["tile"] for p in d["per_shape"])
+
