@@ -97,7 +97,9 @@ typedef enum {
  *                        (a 2-CTA cluster; each SM loads half of A and half of B).
  * QUAD_N256:             512 x 256 tiles computed by two such pairs (a 4-CTA
  *                        cluster) that share the B slab by TMA multicast.
- * AUTO picks per shape from the tile count and the number of workers. */
+ * AUTO: the tile sfc_gemm_tune measured fastest for the shape (and layer
+ * count), else the time model's pick from the tile count and the number of
+ * workers.  Every tile shape gives the same bits. */
 typedef enum {
     SFC_TILE_AUTO = 0,
     SFC_TILE_N128 = 128,
@@ -149,7 +151,8 @@ size_t sfc_gemm_workspace_size(int64_t M, int64_t N, int64_t K, int ca_c);
  *         tile) from a model of the call's time on this device: waves of
  *         items times the length of a layer, plus the reduction's cost for
  *         more than one layer (the replication factor choice of Sec. II-D,
- *         made per call); sfc_gemm_plan reports the choice.
+ *         made per call), or the count sfc_gemm_tune measured fastest for the
+ *         shape; sfc_gemm_plan reports the choice.
  *   stream: a cudaStream_t passed as void*.
  * Alignment: the tile loads (Tensor Memory Accelerator) read 16-byte-aligned
  * rows.  When A or B is not 16-byte aligned, or lda / ldb is not a multiple of
