@@ -1,7 +1,9 @@
 """Seeded random configurations against the oracle: random shapes (ragged in
 every dimension), input type, B layout, tile, layer count, K blocks, order,
 dealing, output type, beta and bias, on integer data, where every fp32 step is
-exact, so the result must equal the oracle bit for bit."""
+exact, so the result must equal the oracle bit for bit; and random host-buffer
+calls (shape, layout, output type, panel count, host row padding), which must
+equal the device call with the same plan bit for bit."""
 import numpy as np
 import pytest
 import torch
@@ -77,3 +79,26 @@ def test_random_configuration(sfc, oracle, i):
     got = C.float().cpu().numpy().astype(np.float64)
     want = ref if cfg["out"] == torch.float32 else oracle.round_bf16(ref)
     assert np.array_equal(got, want), cfg
+
+
+@pytest.mark.parametrize("i", range(16))
+def test_random_host_configuration(sfc, i):
+    # the host-buffer path against the device call with the same plan: bit-identical
+    rng = np.random.default_rng(5000 + i)
+    M, N, K = (int(rng.integers(1, 3000)) for _ in range(3))
+    layout = str(rng.choice(["kn", "nk"]))
+    out = torch.float32 if rng.random() < 0.5 else torch.bfloat16
+    panels = int(rng.choice([0, 1, 2, 3, 7]))
+    A, B = synth.gemm_inputs(M, N, K, "uniform", seed=int(rng.integers(1 << 30)))
+    Bl = B if layout == "kn" else B.t().contiguous()
+
+    def host(t):
+        ld = t.shape[1] + int(rng.integers(0, 5))
+        h = torch.zeros(t.shape[0], ld, dtype=t.dtype, pin_memory=True)
+        h[:, : t.shape[1]] = t
+        return h[:, : t.shape[1]]
+    tile, c = sfc.plan(M, N, K, ca_c=0, out_dtype=out, b_layout=layout)
+    ref = sfc.gemm(padded(A, (K + 7) // 8 * 8), padded(Bl, (Bl.shape[1] + 7) // 8 * 8), ca_c=c, tile=tile,
+                   out_dtype=out, b_layout=layout).cpu()
+    got = sfc.matmul_host(host(A), host(Bl), ca_c=0, out_dtype=out, b_layout=layout, panels=panels)
+    assert torch.equal(got, ref), (M, N, K, layout, out, panels)
