@@ -31,16 +31,23 @@ TILES = {0: 0, "auto": 0, 128: 128, 256: 256, "pair128": 1128, "pair256": 1256, 
 B_LAYOUTS = {"kn": 0, "nk": 1}
 
 
+_AB_CODES = None
+
+
 def _ab_code(dtype) -> int:
     """sfc_ab_t of a torch dtype of A and B."""
-    import torch
-    codes = {torch.bfloat16: 0}
-    for name, code in (("float8_e4m3fn", 1), ("float8_e5m2", 2)):
-        if hasattr(torch, name):
-            codes[getattr(torch, name)] = code
-    if dtype not in codes:
+    global _AB_CODES
+    if _AB_CODES is None:
+        import torch
+        codes = {torch.bfloat16: 0}
+        for name, code in (("float8_e4m3fn", 1), ("float8_e5m2", 2)):
+            if hasattr(torch, name):
+                codes[getattr(torch, name)] = code
+        _AB_CODES = codes
+    code = _AB_CODES.get(dtype)
+    if code is None:
         raise TypeError("A and B must be bfloat16, float8_e4m3fn or float8_e5m2 (got %s)" % dtype)
-    return codes[dtype]
+    return code
 
 EXPORTS = ("sfc_tile_order", "sfc_tile_order_device", "sfc_gemm_workspace_size", "sfc_gemm", "sfc_gemm_ex",
            "sfc_get_device_status", "sfc_last_cuda_error", "sfc_num_workers", "sfc_debug_force_timeout",
@@ -120,10 +127,10 @@ def _check(rc: int, what: str):
 
 
 def _stream_ptr(stream):
-    import torch
     if stream is None:
+        import torch
         stream = torch.cuda.current_stream()
-    return ctypes.c_void_p(stream.cuda_stream)
+    return stream.cuda_stream
 
 
 # ------------------------------------------------------------------ curve
@@ -235,7 +242,7 @@ def gemm(A, B, C=None, *, ca_c: int = 1, out_dtype=None, order: str = "sfc", ass
     tensor of at least ``workspace_size(M, N, K, ca_c, k_block_factor,
     out_dtype)`` bytes."""
     import torch
-    lib = load()
+    lib = _lib or load()
     M, K = A.shape
     if b_layout == "kn":
         K2, N = B.shape
@@ -258,17 +265,17 @@ def gemm(A, B, C=None, *, ca_c: int = 1, out_dtype=None, order: str = "sfc", ass
     if bias is not None:
         if bias.dtype != torch.float32 or bias.numel() != N or not bias.is_contiguous():
             raise ValueError("bias must be a contiguous float32 tensor of N values")
-        bias_ptr = ctypes.c_void_p(bias.data_ptr())
+        bias_ptr = bias.data_ptr()
     lda = _row_major_2d(A, "A")
     ldb = _row_major_2d(B, "B")
     ldc = _row_major_2d(C, "C")
     ws_ptr, ws_bytes = None, 0
     if workspace is not None:
-        ws_ptr, ws_bytes = ctypes.c_void_p(workspace.data_ptr()), workspace.numel() * workspace.element_size()
-    rc = lib.sfc_gemm_ex3(M, N, K, ctypes.c_void_p(A.data_ptr()), ctypes.c_void_p(B.data_ptr()),
-                          ctypes.c_void_p(C.data_ptr()), lda, ldb, ldc, ab, B_LAYOUTS[b_layout], float(beta), bias_ptr,
-                          int(ca_c), int(k_block_factor), SFC_F32 if C.dtype == torch.float32 else SFC_BF16,
-                          ORDERS[order], ASSIGNS[assign], TILES[tile], ws_ptr, ws_bytes, _stream_ptr(stream))
+        ws_ptr, ws_bytes = workspace.data_ptr(), workspace.numel() * workspace.element_size()
+    rc = lib.sfc_gemm_ex3(M, N, K, A.data_ptr(), B.data_ptr(), C.data_ptr(), lda, ldb, ldc, ab,
+                          B_LAYOUTS[b_layout], float(beta), bias_ptr, int(ca_c), int(k_block_factor),
+                          SFC_F32 if C.dtype == torch.float32 else SFC_BF16, ORDERS[order], ASSIGNS[assign],
+                          TILES[tile], ws_ptr, ws_bytes, _stream_ptr(stream))
     _check(rc, "sfc_gemm_ex3")
     return C
 
