@@ -328,6 +328,14 @@ def run_ours(args, rank, local, world):
         sfc.gemm(m["Ad"], m["Bd"], m["C"], ca_c=c, order=args.order, assign=args.assign, stream=stream,
                  b_layout=args.b_layout, k_block_factor=args.k_block_factor)
 
+    # the tensor cores' per-SM rate from resident operands (untimed), for the clock-based peak
+    mma_per_clk = None
+    if args.ab == "bf16":
+        try:
+            mma_per_clk = sfc.mma_peak(iters=2048, stream=stream)[0]
+        except Exception:
+            mma_per_clk = None
+
     # measure each shape's tiles (and layer counts where several are listed) once, untimed; the
     # timed calls below keep tile="auto", which then uses the measured choice (the tile never
     # changes the result's bits)
@@ -495,6 +503,13 @@ def run_ours(args, rank, local, world):
                     peaks["source"], "sustained" if sustained else "burst", elapsed_ms,
                     "" if args.ab == "bf16" else " x %.1f, the nominal 8-bit / bf16 ratio" % ratio),
                 "frac_of_burst_peak": round(achieved / burst, 4)}
+    if mma_per_clk and clock_info is not None and clock_info.get("sm_mhz"):
+        # the same kernel's ceiling at the clock the timed region actually ran at
+        at_clock = world_sms(torch) * mma_per_clk * clock_info["sm_mhz"] * 1e6 / 1e12
+        roofline["clock_peak"] = {"flop_per_clk_per_sm": round(mma_per_clk, 1),
+                                  "source": "sfc_mma_peak: back-to-back pair MMAs from resident operands",
+                                  "tflops_at_median_sm_clock": round(at_clock, 1),
+                                  "frac": round(achieved / at_clock, 4)}
     def launches_per_call(m):
         # GEMM launches (one per K block) plus the reduction when partials go through the workspace
         c = m["c"] if m["c"] else sfc.plan(m["s"]["M"], m["s"]["N"], m["s"]["K"], 0, out_dtype=m["C"].dtype,
@@ -734,6 +749,10 @@ def run_reference(args, rank, world):
                              "sample": sample},
             "e2e": {"value": round(value, 6), "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
             "gpu_launches": 0}
+
+
+def world_sms(torch):
+    return torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
 
 
 def run_sustained(args):

@@ -437,6 +437,22 @@ int sfc_gemm_host(int64_t M, int64_t N, int64_t K,
                   sfc_tile_t tile, int panels, void *stream);
 
 /*
+ * sfc_mma_peak -- the tensor cores' attainable rate on the current device:
+ * every co-schedulable 2-SM pair issues iters x 4 back-to-back 256 x 256 x 16
+ * bf16 MMAs (the GEMM's pair instruction) from zero-filled, resident shared
+ * memory into tensor memory, one CTA per SM.  The per-SM constant of the
+ * roofline the paper's performance model uses (Sec. III-B), measured.
+ *   flop_per_clk_per_sm: FLOP per SM clock cycle (clock64 around the issue
+ *                        loop up to the commit, slowest pair);
+ *   tflops:              the whole device's rate at the clock it ran at (CUDA
+ *                        events around the second of two launches).
+ * Synchronizes `stream`.  Errors: SFC_ERR_INVALID_ARG (iters outside
+ * 1..2^20 or a null output), SFC_ERR_UNSUPPORTED (not sm_103), SFC_ERR_TIMEOUT
+ * (the completion wait, bounded at 2 s, gave up), SFC_ERR_CUDA.
+ */
+int sfc_mma_peak(int iters, double *flop_per_clk_per_sm, double *tflops, void *stream);
+
+/*
  * sfc_debug_force_timeout -- test hook for the failure path: launches one GEMM
  * worker on a tiny problem whose MMA stage waits on a barrier that nothing
  * arrives at, with a wait limit of `limit_ms` milliseconds (1..1000).  The

@@ -53,7 +53,7 @@ EXPORTS = ("sfc_tile_order", "sfc_tile_order_device", "sfc_gemm_workspace_size",
            "sfc_get_device_status", "sfc_last_cuda_error", "sfc_num_workers", "sfc_debug_force_timeout",
            "sfc_gemm_noalloc", "sfc_gemm_plan", "sfc_release", "sfc_gemm_ex2", "sfc_gemm_host", "sfc_gemm_ex3",
            "sfc_gemm_workspace_size2", "sfc_gemm_tune", "sfc_gemm_tune_forget",
-           "sfc_gemm_tune_lookup")
+           "sfc_gemm_tune_lookup", "sfc_mma_peak")
 NOALLOC_SCRATCH_BYTES = 32 << 20
 
 
@@ -113,6 +113,7 @@ def load():
         lib.sfc_gemm_tune.argtypes = [i64, i64, i64, vp, vp, vp, i64, i64, i64, i32, i32, i32, i32, i32, vp, vp, vp, vp]
         lib.sfc_gemm_tune_forget.argtypes = []
         lib.sfc_gemm_tune_lookup.argtypes = [i32]
+        lib.sfc_mma_peak.argtypes = [i32, vp, vp, vp]
         lib.sfc_gemm_workspace_size2.restype = sz
         for name in EXPORTS:
             if name not in ("sfc_gemm_workspace_size", "sfc_gemm_workspace_size2"):
@@ -207,6 +208,14 @@ def tune_lookup(nearest: bool) -> None:
 def tune_forget() -> None:
     """Forget every tuned shape on the current device."""
     _check(load().sfc_gemm_tune_forget(), "sfc_gemm_tune_forget")
+
+
+def mma_peak(iters: int = 4096, stream=None):
+    """``(flop_per_clk_per_sm, tflops)``: the tensor cores' attainable rate
+    from resident operands (``sfc_mma_peak``)."""
+    f, t = ctypes.c_double(0.0), ctypes.c_double(0.0)
+    _check(load().sfc_mma_peak(int(iters), ctypes.byref(f), ctypes.byref(t), _stream_ptr(stream)), "sfc_mma_peak")
+    return f.value, t.value
 
 
 def release() -> None:

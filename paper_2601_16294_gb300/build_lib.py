@@ -15,7 +15,7 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(PKG, "libsfcgemm.so")
-SOURCES = [os.path.join(CSRC, "sfc_gemm.cu"), os.path.join(CSRC, "sfc_host.cpp")]
+SOURCES = [os.path.join(CSRC, "sfc_gemm.cu"), os.path.join(CSRC, "sfc_host.cpp"), os.path.join(CSRC, "sfc_peak.cu")]
 DEPS = SOURCES + [os.path.join(CSRC, f) for f in ("ptx.cuh", "sfc_curve.cuh", "sfc_gemm_kernel.cuh", "sfc_gemm_pair_kernel.cuh",
                                                       "sfc_internal.h")] + [
     os.path.join(INCLUDE, "sfc_gemm.h")]

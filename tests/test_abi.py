@@ -254,3 +254,10 @@ def test_tune_lookup_modes(lib):
     assert lib.sfc_gemm_tune_lookup(0) == binding.SFC_ERR_INVALID_ARG
     assert lib.sfc_gemm_tune_lookup(2) == binding.SFC_OK
     assert lib.sfc_gemm_tune_lookup(1) == binding.SFC_OK
+
+
+def test_mma_peak_validation(lib):
+    f, t = ctypes.c_double(0.0), ctypes.c_double(0.0)
+    assert lib.sfc_mma_peak(0, ctypes.byref(f), ctypes.byref(t), None) == binding.SFC_ERR_INVALID_ARG
+    assert lib.sfc_mma_peak((1 << 20) + 1, ctypes.byref(f), ctypes.byref(t), None) == binding.SFC_ERR_INVALID_ARG
+    assert lib.sfc_mma_peak(16, None, ctypes.byref(t), None) == binding.SFC_ERR_INVALID_ARG

@@ -35,6 +35,8 @@ def test_default_line_keys():
     r = d["roofline"]
     assert r["bound"] == "tensor" and r["unit"] == "TFLOP/s" and r["peak"] > 0
     assert abs(r["frac"] - r["achieved"] / r["peak"]) < 1e-3
+    cp = r["clock_peak"]                                    # the MMA-only ceiling at the sampled clock
+    assert 2000 < cp["flop_per_clk_per_sm"] < 20000 and 0 < cp["frac"] < 1.1
     e = d["e2e"]
     assert e["value"] > 0 and e["h2d_bytes_per_step"] == 2 * 2 * (2048 ** 2 + 4096 ** 2)   # A and B, bf16
     assert e["d2h_bytes_per_step"] == 2 * (2048 ** 2 + 4096 ** 2)
