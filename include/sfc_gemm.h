@@ -30,8 +30,9 @@
  *     validation error launches nothing;
  *   - every function returns an sfc_status_t (0 = success) unless noted.
  *
- * Thread safety: entry points may be called from several host threads; each
- * call only reads immutable library state after a one-time per-device set-up.
+ * Thread safety: entry points may be called from several host threads; after
+ * a one-time per-device set-up the state calls share is either immutable or
+ * guarded (the table of tuned shapes, the staging slots of sfc_gemm_host).
  */
 #ifndef SFC_GEMM_H
 #define SFC_GEMM_H
@@ -265,9 +266,11 @@ size_t sfc_gemm_workspace_size2(int64_t M, int64_t N, int64_t K, int ca_c, int k
  * fastest (the paper's first way to configure a shape: benchmark the small
  * space of knobs exhaustively, Sec. III-C).  For each layer count in 1, 2, 4,
  * ... up to max_layers (and the time model's own choice) every tile shape is
- * timed (one warm-up call, then the mean of three, CUDA events on `stream`);
- * then K blocks 2, 4, ... up to max_kbf are timed on the fastest (tile,
- * layers).  The results go into a per-device table for this (M, N, K,
+ * timed (one warm-up call, then the mean of five, CUDA events on `stream`);
+ * then K blocks 2, 4, ... up to max_kbf are timed on the chosen (tile,
+ * layers).  A measured alternative replaces the time model's tile, layer
+ * count or single K block only when it is at least 3 % faster, so that
+ * candidates within timing noise keep the model's pick.  The results go into a per-device table for this (M, N, K,
  * ab_dtype, b_layout, c_dtype): afterwards calls with tile = SFC_TILE_AUTO and
  * k_block_factor = 1 use the fastest tile measured for their layer count, and
  * with ca_c = 0 also the fastest layer count (sfc_gemm_plan reports the

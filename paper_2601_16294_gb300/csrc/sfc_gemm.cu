@@ -28,7 +28,21 @@ thread_local int t_last_cuda_error = 0;
 
 int cuda_fail(cudaError_t e) {
     t_last_cuda_error = static_cast<int>(e);
+    // the runtime also keeps the error as the thread's last error; the status code reports it, so
+    // clear it (a non-sticky error left there would read as the failure of a later, good launch)
+    (void)cudaGetLastError();
     return SFC_ERR_CUDA;
+}
+
+// Launches check the error cudaLaunchKernelEx returns, never cudaGetLastError (which could hold
+// an earlier, unrelated failure of the caller's).
+template <typename... Params, typename... Args>
+cudaError_t launch_plain(void (*kernel)(Params...), unsigned grid, unsigned block, cudaStream_t s, Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid, 1, 1);
+    cfg.blockDim = dim3(block, 1, 1);
+    cfg.stream = s;
+    return cudaLaunchKernelEx(&cfg, kernel, args...);
 }
 
 namespace {
@@ -415,7 +429,7 @@ cudaError_t launch_gemm(int v, bool f8, const CUtensorMap& ta, const CUtensorMap
     cudaLaunchConfig_t cfg = launch_config(v, grid, s, attr, true);
     cudaError_t e = cudaLaunchKernelEx(&cfg, f8 ? Kernels<OutT, true>::get(v) : Kernels<OutT, false>::get(v), ta, tb,
                                        tc, p);
-    return e != cudaSuccess ? e : cudaGetLastError();
+    return e;
 }
 
 // ------------------------------------------------------------ tuning table
@@ -509,9 +523,9 @@ int pack_operands(const DeviceInfo* dev, int ab, int b_layout, int64_t M, int64_
         if (e != cudaSuccess) return cuda_fail(e);
         int64_t blocks = ceil_div(rows * cols, 256);
         if (blocks > static_cast<int64_t>(dev->num_sms) * 16) blocks = static_cast<int64_t>(dev->num_sms) * 16;
-        pack_rows_kernel<<<static_cast<unsigned>(blocks), 256, 0, stream>>>(
-            static_cast<const uint8_t*>(*ptr), *ld, rows, cols, eb, static_cast<uint8_t*>(packed[which]), ld_dst);
-        e = cudaGetLastError();
+        e = launch_plain(pack_rows_kernel, static_cast<unsigned>(blocks), 256, stream,
+                         static_cast<const uint8_t*>(*ptr), *ld, rows, cols, eb, static_cast<uint8_t*>(packed[which]),
+                         ld_dst);
         if (e != cudaSuccess) return cuda_fail(e);
         *ptr = packed[which];
         *ld = ld_dst;
@@ -550,7 +564,7 @@ cudaError_t launch_reduce(const DeviceInfo* dev, const float* ws, int64_t ldo, i
     else
         e = cudaLaunchKernelEx(&cfg, ca_reduce_kernel<__nv_bfloat16>, ws, ldo, layer_stride, layers, M, N,
                                static_cast<__nv_bfloat16*>(C), ldc, vec, beta, bias);
-    return e == cudaSuccess ? cudaGetLastError() : e;
+    return e;
 }
 
 int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void* C, int64_t lda, int64_t ldb,
@@ -762,9 +776,8 @@ SFC_API int sfc_tile_order_device(int Mt, int Nt, int32_t* out_idx_dev, void* st
     if (rc != SFC_OK) return rc;
     int64_t blocks = (n + 255) / 256;
     if (blocks > 65535) blocks = 65535;
-    tile_order_kernel<<<static_cast<int>(blocks), 256, 0, static_cast<cudaStream_t>(stream)>>>(Mt, Nt,
-                                                                                              out_idx_dev);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_plain(tile_order_kernel, static_cast<unsigned>(blocks), 256,
+                                 static_cast<cudaStream_t>(stream), Mt, Nt, out_idx_dev);
     return e == cudaSuccess ? SFC_OK : cuda_fail(e);
 }
 
@@ -903,49 +916,65 @@ SFC_API int sfc_gemm_tune(int64_t M, int64_t N, int64_t K, const void* A, const 
         return run_gemm(M, N, K, A, B, C, lda, ldb, ldc, c, c_dtype, SFC_ORDER_SFC, SFC_ASSIGN_AUTO, tile, nullptr,
                         0, s, 0, kDefaultTimeoutNs, b_layout, 0.0f, nullptr, ab_dtype, true, kbf);
     };
-    // one call to warm up, then the mean of three
+    // one call to warm up, then the mean of kReps
+    constexpr int kReps = 5;
     auto measure = [&](int c, int tile, int kbf, float* us) {
         int r = call(c, tile, kbf);
         cudaError_t ce = cudaSuccess;
         if (r == SFC_OK) ce = cudaEventRecord(e0, s);
-        for (int i = 0; i < 3 && r == SFC_OK && ce == cudaSuccess; ++i) r = call(c, tile, kbf);
+        for (int i = 0; i < kReps && r == SFC_OK && ce == cudaSuccess; ++i) r = call(c, tile, kbf);
         if (r == SFC_OK && ce == cudaSuccess) ce = cudaEventRecord(e1, s);
         if (r == SFC_OK && ce == cudaSuccess) ce = cudaEventSynchronize(e1);
         float ms = 0.0f;
         if (r == SFC_OK && ce == cudaSuccess) ce = cudaEventElapsedTime(&ms, e0, e1);
         if (r == SFC_OK && ce != cudaSuccess) r = cuda_fail(ce);
-        *us = ms * 1000.0f / 3.0f;
+        *us = ms * 1000.0f / static_cast<float>(kReps);
         return r;
     };
+    // A measured alternative replaces the time model's choice only when it is clearly faster:
+    // candidates within timing noise of each other keep the model's (steadier) pick.
+    constexpr float kMargin = 0.97f;
 
     TuneEntry entry;
     std::memset(&entry, 0, sizeof(entry));
-    float best = -1.0f;
+    float best = -1.0f;            // the fastest configuration so far
+    float model_us = -1.0f;        // the time model's layer count, with its measured tile
     for (int c : counts) {
-        float best_c = -1.0f;
+        const int model_v = make_plan(M, N, K, c, c, *dev, SFC_TILE_AUTO, c_dtype == SFC_F32 ? 4 : 2, b_kmajor,
+                                      ab_dtype).v;
+        float t[kNumVariants];
+        for (int v = 0; v < kNumVariants; ++v) t[v] = -1.0f;
         for (int v = 0; v < kNumVariants && rc == SFC_OK; ++v) {
             if (dev->workers[v] <= 0 || !variant_allowed(v, b_kmajor, ab_dtype)) continue;
-            float us = 0.0f;
-            rc = measure(c, kTileOf[v], 1, &us);
-            if (rc != SFC_OK) break;
-            if (best_c < 0.0f || us < best_c) {
-                best_c = us;
-                entry.tile_for_c[c] = kTileOf[v];
-            }
-            if (best < 0.0f || us < best) {
-                best = us;
-                entry.tile = kTileOf[v];
-                entry.c = c;
-                entry.kbf = 1;
-            }
+            rc = measure(c, kTileOf[v], 1, &t[v]);
         }
         if (rc != SFC_OK) break;
+        int pick = (t[model_v] >= 0.0f) ? model_v : -1;
+        for (int v = 0; v < kNumVariants; ++v) {
+            if (t[v] < 0.0f) continue;
+            if (pick < 0 || t[v] < t[pick] * kMargin) pick = v;
+        }
+        entry.tile_for_c[c] = kTileOf[pick];
+        if (c == model.c) model_us = t[pick];
+        if (best < 0.0f || t[pick] < best) {
+            best = t[pick];
+            entry.tile = kTileOf[pick];
+            entry.c = c;
+            entry.kbf = 1;
+        }
     }
-    // K blocks on the fastest (tile, layers)
-    for (int kbf = 2; rc == SFC_OK && kbf <= max_kbf && Kt / entry.c >= kbf; kbf *= 2) {
+    // the model's layer count stays unless another is clearly faster
+    if (rc == SFC_OK && model_us >= 0.0f && best > model_us * kMargin && entry.tile_for_c[model.c] != 0) {
+        best = model_us;
+        entry.tile = entry.tile_for_c[model.c];
+        entry.c = model.c;
+    }
+    // K blocks on the chosen (tile, layers), taken only when clearly faster
+    const int base_kbf_c = entry.c;
+    for (int kbf = 2; rc == SFC_OK && kbf <= max_kbf && Kt / base_kbf_c >= kbf; kbf *= 2) {
         float us = 0.0f;
         rc = measure(entry.c, entry.tile, kbf, &us);
-        if (rc == SFC_OK && us < best) {
+        if (rc == SFC_OK && us < best * kMargin) {
             best = us;
             entry.kbf = kbf;
         }

@@ -140,7 +140,6 @@ SFC_API int sfc_mma_peak(int iters, double* flop_per_clk_per_sm, double* tflops,
         if (rep == 1) e = cudaEventRecord(e0, s);
         if (e == cudaSuccess)
             e = cudaLaunchKernelEx(&cfg, mma_peak_kernel, iters, static_cast<uint64_t>(2000000000ull), d_cycles);
-        if (e == cudaSuccess) e = cudaGetLastError();
     }
     if (e == cudaSuccess) e = cudaEventRecord(e1, s);
     std::vector<unsigned long long> cyc(static_cast<size_t>(clusters), 0ull);
