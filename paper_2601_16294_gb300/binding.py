@@ -32,6 +32,15 @@ B_LAYOUTS = {"kn": 0, "nk": 1}
 
 
 _AB_CODES = None
+_torch = None
+
+
+def _import_torch():
+    """torch, imported on first use (the curve functions work without it)."""
+    global _torch
+    import torch
+    _torch = torch
+    return torch
 
 
 def _ab_code(dtype) -> int:
@@ -232,9 +241,10 @@ def num_workers() -> int:
 
 
 def _row_major_2d(t, name):
-    if t.dim() != 2 or t.stride(1) != 1:
+    st = t.stride()
+    if len(st) != 2 or st[1] != 1:
         raise ValueError("%s must be a 2-D row-major (unit column stride) tensor" % name)
-    return t.stride(0)
+    return st[0]
 
 
 def gemm(A, B, C=None, *, ca_c: int = 1, out_dtype=None, order: str = "sfc", assign: str = "auto",
@@ -250,8 +260,8 @@ def gemm(A, B, C=None, *, ca_c: int = 1, out_dtype=None, order: str = "sfc", ass
     summed into C (or the layer copies) in place.  ``workspace``: optional CUDA
     tensor of at least ``workspace_size(M, N, K, ca_c, k_block_factor,
     out_dtype)`` bytes."""
-    import torch
     lib = _lib or load()
+    torch = _torch or _import_torch()
     M, K = A.shape
     if b_layout == "kn":
         K2, N = B.shape
@@ -261,14 +271,22 @@ def gemm(A, B, C=None, *, ca_c: int = 1, out_dtype=None, order: str = "sfc", ass
         raise ValueError("b_layout must be 'kn' or 'nk'")
     if K != K2:
         raise ValueError("inner dimensions differ: %d vs %d" % (K, K2))
-    if A.dtype != B.dtype:
+    a_dtype = A.dtype
+    if a_dtype != B.dtype:
         raise TypeError("A and B must have the same dtype")
-    ab = _ab_code(A.dtype)
+    ab = _ab_code(a_dtype)
     if C is None:
         if beta != 0.0:
             raise ValueError("beta != 0 needs an input C")
         C = torch.empty((M, N), dtype=out_dtype or torch.float32, device=A.device)
-    if C.dtype not in (torch.float32, torch.bfloat16) or tuple(C.shape) != (M, N):
+    c_dtype = C.dtype
+    if c_dtype == torch.float32:
+        c_code = SFC_F32
+    elif c_dtype == torch.bfloat16:
+        c_code = SFC_BF16
+    else:
+        c_code = -1
+    if c_code < 0 or C.shape != (M, N):
         raise ValueError("C must be (M, N) float32 or bfloat16")
     bias_ptr = None
     if bias is not None:
@@ -282,10 +300,11 @@ def gemm(A, B, C=None, *, ca_c: int = 1, out_dtype=None, order: str = "sfc", ass
     if workspace is not None:
         ws_ptr, ws_bytes = workspace.data_ptr(), workspace.numel() * workspace.element_size()
     rc = lib.sfc_gemm_ex3(M, N, K, A.data_ptr(), B.data_ptr(), C.data_ptr(), lda, ldb, ldc, ab,
-                          B_LAYOUTS[b_layout], float(beta), bias_ptr, int(ca_c), int(k_block_factor),
-                          SFC_F32 if C.dtype == torch.float32 else SFC_BF16, ORDERS[order], ASSIGNS[assign],
-                          TILES[tile], ws_ptr, ws_bytes, _stream_ptr(stream))
-    _check(rc, "sfc_gemm_ex3")
+                          B_LAYOUTS[b_layout], beta, bias_ptr, ca_c, k_block_factor, c_code, ORDERS[order],
+                          ASSIGNS[assign], TILES[tile], ws_ptr, ws_bytes,
+                          (stream if stream is not None else torch.cuda.current_stream()).cuda_stream)
+    if rc != SFC_OK:
+        _check(rc, "sfc_gemm_ex3")
     return C
 
 
