@@ -696,19 +696,33 @@ def oracle_sample(mats_cpu, rows):
     return flops, t
 
 
-def run_cpu_baseline(mats):
+def run_cpu_baseline(mats, budget_s=12.0, one_core_s=4.0):
     """The oracle as it stands, on this host's cores, on a bounded sample of the
-    workload: a 16-row probe sets the row count for about 12 s of CPU work."""
+    workload: a 16-row probe sets the row count for about ``budget_s`` of CPU
+    work.  Then the same oracle on one core, for about ``one_core_s``."""
+    from oracle import oracle
     os.environ.setdefault("OMP_NUM_THREADS", str(cpu_cores()))
+    cores = int(os.environ["OMP_NUM_THREADS"])
+    oracle.set_threads(cores)
     mats_cpu = [(m["A"], m["B"]) for m in mats]
     _, s_probe = oracle_sample(mats_cpu, 16)
-    rows = int(min(1024, max(16, 16 * 12.0 / max(s_probe, 1e-3))))
+    rows = int(min(1024, max(16, 16 * budget_s / max(s_probe, 1e-3))))
     rows = max(16, rows // 16 * 16)
     flops, secs = oracle_sample(mats_cpu, rows)
+    # one core, on fewer rows: the all-core rate times the core count predicts the time
+    rows1 = int(max(2, min(rows, rows * one_core_s / max(secs * cores, 1e-6))))
+    oracle.set_threads(1)
+    try:
+        flops1, secs1 = oracle_sample(mats_cpu, rows1)
+    finally:
+        oracle.set_threads(cores)
     return {"value": round(flops / secs / 1e12, 6), "unit": "TFLOP/s",
-            "cores": int(os.environ["OMP_NUM_THREADS"]), "kind": "oracle", "seconds": round(secs, 2),
+            "cores": cores, "kind": "oracle", "seconds": round(secs, 2),
             "sample": "%d evenly spaced rows of C for each shape (fp64 triple loop, OpenMP over rows)"
-                      % rows}
+                      % rows,
+            "one_core": {"value": round(flops1 / secs1 / 1e12, 6), "unit": "TFLOP/s", "cores": 1,
+                         "seconds": round(secs1, 2),
+                         "sample": "%d evenly spaced rows of C for each shape" % rows1}}
 
 
 # ------------------------------------------------------------- reference arm

@@ -57,6 +57,7 @@
  *  single step, used to compare bf16 outputs against the fp64 reference.
  */
 #include <math.h>
+#include <omp.h>
 #include <stdint.h>
 #include <string.h>
 
@@ -310,3 +311,13 @@ void oracle_round_bf16_array(const double *v, int64_t n, uint16_t *out)
     #pragma omp parallel for schedule(static)
     for (int64_t i = 0; i < n; ++i) out[i] = oracle_round_bf16(v[i]);
 }
+
+/* Thread count of the parallel loops above, for timing the oracle on a given
+ * number of host cores (no arithmetic: every row is computed the same way). */
+void oracle_set_threads(int n)
+{
+    if (n > 0)
+        omp_set_num_threads(n);
+}
+
+int oracle_max_threads(void) { return omp_get_max_threads(); }

@@ -14,6 +14,8 @@ What the oracle computes, and the passage each part follows:
 * ``gemm_sub_f64(A, B, rows, cols, k0, k1)`` -- selected rows/columns, optionally
   one K range (one layer's partial product of the K split, Sec. II-C/D).
 * ``round_bf16(x)`` -- one-step round-to-nearest-even of doubles to bf16.
+* ``set_threads(n)`` / ``max_threads()`` -- the OpenMP thread count of the loops
+  (for timing on a chosen number of host cores; no arithmetic).
 """
 from __future__ import annotations
 
@@ -72,6 +74,10 @@ def _load():
         lib.oracle_round_bf16.restype = ctypes.c_uint16
         lib.oracle_round_bf16_array.argtypes = [ctypes.c_void_p, i64, ctypes.c_void_p]
         lib.oracle_round_bf16_array.restype = None
+        lib.oracle_set_threads.argtypes = [ctypes.c_int]
+        lib.oracle_set_threads.restype = None
+        lib.oracle_max_threads.argtypes = []
+        lib.oracle_max_threads.restype = ctypes.c_int
         _lib = lib
         return lib
 
@@ -215,3 +221,13 @@ def round_bf16(x) -> np.ndarray:
     """Round doubles to bf16 (nearest, ties to even), returned as float64 values."""
     bits = round_bf16_bits(x)
     return (bits.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+
+
+def set_threads(n: int) -> None:
+    """Run the oracle's parallel loops on ``n`` host threads from now on."""
+    _load().oracle_set_threads(int(n))
+
+
+def max_threads() -> int:
+    """Threads the oracle's next parallel loop will use."""
+    return int(_load().oracle_max_threads())

@@ -43,6 +43,7 @@ def test_default_line_keys():
     assert d["gpu_launches"] == 3 * 2                                    # one GEMM launch per shape per step
     c = d["cpu_baseline"]
     assert c["kind"] == "oracle" and c["cores"] >= 1 and c["value"] > 0
+    assert c["one_core"]["cores"] == 1 and c["one_core"]["value"] > 0
     assert {"sm_mhz", "sm_max_mhz", "reasons"} <= set(d["clocks"])
     assert len(d["per_shape"]) == 2 and all(p["tile"] for p in d["per_shape"])
 
