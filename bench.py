@@ -175,6 +175,18 @@ def roofline_time_s(s, peaks, ab="bf16"):
     return max(t_tc, t_hbm), ("tensor" if t_tc >= t_hbm else "hbm")
 
 
+def method_roofline_time_s(s, peaks, c, ab="bf16"):
+    """roofline_time_s with the K split's own traffic counted: c > 1 fp32 copies
+    of C written and read back by the final reduction (Sec. II-C, Listing 1)."""
+    t, _ = roofline_time_s(s, peaks, ab)
+    if c <= 1:
+        return t
+    o = 4 if s["out"] == "f32" else 2
+    ib = 2 if ab == "bf16" else 1
+    bytes_method = ib * (s["M"] * s["K"] + s["K"] * s["N"]) + o * s["M"] * s["N"] + 8.0 * c * s["M"] * s["N"]
+    return max(t, bytes_method / (peaks["hbm_gbs"] * 1e9))
+
+
 # ------------------------------------------------------------------ distributed
 
 def dist_setup(n_gpus):
@@ -467,7 +479,7 @@ def run_ours(args, rank, local, world):
         flops = 2.0 * s["M"] * s["N"] * s["K"]
         t_roof, bound = roofline_time_s(s, peaks, args.ab)
         row = {"M": s["M"], "N": s["N"], "K": s["K"], "out": s["out"], "ca_c": m["c"],
-               "ms_mean": round(mean, 4), "ms_min": round(min(ts), 4),
+               "ms_mean": round(mean, 4), "ms_median": round(statistics.median(ts), 4), "ms_min": round(min(ts), 4),
                "tflops": round(flops / (mean * 1e-3) / 1e12, 1), "bound": bound,
                "frac_of_roofline": round(t_roof / (mean * 1e-3), 4),
                "ms_back_to_back": round(b2b_ms[i], 4),
@@ -475,8 +487,12 @@ def run_ours(args, rank, local, world):
                "frac_of_roofline_back_to_back": round(t_roof / (b2b_ms[i] * 1e-3), 4)}
         if i in cs_report:
             row["ms_by_ca_c"] = cs_report[i]
-        row["tile"] = sfc.plan(s["M"], s["N"], s["K"], m["c"], out_dtype=m["C"].dtype, in_dtype=m["Ad"].dtype,
-                               b_layout=args.b_layout)[0]
+        tile, c_eff = sfc.plan(s["M"], s["N"], s["K"], m["c"], out_dtype=m["C"].dtype, in_dtype=m["Ad"].dtype,
+                               b_layout=args.b_layout)
+        row["tile"] = tile
+        if c_eff > 1:
+            # the method's roofline: the layer partials' traffic counted too
+            row["frac_of_method_roofline"] = round(method_roofline_time_s(s, peaks, c_eff, args.ab) / (mean * 1e-3), 4)
         per_shape.append(row)
 
     # roofline of the dominant kernel (the GEMM kernel; the K-layer reduction,

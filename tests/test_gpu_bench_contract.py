@@ -46,4 +46,5 @@ def test_default_line_keys():
     assert c["one_core"]["cores"] == 1 and c["one_core"]["value"] > 0
     assert {"sm_mhz", "sm_max_mhz", "reasons"} <= set(d["clocks"])
     assert len(d["per_shape"]) == 2 and all(p["tile"] for p in d["per_shape"])
+    assert all(p["ms_min"] <= p["ms_median"] for p in d["per_shape"])
 
