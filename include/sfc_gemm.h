@@ -33,6 +33,12 @@
  * Thread safety: entry points may be called from several host threads; after
  * a one-time per-device set-up the state calls share is either immutable or
  * guarded (the table of tuned shapes, the staging slots of sfc_gemm_host).
+ * Kernels in flight at the same time -- on several streams, or replays of
+ * captured graphs -- share no device state but the error word that
+ * sfc_get_device_status reads: the counter from which a call's workers take
+ * their items (SFC_ASSIGN_WAVE / AUTO) is memory of that call, taken from a
+ * stream-ordered pool of the library and freed after the call's kernels
+ * (sfc_gemm_noalloc: its scratch area).
  */
 #ifndef SFC_GEMM_H
 #define SFC_GEMM_H
@@ -96,8 +102,6 @@ typedef enum {
  * N128 / N256:           128 x 128 / 128 x 256 tiles, one SM each.
  * PAIR_N128 / PAIR_N256: 256 x 128 / 256 x 256 tiles computed by a pair of SMs
  *                        (a 2-CTA cluster; each SM loads half of A and half of B).
- * QUAD_N256:             512 x 256 tiles computed by two such pairs (a 4-CTA
- *                        cluster) that share the B slab by TMA multicast.
  * AUTO: the tile sfc_gemm_tune measured fastest for the shape (and layer
  * count), else the time model's pick from the tile count and the number of
  * workers.  Every tile shape gives the same bits. */
@@ -106,8 +110,7 @@ typedef enum {
     SFC_TILE_N128 = 128,
     SFC_TILE_N256 = 256,
     SFC_TILE_PAIR_N128 = 1128,
-    SFC_TILE_PAIR_N256 = 1256,
-    SFC_TILE_QUAD_N256 = 2256
+    SFC_TILE_PAIR_N256 = 1256
 } sfc_tile_t;
 
 /*
@@ -165,9 +168,9 @@ size_t sfc_gemm_workspace_size(int64_t M, int64_t N, int64_t K, int ca_c);
  * Accuracy: products are exact and summed in fp32; the tensor core's running
  * sum is restarted every 4096 values of k and the partial sums are added with
  * round-to-nearest fp32 adds, which bounds the error growth of very long K.
- * (Experiments only: the environment variable SFC_GEMM_CHUNK_SLABS, read once
- * per device, sets that restart interval in units of 64 values of k; 0 turns
- * the restarts off.)
+ * Memory: besides the layer workspace, a call with dynamic dealing takes a
+ * 256-byte counter from the library's stream-ordered ticket pool and frees it
+ * after its kernels (both kept by the pools for the next call).
  * Errors: SFC_ERR_INVALID_ARG, SFC_ERR_UNALIGNED, SFC_ERR_CUDA, SFC_ERR_UNSUPPORTED.
  */
 int sfc_gemm(int64_t M, int64_t N, int64_t K,
@@ -203,8 +206,7 @@ int sfc_gemm_ex(int64_t M, int64_t N, int64_t K,
  *             128 values of k, and the N-major (SFC_B_KN) layout is not served
  *             by SFC_TILE_PAIR_N128 (SFC_TILE_N128 is used instead).
  *   b_layout: SFC_B_KN (B is K x N, ldb >= N) or SFC_B_NK (B is stored as its
- *             transpose, N x K, ldb >= K).  SFC_TILE_QUAD_N256 is served by
- *             SFC_TILE_PAIR_N256 with SFC_B_NK.
+ *             transpose, N x K, ldb >= K).
  *   beta:     0 leaves C write-only (its contents may be anything, even NaN);
  *             otherwise C is read once, before it is written.
  *   bias:     NULL or N fp32 device values, 4-byte aligned, added per column.
@@ -319,12 +321,40 @@ int sfc_gemm_tune_lookup(int mode);
 int sfc_gemm_plan(int64_t M, int64_t N, int64_t K, int ca_c, int c_dtype, int tile,
                   int ab_dtype, int b_layout, int *out_tile, int *out_ca_c);
 
+/* A device as the time model sees it (sfc_gemm_plan_desc). */
+typedef struct {
+    int num_sms;       /* SMs: workers of the one-SM tiles (GB300: 152) */
+    int pair_workers;  /* 2-SM pairs that can be resident at once (GB300: 76) */
+    double hbm_gbs;    /* attainable DRAM bandwidth, GB/s (GB300: about 6700 for a copy) */
+    double sm_ghz;     /* SM clock the tensor cores' rate is taken at */
+} sfc_device_desc_t;
+
+/*
+ * sfc_gemm_plan_desc -- the library's time model alone, on a described device
+ * (no GPU needed; tuned shapes are not consulted).  For C = A B of these sizes
+ * and types it returns the tile and K-layer count the model picks (ca_c = 0:
+ * any count up to the limit sfc_gemm_workspace_size assumes; ca_c >= 1: that
+ * count) and the time it predicts, in ns.  The model follows Sec. III-B's
+ * roofline per BRGEMM, T = max(G gamma, beta (S_A + S_B)) (Eqs. 1-4), at two
+ * levels: per worker, a 64-deep slab of a tile costs the longer of its MMA time
+ * and its operand intake (folded into each tile's measured efficiency), over
+ * waves = ceil(tiles * layers / workers) waves of the longest layer's slabs;
+ * per launch, at least the DRAM bytes (A and B once, C or the layers' fp32
+ * partials) at hbm_gbs; for more than one layer the reduction adds its launch
+ * and the partials read back.
+ * Errors: SFC_ERR_INVALID_ARG (as sfc_gemm_plan, a NULL pointer, or a device
+ * with num_sms < 1, pair_workers < 0 or > num_sms / 2, hbm_gbs or sm_ghz <= 0).
+ */
+int sfc_gemm_plan_desc(const sfc_device_desc_t *desc, int64_t M, int64_t N, int64_t K, int ca_c,
+                       int c_dtype, int ab_dtype, int b_layout, int *out_tile, int *out_ca_c,
+                       double *out_ns);
+
 /*
  * sfc_release -- returns to the driver the device memory the library holds
  * between calls on the current device: the staging slots of sfc_gemm_host and
- * what its stream-ordered pool keeps after K-layer workspaces and repacked
- * operands were freed (synchronizes the device first).  SFC_OK, SFC_ERR_CUDA
- * or SFC_ERR_UNSUPPORTED.
+ * what its stream-ordered pools keep after K-layer workspaces, repacked
+ * operands and ticket counters were freed (synchronizes the device first).
+ * SFC_OK, SFC_ERR_CUDA or SFC_ERR_UNSUPPORTED.
  */
 int sfc_release(void);
 
@@ -332,7 +362,11 @@ int sfc_release(void);
  * sfc_get_device_status -- synchronizes `stream`, then returns and clears the
  * device error word that kernels set when a bounded wait gives up
  * (SFC_ERR_TIMEOUT), or SFC_ERR_CUDA if the synchronization itself failed.
- * SFC_OK if no kernel reported a problem since the last call.
+ * SFC_OK if no kernel reported a problem since the last call.  The word is
+ * one per device: a kernel on any stream may have set it, and the first
+ * caller to read it after that gets the report.  Only the bits read are
+ * cleared (atomically, by a kernel on `stream`), so a report that another
+ * stream's kernel makes meanwhile is kept for the next call.
  */
 int sfc_get_device_status(void *stream);
 
@@ -352,22 +386,28 @@ int sfc_num_workers(void);
  * running inside a framework that owns every device allocation, a real-time
  * path where an allocation may block or fail, or a process that has already
  * handed all device memory to its own arena.  For them this entry point takes
- * the fp32 partial copies of C (ca_c > 1) from a fixed scratch area compiled
- * into the library, SFC_NOALLOC_SCRATCH_BYTES bytes of device memory that
+ * the fp32 partial copies of C (ca_c > 1) and the workers' item counter from a
+ * fixed scratch area compiled into the library: SFC_NOALLOC_SCRATCH_BYTES
+ * bytes for the partials plus 256 bytes for the counter, device memory that
  * every GPU which loads the library holds until the process exits.  It calls
- * no cudaMalloc, cudaFree or allocating library routine.
+ * no cudaMalloc, cudaFree or allocating library routine, and takes nothing
+ * from the library's pools.
  *
  *   Arguments as sfc_gemm_ex with order = SFC, assign and tile = AUTO.
- *   Errors: SFC_ERR_WORKSPACE (nothing launched) when
- *           sfc_gemm_workspace_size(M, N, K, ca_c) > SFC_NOALLOC_SCRATCH_BYTES;
+ *   ca_c:   >= 1: that many layers; their partials, ca_c * M * round_up(N, 4)
+ *           * 4 bytes when ca_c > 1, must fit in SFC_NOALLOC_SCRATCH_BYTES.
+ *           0: the library's layer count, limited to what fits.
+ *   Errors: SFC_ERR_WORKSPACE (nothing launched) when ca_c >= 2 and the
+ *           partials exceed SFC_NOALLOC_SCRATCH_BYTES;
  *           SFC_ERR_UNALIGNED when A or B would need repacking (a base not
  *           16-byte aligned or lda / ldb not a multiple of 8), since that
  *           takes memory; otherwise as sfc_gemm_ex.
  * The first call on each device looks up the scratch area's device address
- * (once per device, with that device current); make that first call before
- * any stream capture.  All calls share the one scratch area and leave their
- * partials in it: calls whose kernels can overlap on the GPU (different
- * streams without ordering between them) race on it, so order them.
+ * (with that device current; a lookup that fails is retried by the next
+ * call), so make a first call before any stream capture.  All calls share
+ * the one scratch area and leave their partials in it: calls whose kernels
+ * can overlap on the GPU (different streams without ordering between them)
+ * race on it, so order them.
  */
 #define SFC_NOALLOC_SCRATCH_BYTES ((size_t)32 << 20)
 int sfc_gemm_noalloc(int64_t M, int64_t N, int64_t K,
@@ -387,7 +427,7 @@ int sfc_gemm_noalloc(int64_t M, int64_t N, int64_t K,
  * upload is followed by the GEMM of the strip of C it completes, so GEMMs
  * start after two panels have arrived and finished strips of C go back while
  * later strips compute.  Panel edges fall on multiples of 512 rows or 256
- * columns (the largest output tiles), so the result is bit-identical to
+ * columns (multiples of every output tile), so the result is bit-identical to
  * sfc_gemm_ex2 over the whole problem with the tile and ca_c that
  * sfc_gemm_plan(M, N, K, ca_c, c_dtype, tile, ab_dtype, b_layout, ...)
  * reports, which every strip uses.
@@ -454,6 +494,20 @@ int sfc_gemm_host(int64_t M, int64_t N, int64_t K,
  * (the completion wait, bounded at 2 s, gave up), SFC_ERR_CUDA.
  */
 int sfc_mma_peak(int iters, double *flop_per_clk_per_sm, double *tflops, void *stream);
+
+/*
+ * sfc_debug_pool_used_high -- the high-water mark, in bytes, of the memory in
+ * use from the library's stream-ordered pools on the current device (layer
+ * workspaces, repacked operands, ticket counters) since the last reset; with
+ * reset = 1 the mark is read and then reset, so the next reading covers only
+ * what is used after this call.  A
+ * diagnostic with no counterpart in the paper (the tests use it to show that
+ * sfc_gemm_noalloc takes nothing from the pools).  Does not synchronize: read
+ * it after the calls of interest have completed.
+ * Errors: SFC_ERR_INVALID_ARG (NULL output, reset not 0 or 1), SFC_ERR_CUDA,
+ * SFC_ERR_UNSUPPORTED.
+ */
+int sfc_debug_pool_used_high(size_t *used_high_bytes, int reset);
 
 /*
  * sfc_debug_force_timeout -- test hook for the failure path: launches one GEMM

@@ -27,7 +27,7 @@ _NAMES = {0: "SFC_OK", -1: "SFC_ERR_INVALID_ARG", -2: "SFC_ERR_UNALIGNED", -3: "
 SFC_F32, SFC_BF16 = 0, 1
 ORDERS = {"sfc": 0, "raster": 1}
 ASSIGNS = {"segment": 0, "wave": 1, "auto": 2, "wave_static": 3}
-TILES = {0: 0, "auto": 0, 128: 128, 256: 256, "pair128": 1128, "pair256": 1256, "quad256": 2256}
+TILES = {0: 0, "auto": 0, 128: 128, 256: 256, "pair128": 1128, "pair256": 1256}
 B_LAYOUTS = {"kn": 0, "nk": 1}
 
 
@@ -62,7 +62,7 @@ EXPORTS = ("sfc_tile_order", "sfc_tile_order_device", "sfc_gemm_workspace_size",
            "sfc_get_device_status", "sfc_last_cuda_error", "sfc_num_workers", "sfc_debug_force_timeout",
            "sfc_gemm_noalloc", "sfc_gemm_plan", "sfc_release", "sfc_gemm_ex2", "sfc_gemm_host", "sfc_gemm_ex3",
            "sfc_gemm_workspace_size2", "sfc_gemm_tune", "sfc_gemm_tune_forget",
-           "sfc_gemm_tune_lookup", "sfc_mma_peak")
+           "sfc_gemm_tune_lookup", "sfc_mma_peak", "sfc_debug_pool_used_high", "sfc_gemm_plan_desc")
 NOALLOC_SCRATCH_BYTES = 32 << 20
 
 
@@ -123,6 +123,8 @@ def load():
         lib.sfc_gemm_tune_forget.argtypes = []
         lib.sfc_gemm_tune_lookup.argtypes = [i32]
         lib.sfc_mma_peak.argtypes = [i32, vp, vp, vp]
+        lib.sfc_debug_pool_used_high.argtypes = [vp, i32]
+        lib.sfc_gemm_plan_desc.argtypes = [vp, i64, i64, i64, i32, i32, i32, i32, vp, vp, vp]
         lib.sfc_gemm_workspace_size2.restype = sz
         for name in EXPORTS:
             if name not in ("sfc_gemm_workspace_size", "sfc_gemm_workspace_size2"):
@@ -184,6 +186,29 @@ def plan(M: int, N: int, K: int, ca_c: int = 0, out_dtype=None, tile="auto", in_
                                 ctypes.byref(t), ctypes.byref(c)), "sfc_gemm_plan")
     name = {v: k for k, v in TILES.items() if k not in (0, "auto")}[t.value]
     return name, c.value
+
+
+class DeviceDesc(ctypes.Structure):
+    """``sfc_device_desc_t``: a device as the library's time model sees it."""
+    _fields_ = [("num_sms", ctypes.c_int), ("pair_workers", ctypes.c_int), ("hbm_gbs", ctypes.c_double),
+                ("sm_ghz", ctypes.c_double)]
+
+
+GB300 = dict(num_sms=152, pair_workers=76, hbm_gbs=6700.0, sm_ghz=1.9)
+
+
+def plan_model(M: int, N: int, K: int, ca_c: int = 0, *, out: str = "bf16", ab: str = "bf16",
+               b_layout: str = "kn", device: dict | None = None):
+    """The time model alone (``sfc_gemm_plan_desc``, no GPU): ``(tile, ca_c,
+    predicted_ns)`` for a described device (default: GB300's figures)."""
+    d = DeviceDesc(**(device or GB300))
+    t, c, ns = ctypes.c_int(0), ctypes.c_int(0), ctypes.c_double(0.0)
+    ab_code = {"bf16": 0, "e4m3": 1, "e5m2": 2}[ab]
+    _check(load().sfc_gemm_plan_desc(ctypes.byref(d), int(M), int(N), int(K), int(ca_c),
+                                     SFC_F32 if out == "f32" else SFC_BF16, ab_code, B_LAYOUTS[b_layout],
+                                     ctypes.byref(t), ctypes.byref(c), ctypes.byref(ns)), "sfc_gemm_plan_desc")
+    name = {v: k for k, v in TILES.items() if k not in (0, "auto")}[t.value]
+    return name, c.value, ns.value
 
 
 def tune(A, B, C=None, *, out_dtype=None, b_layout: str = "kn", max_layers: int = 8, max_kbf: int = 4,
@@ -309,19 +334,39 @@ def gemm(A, B, C=None, *, ca_c: int = 1, out_dtype=None, order: str = "sfc", ass
 
 
 def gemm_noalloc(A, B, C, *, ca_c: int = 1, stream=None):
-    """C = A @ B through ``sfc_gemm_noalloc``: the K-layer partials use the
-    library's built-in scratch area, so the call allocates nothing.  C must be
-    preallocated (fp32 or bf16).  Raises SfcError(SFC_ERR_WORKSPACE) when the
-    partials would not fit in ``NOALLOC_SCRATCH_BYTES``."""
-    import torch
+    """C = A @ B through ``sfc_gemm_noalloc``, for callers that cannot allocate
+    device memory: the K-layer partials and the workers' item counter use the
+    library's built-in scratch area, so the call allocates nothing.  A: (M, K)
+    bf16, B: (K, N) bf16, both CUDA tensors with 16-byte-aligned rows (nothing
+    is repacked); C: preallocated (M, N) fp32 or bf16 CUDA tensor.  Raises
+    SfcError(SFC_ERR_WORKSPACE) when ca_c >= 2 layers' partials would not fit in
+    ``NOALLOC_SCRATCH_BYTES`` (ca_c = 0 picks a count that fits)."""
+    torch = _torch or _import_torch()
+    if A.dim() != 2 or B.dim() != 2 or C.dim() != 2:
+        raise ValueError("A, B and C must be 2-D")
     M, K = A.shape
-    N = B.shape[1]
+    K2, N = B.shape
+    if K != K2:
+        raise ValueError("inner dimensions differ: %d vs %d" % (K, K2))
+    if A.dtype != torch.bfloat16 or B.dtype != torch.bfloat16:
+        raise TypeError("A and B must be bfloat16")
+    if C.dtype not in (torch.float32, torch.bfloat16) or tuple(C.shape) != (M, N):
+        raise ValueError("C must be (M, N) float32 or bfloat16")
     rc = load().sfc_gemm_noalloc(M, N, K, ctypes.c_void_p(A.data_ptr()), ctypes.c_void_p(B.data_ptr()),
                                  ctypes.c_void_p(C.data_ptr()), _row_major_2d(A, "A"), _row_major_2d(B, "B"),
                                  _row_major_2d(C, "C"), int(ca_c),
                                  SFC_F32 if C.dtype == torch.float32 else SFC_BF16, _stream_ptr(stream))
     _check(rc, "sfc_gemm_noalloc")
     return C
+
+
+def pool_used_high(reset: bool = False) -> int:
+    """High-water mark in bytes of the memory in use from the library's
+    stream-ordered pools on the current device since the last reset
+    (``sfc_debug_pool_used_high``); ``reset=True`` starts a new count."""
+    v = ctypes.c_size_t(0)
+    _check(load().sfc_debug_pool_used_high(ctypes.byref(v), 1 if reset else 0), "sfc_debug_pool_used_high")
+    return int(v.value)
 
 
 def gemm_raw(M, N, K, A_ptr, B_ptr, C_ptr, lda, ldb, ldc, ca_c=1, stream_ptr=None) -> int:

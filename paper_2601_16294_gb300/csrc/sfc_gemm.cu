@@ -13,6 +13,7 @@
 #include <map>
 #include <mutex>
 #include <tuple>
+#include <unordered_set>
 #include <vector>
 
 #include "sfc_gemm.h"
@@ -52,12 +53,14 @@ constexpr int kMaxLayers = 4096;  // keeps the kernels' layer arithmetic in 32 b
 constexpr int kMaxKBlocks = 64;   // k_block_factor bound (keeps the kernels' pass arithmetic in 32 bits)
 constexpr uint64_t kDefaultTimeoutNs = 2000000000ull;  // 2 s per wait
 
-std::atomic<uint64_t> g_launch_seq{0};  // picks each launch's scheduler counter slot
+constexpr size_t kTicketBytes = 256;  // one call's ticket counter allocation (two words used)
+constexpr double kSlabClockGhz = 1.9;     // SM clock the time model's slab times assume
+constexpr double kHbmBytesPerNs = 6700.0; // attainable DRAM bandwidth of GB300 (a copy's, GB/s)
 
 // ---------------------------------------------------------- per-device state
 
 // Kernel variants.  Stage counts fill ~192 KB of shared memory per block.
-enum Variant { kSingle128 = 0, kSingle256 = 1, kPair128 = 2, kPair256 = 3, kQuad256 = 4, kNumVariants = 5 };
+enum Variant { kSingle128 = 0, kSingle256 = 1, kPair128 = 2, kPair256 = 3, kNumVariants = 4 };
 constexpr int kStagesSingle256 = 4;  // 48 KB stages
 constexpr int kStagesSingle128 = 6;  // 32 KB stages
 constexpr int kStagesPair256 = 6;    // 32 KB stages per CTA
@@ -65,32 +68,29 @@ constexpr int kStagesPair128 = 8;    // 24 KB stages per CTA
 constexpr int kDefaultChunkSlabs = 64;  // 4096 values of k per tensor-memory accumulation chain
 
 constexpr int variant_bn(int v) { return (v == kSingle128 || v == kPair128) ? 128 : 256; }
-constexpr bool variant_pair(int v) { return v == kPair128 || v == kPair256 || v == kQuad256; }
-constexpr int variant_cluster(int v) { return v == kQuad256 ? 4 : (variant_pair(v) ? 2 : 1); }
-constexpr int variant_bm(int v) { return v == kQuad256 ? 512 : (variant_pair(v) ? 256 : 128); }
+constexpr bool variant_pair(int v) { return v == kPair128 || v == kPair256; }
+constexpr int variant_cluster(int v) { return variant_pair(v) ? 2 : 1; }
+constexpr int variant_bm(int v) { return variant_pair(v) ? 256 : 128; }
 
 template <int BN, int STAGES>
 constexpr int single_smem() { return RingLayout<(kBM + BN) * 128, STAGES, BN / 32>::kDynamicBytes; }
 template <int BN, int STAGES>
 constexpr int pair_smem() { return RingLayout<PairStage<BN>::kBytes, STAGES, BN / 32>::kDynamicBytes; }
 
-// Kernel of each variant for one output type and input kind (F8: 8-bit float
-// inputs; their table has no quad kernel, so its entry repeats pair256).
+// Kernel of each variant for one output type and input kind (F8: 8-bit float inputs).
 template <typename OutT, bool F8>
 struct Kernels {
     using Fn = void (*)(CUtensorMap, CUtensorMap, CUtensorMap, GemmParams);
     static constexpr Fn single128 = sfc_gemm_kernel<128, kStagesSingle128, OutT, F8>;
     static constexpr Fn single256 = sfc_gemm_kernel<256, kStagesSingle256, OutT, F8>;
-    static constexpr Fn pair128 = sfc_gemm_pair_kernel<128, kStagesPair128, OutT, false, F8>;
-    static constexpr Fn pair256 = sfc_gemm_pair_kernel<256, kStagesPair256, OutT, false, F8>;
-    static constexpr Fn quad256 = F8 ? pair256 : sfc_gemm_pair_kernel<256, kStagesPair256, OutT, !F8, false>;
+    static constexpr Fn pair128 = sfc_gemm_pair_kernel<128, kStagesPair128, OutT, F8>;
+    static constexpr Fn pair256 = sfc_gemm_pair_kernel<256, kStagesPair256, OutT, F8>;
     static Fn get(int v) {
         switch (v) {
             case kSingle128: return single128;
             case kSingle256: return single256;
             case kPair128: return pair128;
-            case kPair256: return pair256;
-            default: return quad256;
+            default: return pair256;
         }
     }
 };
@@ -99,7 +99,7 @@ constexpr int variant_smem(int v) {
     return v == kSingle128   ? single_smem<128, kStagesSingle128>()
            : v == kSingle256 ? single_smem<256, kStagesSingle256>()
            : v == kPair128   ? pair_smem<128, kStagesPair128>()
-                             : pair_smem<256, kStagesPair256>();  // pair256 and quad256
+                             : pair_smem<256, kStagesPair256>();
 }
 
 // attr must hold two entries.  With `pdl` the kernel may begin launching
@@ -128,17 +128,28 @@ cudaLaunchConfig_t launch_config(int v, int grid, cudaStream_t s, cudaLaunchAttr
     return cfg;
 }
 
+// What the time model needs to know of a device (sfc_gemm_plan_desc takes it from the caller).
+struct Machine {
+    int workers[kNumVariants] = {0, 0, 0, 0};  // co-resident workers (blocks or clusters) per variant
+    double hbm_bytes_per_ns = 0.0;               // attainable DRAM bandwidth (bytes per ns = GB/s)
+    double sm_ghz = 0.0;                         // SM clock the tensor-core rate is taken at
+};
+
 struct DeviceInfo {
     std::once_flag once;
     int status = SFC_ERR_UNSUPPORTED;
     int num_sms = 0;
-    int chunk_slabs = kDefaultChunkSlabs;
-    int serpentine = 0;
-    int one_item_per_worker = 0;
-    int workers[kNumVariants] = {0, 0, 0, 0, 0};  // co-resident workers (blocks or clusters) per variant
+    int workers[kNumVariants] = {0, 0, 0, 0};  // co-resident workers (blocks or clusters) per variant
+    Machine machine;
     // the library's stream-ordered pool (layer workspaces, repacked operands): it keeps
     // freed memory for reuse, so a call after a synchronisation does not map new pages
     cudaMemPool_t pool = nullptr;
+    // ticket counters of the calls (dynamic dealing), from a pool of their own: every
+    // kernel leaves its counter zero, so an address this pool has handed out before
+    // (ticket_seen) is zero again when it is handed out next
+    cudaMemPool_t ticket_pool = nullptr;
+    std::mutex ticket_mu;
+    std::unordered_set<uintptr_t> ticket_seen;
 };
 DeviceInfo g_devices[kMaxDevices];
 
@@ -174,15 +185,6 @@ int device_setup(DeviceInfo** info) {
         if (e != cudaSuccess) { d.status = cuda_fail(e); return; }
         if (prop.major != 10 || prop.minor != 3) { d.status = SFC_ERR_UNSUPPORTED; return; }
         d.num_sms = prop.multiProcessorCount;
-        // experiment override of the accumulation chain length (slabs of 64 k; 0 = one chain per item)
-        if (const char* env = std::getenv("SFC_GEMM_CHUNK_SLABS")) {
-            const int v = std::atoi(env);
-            d.chunk_slabs = v > 0 ? v : (1 << 30);
-        }
-        if (const char* env = std::getenv("SFC_GEMM_SERPENTINE")) d.serpentine = std::atoi(env) != 0;
-        // experiment override: launch one block (pair) per item instead of one per SM, so the
-        // hardware dispatches the items in curve order as SMs free up
-        if (const char* env = std::getenv("SFC_GEMM_ONE_ITEM_PER_WORKER")) d.one_item_per_worker = std::atoi(env) != 0;
         e = set_attrs<float, false>();
         if (e == cudaSuccess) e = set_attrs<__nv_bfloat16, false>();
         if (e == cudaSuccess) e = set_attrs<float, true>();
@@ -197,6 +199,8 @@ int device_setup(DeviceInfo** info) {
         e = cudaMemPoolCreate(&d.pool, &props);
         uint64_t keep = UINT64_MAX;  // released only by sfc_release
         if (e == cudaSuccess) e = cudaMemPoolSetAttribute(d.pool, cudaMemPoolAttrReleaseThreshold, &keep);
+        if (e == cudaSuccess) e = cudaMemPoolCreate(&d.ticket_pool, &props);
+        if (e == cudaSuccess) e = cudaMemPoolSetAttribute(d.ticket_pool, cudaMemPoolAttrReleaseThreshold, &keep);
         if (e != cudaSuccess) { d.status = cuda_fail(e); return; }
         for (int v = 0; v < kNumVariants; ++v) {
             if (!variant_pair(v)) {
@@ -210,6 +214,9 @@ int device_setup(DeviceInfo** info) {
             if (e != cudaSuccess) { d.status = cuda_fail(e); return; }
             d.workers[v] = clusters;
         }
+        for (int v = 0; v < kNumVariants; ++v) d.machine.workers[v] = d.workers[v];
+        d.machine.hbm_bytes_per_ns = kHbmBytesPerNs;
+        d.machine.sm_ghz = kSlabClockGhz;
         d.status = SFC_OK;
     });
     if (d.status == SFC_OK) *info = &d;
@@ -289,21 +296,31 @@ int make_out_map(CUtensorMap* map, const void* ptr, int64_t rows, int64_t cols, 
 
 int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
 
+// row stride (elements) of the fp32 layer copies of C
+int64_t ws_ld(int64_t N) { return (N + 3) / 4 * 4; }
+
 // Planning a call: the tile variant and, when the caller asks for it
-// (ca_c = 0), the number of K layers.  The estimate of a (variant, c) pair is
-//   waves x (slabs of the longest layer) x (time of one slab on one worker)
-//   + for c > 1: the reduction's launch and its partial traffic (c fp32
-//     copies of C written and read back, C written once),
-// where waves = ceil(tiles x c / workers) and a slab's time is a 128 x bn x 64
-// block at the variant's measured tensor-pipe efficiency.  It reproduces the
-// best measured c on the high-K and prefill shapes (GB300, 152 SMs).
-constexpr double kSlabClockGhz = 1.9;        // SM clock the slab times assume
+// (ca_c = 0), the number of K layers, from a time model in the spirit of the
+// paper's fine-grained roofline (Sec. III-B, Eqs. 1-4: a BRGEMM takes
+// max(G gamma, beta (S_A + S_B))), written for the GPU's two levels:
+//   - on a worker, a slab (the BRGEMM step: 128 x bn x 64 per SM) takes the
+//     longer of its MMA time and its operand intake from L2; both are folded
+//     into the variant's measured efficiency kEff (one-SM tiles are intake
+//     bound, 2-SM 256-wide tiles are not), so the launch's tensor time is
+//     waves x (slabs of the longest layer) x slab time, waves = ceil(items /
+//     workers);
+//   - against DRAM, the launch reads A and B at least once (the curve order
+//     keeps the panels of the tiles in flight in L2) and writes C, or for c > 1
+//     the c fp32 partial copies of C: the launch takes at least those bytes /
+//     DRAM bandwidth, and the longer of the two times is the GEMM's;
+//   - for c > 1 the reduction adds its launch and its own DRAM traffic (the c
+//     copies read back, C written).
+// The tile and layer count with the least time win (ties keep fewer layers).
 constexpr double kReduceLaunchNs = 3000.0;   // reduction kernel launch and ramp
-constexpr double kPartialBytesPerNs = 6000.0;
 // relative tensor-pipe efficiency measured on GB300, back to back at 8192 x
 // 8192 x 4096 and 6144^2 x 4096 (256-wide tiles feed the tensor core with fewer
-// shared-memory bytes per flop; the quad variant is kept just below the pair)
-constexpr double kEff[kNumVariants] = {0.60, 0.82, 0.62, 0.95, 0.92};
+// shared-memory bytes per flop)
+constexpr double kEff[kNumVariants] = {0.60, 0.82, 0.62, 0.95};
 
 // Layers ca_c = 0 may choose: enough to give about 320 items of 128 x 128,
 // never more than 64 or the number of K slabs (host-only, so the workspace
@@ -321,16 +338,20 @@ int64_t auto_layer_cap(int64_t M, int64_t N, int64_t K, int ab = SFC_AB_BF16) {
     return cap < 1 ? 1 : cap;
 }
 
-double plan_cost(int64_t M, int64_t N, int64_t K, int c, int v, const DeviceInfo& d, int out_bytes, int ab) {
+double plan_cost(int64_t M, int64_t N, int64_t K, int c, int v, const Machine& m, int out_bytes, int ab) {
     const int64_t items = ceil_div(M, variant_bm(v)) * ceil_div(N, variant_bn(v)) * c;
-    const int64_t waves = ceil_div(items, d.workers[v]);
+    const int64_t waves = ceil_div(items, m.workers[v]);
     // a slab of 8-bit inputs holds twice the k at twice the rate: the same time per slab
     const int64_t slabs = ceil_div(ceil_div(K, slab_k(ab)), c);
-    const double slab_ns = 128.0 * variant_bn(v) * kBK * 2.0 / (8192.0 * kEff[v]) / kSlabClockGhz;
-    double t = static_cast<double>(waves) * static_cast<double>(slabs) * slab_ns;
-    if (c > 1)
-        t += kReduceLaunchNs + (8.0 * c + out_bytes) * static_cast<double>(M) * static_cast<double>(N) /
-                                   kPartialBytesPerNs;
+    const double slab_ns = 128.0 * variant_bn(v) * kBK * 2.0 / (8192.0 * kEff[v]) / m.sm_ghz;
+    const double t_tensor = static_cast<double>(waves) * static_cast<double>(slabs) * slab_ns;
+    const double mn = static_cast<double>(M) * static_cast<double>(N);
+    const double ab_bytes = in_bytes(ab) * (static_cast<double>(M) * K + static_cast<double>(K) * N);
+    const double out_gemm = (c > 1) ? 4.0 * c * static_cast<double>(M) * static_cast<double>(ws_ld(N))
+                                    : out_bytes * mn;
+    const double t_dram = (ab_bytes + out_gemm) / m.hbm_bytes_per_ns;
+    double t = t_tensor > t_dram ? t_tensor : t_dram;
+    if (c > 1) t += kReduceLaunchNs + (4.0 * c + out_bytes) * mn / m.hbm_bytes_per_ns;
     return t;
 }
 
@@ -342,26 +363,22 @@ struct Plan {
 // ca_c >= 1: the variant for it; ca_c = 0: the best (variant, c) with c up to
 // max_c.  A requested tile fixes the variant (falling back to one SM when
 // pairs cannot be co-scheduled).
-// Variants that can serve a call: the quad variant takes bf16 with N-major B
-// only; 8-bit N-major B needs 128-byte (128-column) boxes per CTA, which the
-// 256 x 128 pair tile (64 columns per CTA) does not have.
+// Variants that can serve a call: 8-bit N-major B needs 128-byte (128-column)
+// boxes per CTA, which the 256 x 128 pair tile (64 columns per CTA) does not have.
 bool variant_allowed(int v, bool b_kmajor, int ab) {
-    if (v == kQuad256) return !b_kmajor && ab == SFC_AB_BF16;
     if (v == kPair128 && ab != SFC_AB_BF16 && !b_kmajor) return false;
     return true;
 }
 
-Plan make_plan(int64_t M, int64_t N, int64_t K, int ca_c, int max_c, const DeviceInfo& d, sfc_tile_t tile,
-               int out_bytes, bool b_kmajor = false, int ab = SFC_AB_BF16) {
+Plan make_plan(int64_t M, int64_t N, int64_t K, int ca_c, int max_c, const Machine& d, sfc_tile_t tile,
+               int out_bytes, bool b_kmajor = false, int ab = SFC_AB_BF16, double* t_out = nullptr) {
     int fixed = -1;
-    if (tile == SFC_TILE_QUAD_N256 && !variant_allowed(kQuad256, b_kmajor, ab)) tile = SFC_TILE_PAIR_N256;
     if (tile == SFC_TILE_PAIR_N128 && !variant_allowed(kPair128, b_kmajor, ab)) tile = SFC_TILE_N128;
     switch (tile) {
         case SFC_TILE_N128: fixed = kSingle128; break;
         case SFC_TILE_N256: fixed = kSingle256; break;
         case SFC_TILE_PAIR_N128: fixed = d.workers[kPair128] > 0 ? kPair128 : kSingle128; break;
         case SFC_TILE_PAIR_N256: fixed = d.workers[kPair256] > 0 ? kPair256 : kSingle256; break;
-        case SFC_TILE_QUAD_N256: fixed = d.workers[kQuad256] > 0 ? kQuad256 : kSingle256; break;
         default: break;
     }
     Plan best{fixed >= 0 ? fixed : kSingle128, ca_c > 0 ? ca_c : 1};
@@ -377,6 +394,7 @@ Plan make_plan(int64_t M, int64_t N, int64_t K, int ca_c, int max_c, const Devic
             }
         }
     }
+    if (t_out) *t_out = best_t;
     return best;
 }
 
@@ -395,7 +413,7 @@ int validate(int64_t M, int64_t N, int64_t K, const void* A, const void* B, cons
         assign != SFC_ASSIGN_WAVE_STATIC)
         return SFC_ERR_INVALID_ARG;
     if (tile != SFC_TILE_AUTO && tile != SFC_TILE_N128 && tile != SFC_TILE_N256 && tile != SFC_TILE_PAIR_N128 &&
-        tile != SFC_TILE_PAIR_N256 && tile != SFC_TILE_QUAD_N256)
+        tile != SFC_TILE_PAIR_N256)
         return SFC_ERR_INVALID_ARG;
     // TMA coordinates and tile indices are 32-bit
     if (M > (int64_t(1) << 31) - kBM || N > (int64_t(1) << 31) - 256 || K > (int64_t(1) << 31) - slab_k(ab))
@@ -411,8 +429,6 @@ int validate(int64_t M, int64_t N, int64_t K, const void* A, const void* B, cons
     if (lda >= (int64_t(1) << 39) || ldb >= (int64_t(1) << 39)) return SFC_ERR_INVALID_ARG;
     return SFC_OK;
 }
-
-int64_t ws_ld(int64_t N) { return (N + 3) / 4 * 4; }
 
 // fp32 workspace of a call: one copy of C per K layer when there is more than
 // one layer, and one copy when K blocks are summed for a bf16 C (an fp32 C
@@ -459,8 +475,7 @@ struct TuneTable {
 TuneTable g_tune[kMaxDevices];
 std::atomic<int> g_tune_lookup{1};  // 1: exact shape only; 2: else the nearest tuned shape (Sec. III-C, third way)
 
-constexpr int kTileOf[kNumVariants] = {SFC_TILE_N128, SFC_TILE_N256, SFC_TILE_PAIR_N128, SFC_TILE_PAIR_N256,
-                                       SFC_TILE_QUAD_N256};
+constexpr int kTileOf[kNumVariants] = {SFC_TILE_N128, SFC_TILE_N256, SFC_TILE_PAIR_N128, SFC_TILE_PAIR_N256};
 
 // Tuned (tile, layers) for a call that lets the library choose the tile:
 // with ca_c > 0 the fastest tile for that layer count, with ca_c = 0 the
@@ -538,6 +553,37 @@ void free_packed(void* packed[2], cudaStream_t stream) {
         if (packed[i]) cudaFreeAsync(packed[i], stream);  // stream-ordered: after the kernels that read them
 }
 
+// The ticket counter of one call's kernels (dynamic dealing), in memory the
+// call owns: stream-ordered from the ticket pool, freed after the call's last
+// kernel, so launches in flight at the same time -- on other streams, or
+// replays of captured graphs -- never share a counter.  It must read zero when
+// the first kernel starts.  The kernels leave it zero, and the pool hands an
+// address out again only after the free that follows them, so an address seen
+// before needs nothing; an address not seen before, and graph memory taken
+// during a stream capture, is zeroed on the stream first.
+int take_ticket(DeviceInfo* dev, cudaStream_t stream, unsigned int** out) {
+    cudaStreamCaptureStatus capture = cudaStreamCaptureStatusNone;
+    cudaError_t e = cudaStreamIsCapturing(stream, &capture);
+    if (e != cudaSuccess) return cuda_fail(e);
+    void* ptr = nullptr;
+    e = cudaMallocFromPoolAsync(&ptr, kTicketBytes, dev->ticket_pool, stream);
+    if (e != cudaSuccess) return cuda_fail(e);
+    bool seen = false;
+    if (capture == cudaStreamCaptureStatusNone) {
+        std::lock_guard<std::mutex> lock(dev->ticket_mu);
+        seen = !dev->ticket_seen.insert(reinterpret_cast<uintptr_t>(ptr)).second;
+    }
+    if (!seen) {
+        e = cudaMemsetAsync(ptr, 0, kTicketBytes, stream);
+        if (e != cudaSuccess) {
+            cudaFreeAsync(ptr, stream);
+            return cuda_fail(e);
+        }
+    }
+    *out = static_cast<unsigned int*>(ptr);
+    return SFC_OK;
+}
+
 // C = cvt(sum over layers of the fp32 copies in ws [+ beta * C + bias]), Listing 1's final reduction.
 cudaError_t launch_reduce(const DeviceInfo* dev, const float* ws, int64_t ldo, int64_t layer_stride, int layers,
                           int64_t M, int64_t N, void* C, int64_t ldc, int c_dtype, float beta, const float* bias,
@@ -571,7 +617,7 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
              int64_t ldc, int ca_c, int c_dtype, int order, int assign, int tile, void* workspace,
              size_t workspace_bytes, cudaStream_t stream, int debug_never, uint64_t timeout_ns,
              int b_layout = SFC_B_KN, float beta = 0.0f, const float* bias = nullptr, int ab = SFC_AB_BF16,
-             bool allow_pack = true, int kbf = 1) {
+             bool allow_pack = true, int kbf = 1, unsigned int* fixed_ticket = nullptr) {
     int rc = validate(M, N, K, A, B, C, lda, ldb, ldc, ca_c, c_dtype, order, assign, tile, b_layout, ab);
     if (rc != SFC_OK) return rc;
     // K blocks per layer (Listing 1's k_block_factor): every layer needs at least kbf slabs
@@ -610,7 +656,7 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     if (max_c > Kt_all / kbf) max_c = static_cast<int>(Kt_all / kbf);
     while (ca_c == 0 && workspace && max_c > 1 && workspace_bytes < workspace_bytes_for(M, N, max_c, kbf, c_dtype))
         --max_c;
-    const Plan plan = make_plan(M, N, K, ca_c, max_c, *dev, static_cast<sfc_tile_t>(tile), c_dtype == SFC_F32 ? 4 : 2,
+    const Plan plan = make_plan(M, N, K, ca_c, max_c, dev->machine, static_cast<sfc_tile_t>(tile), c_dtype == SFC_F32 ? 4 : 2,
                                 b_kmajor, ab);
     const int v = plan.v;
     ca_c = plan.c;
@@ -631,9 +677,8 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
             // B given as N x K: boxes of (this CTA's share of the tile's N rows) x one slab of k, like A
             rc = make_in_map(&tb, B, N, K, ldb, eb, variant_pair(v) ? bn / 2 : bn, sk);
         } else {
-            // N-major B boxes: one slab of k rows x 128 bytes of columns; with two pairs
-            // sharing B each CTA loads half the slab's rows
-            rc = make_in_map(&tb, B, K, N, ldb, eb, v == kQuad256 ? sk / 2 : sk, 128 / eb);
+            // N-major B boxes: one slab of k rows x 128 bytes of columns
+            rc = make_in_map(&tb, B, K, N, ldb, eb, sk, 128 / eb);
         }
     }
     if (rc != SFC_OK) {
@@ -651,14 +696,13 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     p.grid_tiles = p.Mt * p.Nt;
     p.kq = p.Kt / ca_c;
     p.kr = p.Kt % ca_c;
-    p.kc = dev->chunk_slabs;
-    p.serpentine = dev->serpentine;
+    p.kc = kDefaultChunkSlabs;
     p.num_items = static_cast<int64_t>(p.Mt) * p.Nt * ca_c;
     p.order = order;
     p.assign = (assign == SFC_ASSIGN_SEGMENT) ? 0 : 1;
     // dynamic dealing of curve positions for WAVE / AUTO; the static deals stay for comparison
     p.dynamic = (assign == SFC_ASSIGN_WAVE || assign == SFC_ASSIGN_AUTO) ? 1 : 0;
-    p.sched_slot = static_cast<int>(g_launch_seq.fetch_add(1, std::memory_order_relaxed) % kSchedSlots);
+    p.ticket = nullptr;
     p.debug_never = debug_never;
     p.timeout_ns = timeout_ns;
     p.b_kmajor = b_kmajor ? 1 : 0;
@@ -671,7 +715,7 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     p.kbf = 1;
     p.pass = 0;
     p.accumulate = 0;
-    const int64_t workers = dev->one_item_per_worker ? p.num_items : dev->workers[v];
+    const int64_t workers = dev->workers[v];
     const int64_t used = p.num_items < workers ? p.num_items : workers;
     const int grid = static_cast<int>(variant_cluster(v) * used);
 
@@ -684,6 +728,22 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
             return cuda_fail(e);
         }
         pooled = true;
+    }
+    // dynamic dealing: the call's own ticket counter (the K-block passes share it: each
+    // kernel leaves it zero, and a pass touches it only after the previous pass has finished)
+    bool own_ticket = false;
+    if (p.dynamic) {
+        if (fixed_ticket) {
+            p.ticket = fixed_ticket;
+        } else {
+            rc = take_ticket(dev, stream, &p.ticket);
+            if (rc != SFC_OK) {
+                if (pooled) cudaFreeAsync(ws, stream);
+                release_packed();
+                return rc;
+            }
+            own_ticket = true;
+        }
     }
 
     cudaError_t e = cudaSuccess;
@@ -709,7 +769,6 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
                 p.accumulate = p.tma_store;
                 p.beta = p.tma_store ? 0.0f : 1.0f;
                 p.bias = nullptr;
-                p.sched_slot = static_cast<int>(g_launch_seq.fetch_add(1, std::memory_order_relaxed) % kSchedSlots);
             }
             p.kbf = kbf;
             p.pass = pass;
@@ -732,7 +791,6 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
                 p.c_in = ws;
                 p.ldc_in = p.ldo;
                 p.c_in_layer_stride = p.layer_stride;
-                p.sched_slot = static_cast<int>(g_launch_seq.fetch_add(1, std::memory_order_relaxed) % kSchedSlots);
             }
             p.kbf = kbf;
             p.pass = pass;
@@ -744,6 +802,10 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     }
     if (pooled) {
         cudaError_t f = cudaFreeAsync(ws, stream);
+        if (e == cudaSuccess) e = f;
+    }
+    if (own_ticket) {
+        cudaError_t f = cudaFreeAsync(p.ticket, stream);
         if (e == cudaSuccess) e = f;
     }
     release_packed();  // stream-ordered: after the kernels that read the packed copies
@@ -806,11 +868,36 @@ SFC_API int sfc_gemm_plan(int64_t M, int64_t N, int64_t K, int ca_c, int c_dtype
             ca_c = t_c;
         }
     }
-    const Plan plan = make_plan(M, N, K, ca_c, static_cast<int>(auto_layer_cap(M, N, K, ab_dtype)), *dev,
+    const Plan plan = make_plan(M, N, K, ca_c, static_cast<int>(auto_layer_cap(M, N, K, ab_dtype)), dev->machine,
                                 static_cast<sfc_tile_t>(tile), c_dtype == SFC_F32 ? 4 : 2, b_layout == SFC_B_NK,
                                 ab_dtype);
     *out_tile = kTileOf[plan.v];
     *out_ca_c = plan.c;
+    return SFC_OK;
+}
+
+SFC_API int sfc_gemm_plan_desc(const sfc_device_desc_t* desc, int64_t M, int64_t N, int64_t K, int ca_c,
+                               int c_dtype, int ab_dtype, int b_layout, int* out_tile, int* out_ca_c,
+                               double* out_ns) {
+    if (!desc || !out_tile || !out_ca_c || !out_ns) return SFC_ERR_INVALID_ARG;
+    if (desc->num_sms < 1 || desc->pair_workers < 0 || 2 * desc->pair_workers > desc->num_sms ||
+        !(desc->hbm_gbs > 0.0) || !(desc->sm_ghz > 0.0))
+        return SFC_ERR_INVALID_ARG;
+    const int64_t kp = K + (16 - K % 16) % 16, np = N + (16 - N % 16) % 16;  // strides that pass the checks
+    int rc = validate(M, N, K, reinterpret_cast<const void*>(16), reinterpret_cast<const void*>(16),
+                      reinterpret_cast<const void*>(16), kp, b_layout == SFC_B_NK ? kp : np, N, ca_c, c_dtype,
+                      SFC_ORDER_SFC, SFC_ASSIGN_AUTO, SFC_TILE_AUTO, b_layout, ab_dtype);
+    if (rc != SFC_OK) return rc;
+    Machine m;
+    for (int v = 0; v < kNumVariants; ++v) m.workers[v] = variant_pair(v) ? desc->pair_workers : desc->num_sms;
+    m.hbm_bytes_per_ns = desc->hbm_gbs;
+    m.sm_ghz = desc->sm_ghz;
+    double t = 0.0;
+    const Plan plan = make_plan(M, N, K, ca_c, static_cast<int>(auto_layer_cap(M, N, K, ab_dtype)), m, SFC_TILE_AUTO,
+                                c_dtype == SFC_F32 ? 4 : 2, b_layout == SFC_B_NK, ab_dtype, &t);
+    *out_tile = kTileOf[plan.v];
+    *out_ca_c = plan.c;
+    *out_ns = t;
     return SFC_OK;
 }
 
@@ -825,6 +912,12 @@ SFC_API int sfc_release(void) {
     if (rc != SFC_OK) return rc;
     cudaError_t e = cudaDeviceSynchronize();
     if (e == cudaSuccess) e = cudaMemPoolTrimTo(dev->pool, 0);
+    if (e == cudaSuccess) {
+        // memory the ticket pool maps again later holds anything: forget the addresses seen
+        std::lock_guard<std::mutex> lock(dev->ticket_mu);
+        e = cudaMemPoolTrimTo(dev->ticket_pool, 0);
+        dev->ticket_seen.clear();
+    }
     return e == cudaSuccess ? SFC_OK : cuda_fail(e);
 }
 
@@ -900,7 +993,7 @@ SFC_API int sfc_gemm_tune(int64_t M, int64_t N, int64_t K, const void* A, const 
     // layer counts 1, 2, 4, ... and the time model's own choice
     std::vector<int> counts;
     for (int c = 1; c <= max_layers && c <= Kt; c *= 2) counts.push_back(c);
-    const Plan model = make_plan(M, N, K, 0, static_cast<int>(auto_layer_cap(M, N, K, ab_dtype)), *dev,
+    const Plan model = make_plan(M, N, K, 0, static_cast<int>(auto_layer_cap(M, N, K, ab_dtype)), dev->machine,
                                  SFC_TILE_AUTO, c_dtype == SFC_F32 ? 4 : 2, b_kmajor, ab_dtype);
     if (model.c <= max_layers && std::find(counts.begin(), counts.end(), model.c) == counts.end())
         counts.push_back(model.c);
@@ -940,7 +1033,7 @@ SFC_API int sfc_gemm_tune(int64_t M, int64_t N, int64_t K, const void* A, const 
     float best = -1.0f;            // the fastest configuration so far
     float model_us = -1.0f;        // the time model's layer count, with its measured tile
     for (int c : counts) {
-        const int model_v = make_plan(M, N, K, c, c, *dev, SFC_TILE_AUTO, c_dtype == SFC_F32 ? 4 : 2, b_kmajor,
+        const int model_v = make_plan(M, N, K, c, c, dev->machine, SFC_TILE_AUTO, c_dtype == SFC_F32 ? 4 : 2, b_kmajor,
                                       ab_dtype).v;
         float t[kNumVariants];
         for (int v = 0; v < kNumVariants; ++v) t[v] = -1.0f;
@@ -1011,19 +1104,16 @@ SFC_API int sfc_gemm_tune_forget(void) {
 }
 
 SFC_API int sfc_get_device_status(void* stream) {
-    cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    cudaError_t e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return cuda_fail(e);
     unsigned int word = 0;
     e = cudaMemcpyFromSymbol(&word, g_sfc_status, sizeof(word));
     if (e != cudaSuccess) return cuda_fail(e);
     if (word == 0) return SFC_OK;
-    const unsigned int zero = 0;
-    e = cudaMemcpyToSymbol(g_sfc_status, &zero, sizeof(zero));
-    if (e != cudaSuccess) return cuda_fail(e);
-    // a launch that gave up still returns its scheduler slot, but make sure
-    static const unsigned int zeros[kSchedSlots] = {};
-    e = cudaMemcpyToSymbol(g_sched_next, zeros, sizeof(zeros));
-    if (e == cudaSuccess) e = cudaMemcpyToSymbol(g_sched_done, zeros, sizeof(zeros));
+    // clear the bits that were read (atomically: a kernel on another stream may be setting others)
+    e = launch_plain(status_clear_kernel, 1, 1, s, word);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(s);
     if (e != cudaSuccess) return cuda_fail(e);
     return SFC_ERR_TIMEOUT;
 }
@@ -1045,18 +1135,20 @@ SFC_API int sfc_debug_force_timeout(const void* A, const void* B, void* C, int l
 
 // ---------------------------------------------------------------------------
 // Allocation-free entry point.  The fp32 partial copies of C live in a fixed
-// device array of this module instead of caller or pool memory; host code
-// must not pass the array's name to a kernel (on the host it is only a
-// stand-in symbol), so its device address is looked up once per device.
+// device array of this module instead of caller or pool memory, and so does
+// the call's ticket counter (after the partials).  Host code must not pass
+// the array's name to a kernel (on the host it is only a stand-in symbol), so
+// its device address is looked up once per device.
 // ---------------------------------------------------------------------------
 namespace sfc {
 namespace {
 
-static __device__ __align__(256) unsigned char g_noalloc_scratch[SFC_NOALLOC_SCRATCH_BYTES];
+// zero when the module loads; every kernel leaves the ticket counter zero again
+static __device__ __align__(256) unsigned char g_noalloc_scratch[SFC_NOALLOC_SCRATCH_BYTES + kTicketBytes];
 
 struct NoAllocScratch {
-    std::once_flag once;
-    int status = SFC_ERR_CUDA;
+    std::mutex mu;
+    bool found = false;  // set only once a lookup has succeeded; a failed one is retried next call
     void* ptr = nullptr;
 };
 NoAllocScratch g_noalloc[kMaxDevices];
@@ -1066,15 +1158,16 @@ int noalloc_scratch(void** ptr) {
     int rc = current_device(&dev);
     if (rc != SFC_OK) return rc;
     NoAllocScratch& s = g_noalloc[dev];
-    std::call_once(s.once, [&]() {
+    std::lock_guard<std::mutex> lock(s.mu);
+    if (!s.found) {
         void* p = nullptr;
         cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-        if (e != cudaSuccess) { s.status = cuda_fail(e); return; }
+        if (e != cudaSuccess) return cuda_fail(e);
         s.ptr = p;
-        s.status = SFC_OK;
-    });
-    if (s.status == SFC_OK) *ptr = s.ptr;
-    return s.status;
+        s.found = true;
+    }
+    *ptr = s.ptr;
+    return SFC_OK;
 }
 
 }  // namespace
@@ -1083,12 +1176,35 @@ int noalloc_scratch(void** ptr) {
 SFC_API int sfc_gemm_noalloc(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void* C,
                              int64_t lda, int64_t ldb, int64_t ldc, int ca_c, sfc_dtype_t c_dtype,
                              void* stream) {
-    if (sfc_gemm_workspace_size(M, N, K, ca_c) > SFC_NOALLOC_SCRATCH_BYTES) return SFC_ERR_WORKSPACE;
     void* scratch = nullptr;
     int rc = noalloc_scratch(&scratch);
     if (rc != SFC_OK) return rc;
+    // ca_c > 0 whose partials exceed the scratch area: SFC_ERR_WORKSPACE from run_gemm;
+    // ca_c = 0: the library's layer count is limited to what fits
+    unsigned int* ticket = reinterpret_cast<unsigned int*>(static_cast<unsigned char*>(scratch) +
+                                                           SFC_NOALLOC_SCRATCH_BYTES);
     return run_gemm(M, N, K, A, B, C, lda, ldb, ldc, ca_c, c_dtype, SFC_ORDER_SFC, SFC_ASSIGN_AUTO, SFC_TILE_AUTO,
                     scratch, SFC_NOALLOC_SCRATCH_BYTES, static_cast<cudaStream_t>(stream), 0, kDefaultTimeoutNs,
-                    SFC_B_KN, 0.0f, nullptr, SFC_AB_BF16, /*allow_pack=*/false);
+                    SFC_B_KN, 0.0f, nullptr, SFC_AB_BF16, /*allow_pack=*/false, /*kbf=*/1, ticket);
 }
 
+SFC_API int sfc_debug_pool_used_high(size_t* used_high_bytes, int reset) {
+    if (!used_high_bytes || (reset != 0 && reset != 1)) return SFC_ERR_INVALID_ARG;
+    DeviceInfo* dev = nullptr;
+    int rc = device_setup(&dev);
+    if (rc != SFC_OK) return rc;
+    size_t total = 0;
+    for (cudaMemPool_t pool : {dev->pool, dev->ticket_pool}) {
+        cuuint64_t v = 0;
+        cudaError_t e = cudaMemPoolGetAttribute(pool, cudaMemPoolAttrUsedMemHigh, &v);
+        if (e != cudaSuccess) return cuda_fail(e);
+        total += static_cast<size_t>(v);
+        if (reset) {
+            cuuint64_t zero = 0;
+            e = cudaMemPoolSetAttribute(pool, cudaMemPoolAttrUsedMemHigh, &zero);
+            if (e != cudaSuccess) return cuda_fail(e);
+        }
+    }
+    *used_high_bytes = total;
+    return SFC_OK;
+}

@@ -83,13 +83,12 @@ enum WaitSite : unsigned int {
 // of the worker through a small queue in shared memory.  Static dealing gives
 // worker w the items first + j * step; dynamic dealing gives it item w first
 // (so no block waits on a counter to start) and then workers + the next value
-// of a per-launch counter, i.e. curve positions are taken in order as workers
-// free up.  The counters form a ring of slots, one per launch, each reset by
-// the last scheduler of its launch to finish.
-constexpr int kSchedSlots = 1024;
+// of the launch's ticket counter, i.e. curve positions are taken in order as
+// workers free up.  The counter ({next ticket, schedulers done}, two words) is
+// memory of the call that launched the kernel, so no other launch can share
+// it; it must be zero when the kernel starts and is zero again when it ends
+// (the last scheduler to finish resets both words, also after a wait gave up).
 constexpr int kQueue = 4;
-__device__ unsigned int g_sched_next[kSchedSlots];
-__device__ unsigned int g_sched_done[kSchedSlots];
 
 struct GemmParams {
     int64_t M, N;
@@ -105,10 +104,9 @@ struct GemmParams {
     int order;             // 0 = generalized Hilbert, 1 = raster
     int assign;            // static deal: 0 = contiguous segments, 1 = strided waves
     int dynamic;           // 1: workers take the next curve position from a shared counter
-    int sched_slot;        // counter slot of this launch (dynamic)
+    unsigned int* ticket;  // dynamic dealing: this launch's counter {next, done}, zero at start
     int vec_store;         // 1 if 16-byte vector stores are aligned
     int tma_store;         // 1: stores go through smem staging and the output tensor map
-    int serpentine;        // 1: alternate the K direction between a worker's consecutive items
     int debug_never;       // test hook: MMA warp waits on a barrier nobody arrives at
     uint64_t timeout_ns;   // bound for every mbarrier wait
     int b_kmajor;          // 1: B is given as N x K row-major (B transposed), loaded K-major
@@ -124,11 +122,10 @@ struct GemmParams {
 
 struct WorkItem {
     int tm, tn, k0, k1, layer;
-    int rev;  // 1: walk this item's K slabs from k1-1 down to k0
 };
 
-// Slab index of the q-th slab this item processes.
-__device__ __forceinline__ int slab_at(const WorkItem& w, int q) { return w.rev ? (w.k1 - 1 - q) : (w.k0 + q); }
+// Slab index of the q-th slab this item processes (K slabs in increasing order).
+__device__ __forceinline__ int slab_at(const WorkItem& w, int q) { return w.k0 + q; }
 
 // First K slab of layer l: floor(l * Kt / c) = l * (Kt / c) + floor(l * (Kt % c) / c),
 // in 32-bit arithmetic (c <= 4096 keeps l * (Kt % c) below 2^24).
@@ -160,7 +157,6 @@ __device__ __forceinline__ WorkItem decode_item(int64_t i64, const GemmParams& p
     w.layer = layer;
     w.k0 = layer_k0(layer, p);
     w.k1 = layer_k0(layer + 1, p);
-    w.rev = 0;
     narrow_to_pass(w, p);
     return w;
 }
@@ -355,7 +351,6 @@ __device__ __forceinline__ int64_t src_take(const ItemSource& S, int j, const Ge
     ptx::mbar_arrive_remote(S.q_empty0 + 8u * q);  // slot free once every consumer has read it
     w.k0 = (p.ca_c == 1) ? 0 : layer_k0(w.layer, p);
     w.k1 = (p.ca_c == 1) ? p.Kt : layer_k0(w.layer + 1, p);
-    w.rev = p.serpentine ? (j & 1) : 0;
     narrow_to_pass(w, p);
     return item;
 }
@@ -396,7 +391,7 @@ __device__ __forceinline__ void sched_send(const ItemSource& S, int j, const Que
 __device__ __forceinline__ int sched_next(const ItemSource& S, int j, const GemmParams& p) {
     int64_t pos;
     if (S.dynamic)
-        pos = (j == 0) ? S.worker : S.workers + static_cast<int64_t>(atomicAdd(&g_sched_next[p.sched_slot], 1u));
+        pos = (j == 0) ? S.worker : S.workers + static_cast<int64_t>(atomicAdd(&p.ticket[0], 1u));
     else
         pos = S.first + j * S.step;
     const int64_t end = S.dynamic ? p.num_items : S.end;
@@ -425,12 +420,12 @@ __device__ __forceinline__ bool run_scheduler(const ItemSource& S, int item0, co
         if (item < 0) break;
     }
     if (S.dynamic) {
-        // the last scheduler of the launch returns the counter slot to zero
+        // the last scheduler of the launch returns the counter to zero
         __threadfence();
-        const unsigned int before = atomicAdd(&g_sched_done[p.sched_slot], 1u);
+        const unsigned int before = atomicAdd(&p.ticket[1], 1u);
         if (static_cast<int64_t>(before) == S.workers - 1) {
-            g_sched_next[p.sched_slot] = 0;
-            g_sched_done[p.sched_slot] = 0;
+            p.ticket[0] = 0;
+            p.ticket[1] = 0;
             __threadfence();
         }
     }
@@ -516,7 +511,6 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
     OutT* out = static_cast<OutT*>(p.out);
     const uint32_t acce_target = PAIR ? ptx::map_to_cta(B.acc_empty(0), pair_leader) : B.acc_empty(0);
     float run[kEpiCols];
-    int nbox = 0;  // boxes this warp has stored (selects the staging half)
     // beta C_in + bias in this epilogue only without K layers (else the reduction applies
     // it), or when a later K block adds into the layer copies (k_block_factor > 1)
     const bool affine = (p.ca_c == 1 || p.c_in_layer_stride != 0) && (p.beta != 0.0f || p.bias != nullptr);
@@ -586,30 +580,42 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
             // stage 32-row boxes and let the TMA write them (edges clipped by the map);
             // the two boxes of the buffer alternate
             constexpr int kCols = box_cols<OutT>();
+            // the two boxes of the warp's buffer are staged together, then one proxy fence,
+            // one warp sync and one bulk group store both (a round per pair of boxes, not per box)
+            uint8_t* buf = staging + ew * kStageBufBytes;
 #pragma unroll
-            for (int g = 0; g < kEpiCols / kCols; ++g) {
+            for (int g = 0; g < kEpiCols / kCols; g += 2) {
                 if (col_base + g * kCols >= p.N) break;  // warp-uniform
-                uint8_t* box = staging + ew * kStageBufBytes + (nbox & 1) * kBoxBytes;
-                if (affine)
+                const bool has1 = col_base + (g + 1) * kCols < p.N;
+                if (affine) {
                     apply_affine<OutT, kCols>(p, warp_row + lane, col_base + g * kCols, w.layer, run + g * kCols);
-                if (lane == 0) ptx::bulk_wait_read_1();  // the store that last used this box has read it
+                    if (has1)
+                        apply_affine<OutT, kCols>(p, warp_row + lane, col_base + (g + 1) * kCols, w.layer,
+                                                  run + (g + 1) * kCols);
+                }
+                if (lane == 0) ptx::bulk_wait_read_all();  // the previous pair's stores have read the buffer
                 __syncwarp();
-                stage_row<OutT>(box, lane, run + g * kCols);
+                stage_row<OutT>(buf, lane, run + g * kCols);
+                if (has1) stage_row<OutT>(buf + kBoxBytes, lane, run + (g + 1) * kCols);
                 ptx::fence_proxy_async_smem();
                 __syncwarp();
                 if (lane == 0) {
-                    const uint32_t box_addr = ptx::smem_addr(box);
-                    const int32_t x = static_cast<int32_t>(col_base + g * kCols), y = static_cast<int32_t>(warp_row);
-                    if (p.ca_c > 1) {
-                        if (p.accumulate) ptx::tma_reduce_add_3d(tmap_c, box_addr, x, y, w.layer);
-                        else ptx::tma_store_3d(tmap_c, box_addr, x, y, w.layer);
-                    } else {
-                        if (p.accumulate) ptx::tma_reduce_add_2d(tmap_c, box_addr, x, y);
-                        else ptx::tma_store_2d(tmap_c, box_addr, x, y);
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        if (h == 1 && !has1) break;
+                        const uint32_t box_addr = ptx::smem_addr(buf + h * kBoxBytes);
+                        const int32_t x = static_cast<int32_t>(col_base + (g + h) * kCols);
+                        const int32_t y = static_cast<int32_t>(warp_row);
+                        if (p.ca_c > 1) {
+                            if (p.accumulate) ptx::tma_reduce_add_3d(tmap_c, box_addr, x, y, w.layer);
+                            else ptx::tma_store_3d(tmap_c, box_addr, x, y, w.layer);
+                        } else {
+                            if (p.accumulate) ptx::tma_reduce_add_2d(tmap_c, box_addr, x, y);
+                            else ptx::tma_store_2d(tmap_c, box_addr, x, y);
+                        }
                     }
                     ptx::bulk_commit();
                 }
-                ++nbox;
             }
         } else {
             const int64_t row = warp_row + lane;
@@ -892,6 +898,9 @@ pack_rows_kernel(const uint8_t* __restrict__ src, int64_t ld_src, int64_t rows, 
             dst[r * ld_dst + c] = src[r * ld_src + c];
     }
 }
+
+// Clears `bits` of the device error word (after the host has read them).
+__global__ void status_clear_kernel(unsigned int bits) { atomicAnd(&g_sfc_status, ~bits); }
 
 // out[s] = tm * Nt + tn for every curve position s, with the kernels' decoder.
 __global__ void tile_order_kernel(int Mt, int Nt, int32_t* __restrict__ out) {

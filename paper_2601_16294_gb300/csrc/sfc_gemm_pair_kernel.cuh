@@ -1,5 +1,4 @@
-// sfc_gemm_pair_kernel.cuh -- the SFC / SFC-CA GEMM on 2-SM CTA pairs (and on
-// clusters of two pairs that share the B slab).
+// sfc_gemm_pair_kernel.cuh -- the SFC / SFC-CA GEMM on 2-SM CTA pairs.
 //
 // Same task space, item order, accumulation chunks and epilogue as
 // sfc_gemm_kernel, but each worker is a cluster of two CTAs on two SMs that
@@ -18,12 +17,9 @@
 //     epilogue warps drain them and arrive on the leader's accumulator-empty
 //     barrier.
 //
-// QUAD variant: a 4-CTA cluster holds two pairs stacked in M, so an item is a
-// 512 x BN tile.  Both pairs need the same B slab: CTA r of each pair loads 32 of
-// the 64 K rows of its B half and multicasts them to itself and its counterpart
-// in the other pair, which halves the B bytes each SM requests from L2.  A stage
-// of a CTA is then written by two producers, so it is free only after both
-// pairs' MMAs have committed it (empty barriers count two arrivals).
+// Every TMA load writes the shared memory of the CTA that issues it (no
+// multicast loads); only the MMA completion signals (tcgen05.commit) are
+// multicast, as mbarrier arrivals within the pair.
 //
 // Waits are bounded as in the single-SM kernel.  The pair meets at a cluster
 // barrier after set-up (barriers initialised before any remote signal) and
@@ -46,12 +42,11 @@ struct PairStage {
     static_assert(kABytes % 1024 == 0 && kBBytes % 1024 == 0, "swizzle atoms need 1 KB alignment");
 };
 
-template <int BN, int STAGES, typename OutT, bool QUAD, bool F8>
+template <int BN, int STAGES, typename OutT, bool F8>
 __global__ void __launch_bounds__(block_threads(BN), 1)
 sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constant__ CUtensorMap tmap_b,
                      const __grid_constant__ CUtensorMap tmap_c, const GemmParams p) {
     static_assert(BN == 128 || BN == 256, "pair tiles are 256 x 128 or 256 x 256");
-    static_assert(!(QUAD && F8), "the quad variant takes bf16 inputs");
     using I = InKind<F8>;
     using S = PairStage<BN>;
     constexpr int kEpiWarps = BN / 32;
@@ -59,9 +54,8 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
     constexpr int kHalfN = S::kHalfN;
 
     constexpr uint32_t kTmemCols = 2 * BN;
-    // QUAD: a cluster of two pairs stacked in M (a 512 x BN item) sharing the B slab
-    constexpr int kCtas = QUAD ? 4 : 2;
-    constexpr int kItemRows = QUAD ? 2 * kPairBM : kPairBM;
+    constexpr int kCtas = 2;
+    constexpr int kItemRows = kPairBM;
 
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = ptx::smem_addr(smem_raw);
@@ -75,12 +69,10 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
     const int warp = threadIdx.x / 32;
     const int lane = threadIdx.x % 32;
     const uint32_t rank = ptx::cluster_ctarank();
-    const uint32_t r = rank & 1u;               // position in the pair
-    const uint32_t pair_idx = rank >> 1;        // which pair of the cluster
-    const uint32_t pair_leader = rank & ~1u;    // the pair's MMA-issuing CTA
+    const uint32_t r = rank;                    // position in the pair
+    const uint32_t pair_leader = 0;             // the pair's MMA-issuing CTA
     const bool leader = (r == 0);
-    const uint16_t pair_mask = static_cast<uint16_t>(0x3u << (2 * pair_idx));
-    const uint16_t stage_mask = QUAD ? 0xF : 0x3;  // CTAs whose smem a stage's loads write
+    const uint16_t pair_mask = 0x3;             // both CTAs of the pair
     ItemSource src;
     worker_items(p, blockIdx.x / kCtas, gridDim.x / kCtas, src.first, src.end, src.step);
     src.worker = blockIdx.x / kCtas;
@@ -103,8 +95,8 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
     if (threadIdx.x == 0) {
         ptx::pdl_launch_dependents();
         for (int s = 0; s < STAGES; ++s) {
-            ptx::mbar_init(B.full(s), 1);           // the pair leader's producer arrives once (+ tx bytes)
-            ptx::mbar_init(B.empty(s), QUAD ? 2 : 1);  // a commit from each pair whose loads share the stage
+            ptx::mbar_init(B.full(s), 1);   // the pair leader's producer arrives once (+ tx bytes)
+            ptx::mbar_init(B.empty(s), 1);  // one multicast commit of the pair's MMAs
         }
         for (int a = 0; a < 2; ++a) {
             ptx::mbar_init(B.acc_full(a), 1);               // one multicast commit per chunk
@@ -114,9 +106,9 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
         ptx::mbar_init(B.never(), 1);
         for (int q = 0; q < kQueue; ++q) {
             ptx::mbar_init(B.q_full(q), 1);  // the cluster's scheduler (in CTA 0) publishes
-            // (CTA 0's copy is used) every consuming role of the cluster has read: all producers,
-            // the pair leaders' MMA warps and all epilogue warps
-            ptx::mbar_init(B.q_empty(q), kCtas + kCtas / 2 + kCtas * kEpiWarps);
+            // (CTA 0's copy is used) every consuming role of the pair has read: both producers,
+            // the leader's MMA warp and all epilogue warps
+            ptx::mbar_init(B.q_empty(q), kCtas + 1 + kCtas * kEpiWarps);
         }
         ptx::mbar_init(B.q_taken(), 1);  // CTA 0's producer took an item (CTA 0's copy is used)
         *abort_flag = 0;
@@ -146,26 +138,16 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
             int64_t issued = 0;
             bool ok = produce<STAGES>(src, p, B, abort_flag, /*signal_taken=*/rank == 0, issued,
                                       [&](const WorkItem& w, int kt, int stage) {
-                const int32_t a_row = w.tm * kItemRows + static_cast<int32_t>(pair_idx * kPairBM + r * 128);
+                const int32_t a_row = w.tm * kItemRows + static_cast<int32_t>(r * 128);
                 const int32_t b_col = w.tn * BN + static_cast<int32_t>(r) * kHalfN;
                 if (leader) ptx::mbar_arrive_expect_tx(B.full(stage), 2 * S::kBytes);
                 const uint32_t leader_full = ptx::map_to_cta(B.full(stage), pair_leader);
                 const uint32_t sa = ring + stage * S::kBytes;
                 const uint32_t sb = sa + S::kABytes;
                 ptx::tma_load_2d_pair(sa, &tmap_a, leader_full, kt * I::kSlabK, a_row);
-                if (!QUAD && p.b_kmajor) {
+                if (p.b_kmajor) {
                     // this CTA's half of the B^T rows (N) x one slab of k, K-major like A
                     ptx::tma_load_2d_pair(sb, &tmap_b, leader_full, kt * I::kSlabK, b_col);
-                } else if constexpr (QUAD) {
-                    // the same B half-slab goes to this CTA and its counterpart in the
-                    // other pair: each loads 32 of the 64 K rows for both
-                    const uint16_t mask = static_cast<uint16_t>((1u << r) | (1u << (r + 2)));
-#pragma unroll
-                    for (int jb = 0; jb < kHalfN / I::kBCols; ++jb)
-                        ptx::tma_load_2d_pair_multicast(sb + jb * I::kBBoxBytes + pair_idx * (I::kSlabK / 2 * 128),
-                                                        &tmap_b, leader_full, b_col + jb * I::kBCols,
-                                                        kt * I::kSlabK + static_cast<int32_t>(pair_idx) * (I::kSlabK / 2),
-                                                        mask);
                 } else {
                     // N-major boxes of 128-byte rows (the host keeps 8-bit inputs with BN/2 >= 128 here)
 #pragma unroll
@@ -203,7 +185,7 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
             int acc = 0;
             uint32_t acc_phase = 0;
             bool ok = true;
-            const bool bk = !QUAD && p.b_kmajor;
+            const bool bk = p.b_kmajor != 0;
             const uint32_t idesc = ptx::idesc_f32(kPairBM, BN, /*A K-major*/ 0, bk ? 0u : 1u, p.ab_fmt);
             if (p.debug_never) ok = wait_bounded(B.never(), 0, abort_flag, p.timeout_ns, kWaitDebugNever);
             for (int j = 0; ok; ++j) {
@@ -243,9 +225,8 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
                         for (int kk = 0; kk < I::kSlabK / I::kMmaK; ++kk)
                             ptx::tc_mma_pair<F8>(d_tmem, adesc + 2u * kk, bdesc + bstep * kk, idesc,
                                                  (q > kb || kk > 0) ? 1u : 0u);
-                        // the stage is free in every CTA whose smem this pair read (and, with
-                        // QUAD, whose producer also wrote into this pair's smem)
-                        ptx::tc_commit_pair_multicast(B.empty(stage), stage_mask);
+                        // the stage is free in both CTAs once these MMAs have read it
+                        ptx::tc_commit_pair_multicast(B.empty(stage), pair_mask);
                         if (++stage == STAGES) {
                             stage = 0;
                             phase ^= 1u;
@@ -266,7 +247,7 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
         }
     } else if (warp < scheduler_warp(BN)) {
         run_epilogue<BN, OutT, true>(p, B, tmem_base, abort_flag, src, kItemRows,
-                                     static_cast<int>(pair_idx * kPairBM + r * 128), warp, lane, &tmap_c,
+                                     static_cast<int>(r * 128), warp, lane, &tmap_c,
                                      smem + L::kStagingOffset, pair_leader);
     } else if (sched_thread) {
         // -------------------------------------------------------- scheduler

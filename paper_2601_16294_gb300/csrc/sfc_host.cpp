@@ -41,7 +41,7 @@ namespace {
 
 constexpr int kMaxDevices = 64;
 constexpr int64_t kMaxPanels = 64;
-constexpr int64_t kPanelRowsM = 512;    // rows of the largest output tile (two stacked 2-SM pairs)
+constexpr int64_t kPanelRowsM = 512;    // a multiple of the rows of every output tile (256 at most)
 constexpr int64_t kPanelColsN = 256;    // columns of the widest output tile
 constexpr int64_t kAutoPanelSpan = 2048;  // automatic panels: about this many rows or columns each
 constexpr int64_t kAutoMaxPanels = 8;  // panels of the automatic span before the span grows

@@ -51,6 +51,22 @@ def test_sweep_of_125_shapes():
     assert all(s["shared"] and s["cs"] == CS for s in bench.WORKLOADS["sweep125"]["shapes"])
 
 
+def test_default_workload_is_configs_two_to_five():
+    # the metric's weighted harmonic mean spans the square, prefill, irregular and high-K sets
+    assert bench.parse_args.__defaults__ is None
+    import sys as _sys
+    argv = _sys.argv
+    try:
+        _sys.argv = ["bench.py"]
+        assert bench.parse_args().workload == "configs"
+    finally:
+        _sys.argv = argv
+    shapes = bench.WORKLOADS["configs"]["shapes"]
+    assert len(shapes) == 29
+    assert shapes == (bench.WORKLOADS["square"]["shapes"] + bench.WORKLOADS["prefill"]["shapes"] +
+                      bench.WORKLOADS["irregular"]["shapes"] + bench.WORKLOADS["highk"]["shapes"])
+
+
 def test_single_512_cube():
     assert dims("cube512") == [(512, 512, 512)]
     assert bench.WORKLOADS["cube512"]["shapes"][0]["out"] == "f32"

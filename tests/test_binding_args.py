@@ -112,3 +112,54 @@ def test_library_errors_become_sfc_errors(monkeypatch):
     with pytest.raises(binding.SfcError) as e:
         binding.gemm(bf(8, 8), bf(8, 8), torch.zeros(8, 8), stream=FakeStream())
     assert e.value.code == binding.SFC_ERR_UNALIGNED
+
+
+class FakeNoAlloc:
+    def __init__(self):
+        self.calls = []
+
+    def sfc_gemm_noalloc(self, *args):
+        self.calls.append(args)
+        return binding.SFC_OK
+
+
+@pytest.mark.parametrize("case", ["A_3d", "inner", "A_f32", "B_f16", "C_dtype", "C_shape", "A_col_stride"])
+def test_malformed_noalloc_calls_raise_before_the_library(monkeypatch, case):
+    # the allocation-free entry point's tensor maps take their extents from M, N and K,
+    # so a mis-shaped C or B would be read or written past its end: the binding refuses it
+    lib = FakeNoAlloc()
+    monkeypatch.setattr(binding, "_lib", lib)
+    A, B, C = bf(64, 32), bf(32, 48), torch.zeros(64, 48)
+    err = ValueError
+    if case == "A_3d":
+        A = bf(2, 64, 32)
+    elif case == "inner":
+        B = bf(40, 48)
+    elif case == "A_f32":
+        A = torch.zeros(64, 32)
+        err = TypeError
+    elif case == "B_f16":
+        B = B.half()
+        err = TypeError
+    elif case == "C_dtype":
+        C = C.half()
+    elif case == "C_shape":
+        C = torch.zeros(64, 40)
+    elif case == "A_col_stride":
+        A = bf(32, 64).t()
+    with pytest.raises(err):
+        binding.gemm_noalloc(A, B, C, ca_c=2, stream=FakeStream())
+    assert lib.calls == []
+
+
+def test_noalloc_passes_sizes_strides_and_codes(monkeypatch):
+    lib = FakeNoAlloc()
+    monkeypatch.setattr(binding, "_lib", lib)
+    A = bf(64, 40)[:, :32]
+    B = bf(32, 56)[:, :48]
+    C = torch.zeros(64, 52, dtype=torch.bfloat16)[:, :48]
+    assert binding.gemm_noalloc(A, B, C, ca_c=0, stream=FakeStream()) is C
+    (M, N, K, a, b, c, lda, ldb, ldc, ca_c, c_code, stream) = lib.calls[0]
+    assert (M, N, K, lda, ldb, ldc, ca_c) == (64, 48, 32, 40, 56, 52, 0)
+    assert (a.value, b.value, c.value) == (A.data_ptr(), B.data_ptr(), C.data_ptr())
+    assert c_code == binding.SFC_BF16 and stream == 0x1234

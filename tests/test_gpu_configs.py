@@ -1,11 +1,20 @@
-"""Full-size parity: every shape of the five benchmark configurations, run the
-way bench.py runs it (curve order, automatic assignment and tile width), checked
-on sampled rows and columns the oracle computes one by one.
+"""Full-size parity: every shape of the four measured configurations (square,
+prefill, irregular, high-K), run the way bench.py runs them (curve order,
+automatic dealing and tile), against the fp64 oracle.
 
-Sampled rows / columns always include the first and last, both sides of a
-tile boundary and the ragged tail, plus seeded random ones.  Tolerances are
-those of parity.py (R8 / R9 readings for bf16 output and the prefill
-distribution).
+Where 2 M N K <= 1.2e12 the whole of C is compared with the oracle's whole C,
+element by element.  Larger shapes (16384^3, 2048 x 128256 x 4096 and
+8192 x 128256 x 4096) are compared on at least 256 full rows and 256 full
+columns of C: the first and last, both sides of every multiple of 256 (and so
+of 512) -- the tile edges of every tile shape, including the ragged tail --
+and seeded random ones up to 256.  C is filled with NaN before each call and
+must come back finite everywhere, so an unwritten tile fails even where no
+sample falls.
+
+Tolerances are those of parity.py: fp32 output within the relative Frobenius
+and 2e-6 K bounds, bf16 output within one bf16 ulp of RNE(C_ref) (or the fp32
+bound where cancellation makes C_ref tiny), and for the prefill distribution
+the bound 2e-6 sum_k |A_ik| |B_kj| from the oracle's |A| @ |B|.
 """
 import numpy as np
 import pytest
@@ -15,6 +24,9 @@ from paper_2601_16294_gb300 import synth
 from parity import bf16_ulp, rel_frobenius
 
 pytestmark = pytest.mark.gpu
+
+FULL_FLOP_LIMIT = 1.2e12  # 2 M N K up to which the whole of C is checked
+EDGE = 256                # tile edges: every tile's rows and columns are multiples of 128 or 256
 
 CONFIGS = {
     "square": [(n, n, n, "uniform", "bf16", (1,)) for n in (2048, 4096, 8192, 16384)],
@@ -28,6 +40,10 @@ CONFIGS = {
 CASES = [(name, shape) for name, shapes in CONFIGS.items() for shape in shapes]
 
 
+def is_full(M, N, K):
+    return 2.0 * M * N * K <= FULL_FLOP_LIMIT
+
+
 @pytest.fixture(scope="module")
 def sfc():
     from paper_2601_16294_gb300 import build_lib
@@ -36,11 +52,26 @@ def sfc():
     return s
 
 
-def sample_indices(n, seed, extra=4):
-    idx = {0, n - 1, min(127, n - 1), min(128, n - 1), min(255, n - 1), min(256, n - 1), (n // 2)}
+def sample_indices(n, seed, want=256):
+    """Sorted indices into 0..n-1: first, last, both sides of every multiple of
+    EDGE, then seeded random ones until there are at least `want` (or n)."""
+    idx = {0, n - 1}
+    for e in range(EDGE, n, EDGE):
+        idx.update((e - 1, e))
     g = np.random.default_rng(seed)
-    idx.update(int(x) for x in g.integers(0, n, size=extra))
+    while len(idx) < min(want, n):
+        idx.add(int(g.integers(0, n)))
     return np.array(sorted(idx), dtype=np.int64)
+
+
+def test_sample_indices_cover_edges_and_count():
+    r = sample_indices(16384, seed=1)
+    assert r.size >= 256 and r[0] == 0 and r[-1] == 16383
+    for e in range(256, 16384, 256):
+        assert e - 1 in r and e in r
+    c = sample_indices(128256, seed=2)
+    assert 128255 in c and 128000 in c and 127999 in c and c.size >= 256
+    assert sample_indices(129, seed=3).size == 129  # fewer than 256: every index
 
 
 def dev(t):
@@ -48,49 +79,57 @@ def dev(t):
     return full.contiguous().cuda()[:, : t.shape[1]]
 
 
-def check_samples(oracle, got, ref, ref_mag, K, out):
-    """got / ref / ref_mag: the same sampled entries (got widened to fp64)."""
+def check(oracle, got, ref, ref_mag, K, out):
+    """got / ref / ref_mag: the same entries of C (got widened to fp64)."""
     bound = 2e-6 * ref_mag if ref_mag is not None else 2e-6 * K
     if out == "f32":
-        assert rel_frobenius(got, ref) <= 1e-5
-        assert np.all(np.abs(got - ref) <= bound)
+        rf = rel_frobenius(got, ref)
+        assert rf <= 1e-5, "relative Frobenius error %.3e" % rf
+        bad = np.abs(got - ref) > bound
+        assert not bad.any(), "%d entries beyond the bound (worst %.3e)" % (
+            int(bad.sum()), float(np.abs(got - ref).max()))
     else:
         rounded = oracle.round_bf16(ref)
         ok = (np.abs(got - rounded) <= bf16_ulp(rounded)) | (np.abs(got - ref) <= bound)
-        assert np.all(ok), "%d sampled bf16 entries off by more than 1 ulp" % int((~ok).sum())
+        assert ok.all(), "%d bf16 entries off by more than 1 ulp" % int((~ok).sum())
 
 
 @pytest.mark.parametrize("name,shape", CASES, ids=["%s-%dx%dx%d" % (n, s[0], s[1], s[2]) for n, s in CASES])
-def test_full_size_sampled(sfc, oracle, name, shape):
+def test_full_size(sfc, oracle, name, shape):
     M, N, K, kind, out, cs = shape
     lda, ldb = synth.pad8(K), synth.pad8(N)
     A, B = synth.gemm_inputs(M, N, K, kind, seed=0, lda=lda, ldb=ldb)
-    rows = sample_indices(M, seed=M + K)
-    cols = sample_indices(N, seed=N + K)
     Ac, Bc = A.contiguous(), B.contiguous()
-    ref_rows = oracle.gemm_sub_f64(Ac, Bc, rows, None)
-    ref_cols = oracle.gemm_sub_f64(Ac, Bc, None, cols)
-    mag_rows = mag_cols = None
+    absA = absB = None
     if kind == "prefill":
-        absA = Ac.float().abs().to(torch.bfloat16)
+        absA = Ac.float().abs().to(torch.bfloat16)  # exact: |x| of a bf16 value is a bf16 value
         absB = Bc.float().abs().to(torch.bfloat16)
-        mag_rows = oracle.gemm_sub_f64(absA, absB, rows, None)
-        mag_cols = oracle.gemm_sub_f64(absA, absB, None, cols)
+    full = is_full(M, N, K)
+    if full:
+        refs = [(None, None, oracle.gemm_f64(Ac, Bc), oracle.gemm_f64(absA, absB) if absA is not None else None)]
+    else:
+        rows = sample_indices(M, seed=M + K)
+        cols = sample_indices(N, seed=N + K)
+        refs = [(rows, None, oracle.gemm_sub_f64(Ac, Bc, rows, None),
+                 oracle.gemm_sub_f64(absA, absB, rows, None) if absA is not None else None),
+                (None, cols, oracle.gemm_sub_f64(Ac, Bc, None, cols),
+                 oracle.gemm_sub_f64(absA, absB, None, cols) if absA is not None else None)]
     Ad, Bd = dev(A), dev(B)
-    del A, B, Ac, Bc
+    del A, B, Ac, Bc, absA, absB
     out_dtype = torch.float32 if out == "f32" else torch.bfloat16
     C = torch.empty((M, N), dtype=out_dtype, device="cuda")
     Kt = (K + 63) // 64
-    rows_t = torch.from_numpy(rows).cuda()
-    cols_t = torch.from_numpy(cols).cuda()
     for c in [c for c in cs if c <= Kt]:
         C.fill_(float("nan"))
         sfc.gemm(Ad, Bd, C, ca_c=c)
         torch.cuda.synchronize()
         assert sfc.device_status() == 0
-        got_rows = C.index_select(0, rows_t).double().cpu().numpy()
-        got_cols = C.index_select(1, cols_t).double().cpu().numpy()
-        check_samples(oracle, got_rows, ref_rows, mag_rows, K, out)
-        check_samples(oracle, got_cols, ref_cols, mag_cols, K, out)
-        # whole output written, nothing non-finite
-        assert torch.isfinite(C).all().item()
+        assert torch.isfinite(C).all().item(), "unwritten or non-finite entries (ca_c=%d)" % c
+        for rows, cols, ref, mag in refs:
+            if rows is None and cols is None:
+                got = C.double().cpu().numpy()
+            elif rows is not None:
+                got = C.index_select(0, torch.from_numpy(rows).cuda()).double().cpu().numpy()
+            else:
+                got = C.index_select(1, torch.from_numpy(cols).cuda()).double().cpu().numpy()
+            check(oracle, got, ref, mag, K, out)

@@ -13,7 +13,7 @@ from paper_2601_16294_gb300 import synth
 pytestmark = pytest.mark.gpu
 
 CASES = 48
-TILES = ["auto", 128, 256, "pair128", "pair256", "quad256"]
+TILES = ["auto", 128, 256, "pair128", "pair256"]
 
 
 @pytest.fixture(scope="module")

@@ -80,7 +80,7 @@ def test_matches_device_call_bit_exact(sfc, M, N, K, lda, ldb, out_dtype):
 def test_layers_and_tiles(sfc):
     A, B = synth.gemm_inputs(1536, 900, 3000, "uniform", seed=3)
     Ah, Bh = host(A), host(B)
-    for ca_c, tile in ((3, "auto"), (1, 128), (2, "pair128"), (1, "quad256"), (4, 256)):
+    for ca_c, tile in ((3, "auto"), (1, 128), (2, "pair128"), (1, "pair256"), (4, 256)):
         ref = on_device(sfc, A, B, ca_c=ca_c, tile=tile)
         C = sfc.matmul_host(Ah, Bh, ca_c=ca_c, tile=tile, panels=3)
         assert torch.equal(C, ref), (ca_c, tile)

@@ -17,7 +17,7 @@ from parity import check_bf16, check_fp32
 
 pytestmark = pytest.mark.gpu
 
-TILES = [128, 256, "pair128", "pair256", "quad256"]
+TILES = [128, 256, "pair128", "pair256"]
 
 
 @pytest.fixture(scope="module")
@@ -76,7 +76,7 @@ def test_passes_compose_from_separate_calls(sfc):
     A, B = synth.gemm_inputs(M, N, K, "uniform", seed=61)
     Ad, Bd = padded(A, K), padded(B, synth.pad8(N))
     edges = [64 * (ik * 20 // 3) for ik in range(4)]
-    for tile in (128, "pair256", "quad256"):
+    for tile in (128, "pair256"):
         got = sfc.gemm(Ad, Bd, ca_c=1, k_block_factor=3, tile=tile)
         C = torch.empty(M, N, dtype=torch.float32, device="cuda")
         for ik in range(3):

@@ -85,3 +85,48 @@ def test_threads_on_separate_streams(sfc):
     for out, ref in zip(outs, refs):
         assert torch.equal(out, ref)
     assert sfc.device_status() == 0
+
+
+def test_graph_replays_beside_more_than_1024_eager_calls(sfc, oracle):
+    """A captured graph keeps whatever the capture gave its launches.  Its
+    replays on one stream run beside 1100 eager calls on another stream (more
+    than any ring of per-launch counter slots would hold), all with dynamic
+    dealing, so a counter two launches shared would drop or repeat tiles.  The
+    graph adds A B into C at every replay (C += A B, integer data: exact), so
+    a tile dropped or repeated by any replay shows in the final C; every eager
+    call writes its own output."""
+    # graph: 4096 x 2048 x 1024 on 2-SM pairs: 128 tiles for 76 pairs, so workers take tickets
+    Ag, Bg = synth.gemm_inputs(4096, 2048, 1024, "int", seed=91)
+    ref_g = torch.from_numpy(oracle.gemm_f64(Ag, Bg)).float()
+    # eager: 2048 x 2048 x 128 on single SMs: 256 tiles for 152 workers
+    Ae, Be = synth.gemm_inputs(2048, 2048, 128, "int", seed=92)
+    ref_e = torch.from_numpy(oracle.round_bf16(oracle.gemm_f64(Ae, Be))).to(torch.bfloat16).cuda()
+    Ag, Bg, Ae, Be = Ag.cuda(), Bg.cuda(), Ae.cuda(), Be.cuda()
+    n_gemms, replays, eager = 8, 64, 1100
+    Cg = [torch.zeros(4096, 2048, dtype=torch.float32, device="cuda") for _ in range(n_gemms)]
+    outs = [torch.empty(2048, 2048, dtype=torch.bfloat16, device="cuda") for _ in range(eager)]
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    with torch.cuda.stream(s1):
+        for C in Cg:  # set-up and warm-up before the capture, then back to zero
+            sfc.gemm(Ag, Bg, C, ca_c=1, tile="pair256", assign="wave", beta=1.0, stream=s1)
+            C.zero_()
+    s1.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s1):
+        for C in Cg:
+            sfc.gemm(Ag, Bg, C, ca_c=1, tile="pair256", assign="wave", beta=1.0, stream=s1)
+    for C in Cg:
+        C.zero_()
+    torch.cuda.synchronize()
+    with torch.cuda.stream(s1):
+        for _ in range(replays):
+            g.replay()
+    for C in outs:
+        sfc.gemm(Ae, Be, C, ca_c=1, tile=128, assign="wave", stream=s2)
+    torch.cuda.synchronize()
+    assert sfc.device_status() == 0
+    want = (ref_g * replays).cuda()
+    for C in Cg:
+        assert torch.equal(C, want)
+    bad = [i for i, C in enumerate(outs) if not torch.equal(C, ref_e)]
+    assert not bad, "eager calls with wrong results: %s" % bad[:10]

@@ -16,7 +16,7 @@ from paper_2601_16294_gb300 import synth
 
 pytestmark = pytest.mark.gpu
 
-TILES = [128, 256, "pair128", "pair256", "quad256"]
+TILES = [128, 256, "pair128", "pair256"]
 SLABS = [1, 2, 3, 4, 5, 6, 7, 8, 9, 13, 17]
 
 

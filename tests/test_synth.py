@@ -1,6 +1,8 @@
 """The seeded input generator shared by the tests and the benchmark: the same
-seed gives the same bits, A is drawn before B from one generator, and each
-recipe has the distribution the workloads state (CPU only)."""
+seed gives the same bits, each 2^22-element block of an operand comes from its
+own generator seeded as the module states (so the bits do not depend on the
+number of threads), and each recipe has the distribution the workloads state
+(CPU only)."""
 import pytest
 import torch
 
@@ -16,12 +18,30 @@ def test_same_seed_same_bits_other_seed_other_bits():
     assert not torch.equal(A1, A3)
 
 
-def test_a_is_drawn_before_b_from_one_generator():
-    g = torch.Generator().manual_seed(11)
-    A_ref = (torch.rand((40, 24), generator=g) * 2 - 1).to(torch.bfloat16)
-    B_ref = (torch.rand((24, 56), generator=g) * 2 - 1).to(torch.bfloat16)
-    A, B = synth.gemm_inputs(40, 56, 24, "uniform", seed=11)
-    assert torch.equal(A, A_ref) and torch.equal(B, B_ref)
+def test_blocks_follow_the_stated_seeds():
+    # A (operand 0) spans two blocks and a ragged third; B is operand 1
+    M, K, N = 3000, 3000, 24
+    A, B = synth.gemm_inputs(M, N, K, "uniform", seed=11)
+    flat = A.reshape(-1)
+    n = M * K
+    assert n > 2 * synth.BLOCK
+    for b in range(3):
+        g = torch.Generator().manual_seed(((11 * 1000003 + 0) * 1000003 + b) % (1 << 63))
+        lo, hi = b * synth.BLOCK, min(n, (b + 1) * synth.BLOCK)
+        want = (torch.rand(hi - lo, generator=g) * 2 - 1).to(torch.bfloat16)
+        assert torch.equal(flat[lo:hi], want)
+    g = torch.Generator().manual_seed((11 * 1000003 + 1) * 1000003)
+    assert torch.equal(B.reshape(-1), (torch.rand(K * N, generator=g) * 2 - 1).to(torch.bfloat16))
+    # the prefill weights: N(0, 1) draws times 0.02, rounded once
+    _, Bp = synth.gemm_inputs(8, 16, 32, "prefill", seed=3)
+    g = torch.Generator().manual_seed((3 * 1000003 + 1) * 1000003)
+    assert torch.equal(Bp.reshape(-1), (torch.randn(32 * 16, generator=g) * 0.02).to(torch.bfloat16))
+
+
+def test_bits_do_not_depend_on_threads():
+    one = synth.draw((2100, 4100), 9, 1, "normal", 0.02, threads=1)
+    many = synth.draw((2100, 4100), 9, 1, "normal", 0.02, threads=7)
+    assert torch.equal(one.view(torch.int16), many.view(torch.int16))
 
 
 def test_uniform_recipe():
