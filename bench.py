@@ -118,6 +118,9 @@ def parse_args():
     ap.add_argument("--assign", choices=("auto", "wave", "wave_static", "segment"), default="auto")
     ap.add_argument("--sizes", type=str, default=None,
                     help="square workload only: comma-separated sizes instead of the full sweep")
+    ap.add_argument("--shapes", type=str, default=None,
+                    help="comma-separated MxNxK shapes instead of the workload's (uniform [-1,1] inputs, output "
+                         "per --out, bf16 by default; K-layer counts per --ca-c, else 1,2,4,8)")
     ap.add_argument("--ca-c", type=int, default=None, help="force one K-layer count for every shape")
     ap.add_argument("--b-layout", choices=("kn", "nk"), default="kn",
                     help="storage of B: K x N row-major (the paper's), or N x K (a linear layer's weight)")
@@ -147,9 +150,17 @@ def parse_args():
 
 
 def workload_shapes(args):
+    if getattr(args, "shapes", None):
+        out = args.out if args.out != "workload" else "bf16"
+        shapes = []
+        for item in args.shapes.split(","):
+            M, N, K = (int(x) for x in item.lower().split("x"))
+            shapes.append(_shape(M, N, K, "uniform", out, CS if args.ca_c is None else (args.ca_c,)))
+        return shapes
     shapes = [dict(s) for s in WORKLOADS[args.workload]["shapes"]]
     if args.sizes:
-        if args.workload != "square":
+        # square shapes of the given sizes (with the default workload, or the square one)
+        if args.workload not in ("square", "configs"):
             raise SystemExit("--sizes applies to the square workload only")
         shapes = [_shape(int(n), int(n), int(n)) for n in args.sizes.split(",")]
     if args.ca_c is not None:
@@ -159,6 +170,14 @@ def workload_shapes(args):
         for s in shapes:
             s["out"] = args.out
     return shapes
+
+
+def describe(args) -> str:
+    if getattr(args, "shapes", None):
+        return "shapes %s, uniform [-1,1] bf16 inputs" % args.shapes
+    if args.sizes:
+        return "square sweep sizes %s" % args.sizes
+    return WORKLOADS[args.workload]["desc"]
 
 
 def kernel_sha() -> str:
@@ -374,7 +393,11 @@ def run_ours(args, rank, local, world):
     tuned = {}
     if not args.no_tune and args.k_block_factor == 1:
         for i, m in enumerate(mats):
-            tuned[i] = sfc.tune(m["Ad"], m["Bd"], m["C"], max_layers=max(m["s"]["cs"]), max_kbf=1,
+            # the configured layer counts, and the time model's own count, so that the library's
+            # choice (ca_c = 0) is measured too
+            model_c = sfc.plan(m["s"]["M"], m["s"]["N"], m["s"]["K"], 0, out_dtype=m["C"].dtype,
+                               in_dtype=m["Ad"].dtype, b_layout=args.b_layout)[1]
+            tuned[i] = sfc.tune(m["Ad"], m["Bd"], m["C"], max_layers=max(max(m["s"]["cs"]), model_c), max_kbf=1,
                                 b_layout=args.b_layout, stream=stream)
         torch.cuda.synchronize()
 
@@ -455,6 +478,9 @@ def run_ours(args, rank, local, world):
     per_launch = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
                    for _ in mats] for _ in range(args.steps)]
     torch.cuda.synchronize()
+    # one untimed step first: the recorded launches then find the device busy with earlier work,
+    # so each event pair holds the launch's device time, not the host's issue of the first call
+    step()
     for k in range(args.steps):
         step(per_launch[k])
     torch.cuda.synchronize()
@@ -536,7 +562,8 @@ def run_ours(args, rank, local, world):
     try:
         with open(TRAFFIC_FILE) as f:
             tr = json.load(f)
-        if tr.get("kernel_sha") == kernel_sha() and tr.get("workload") == args.workload and not args.sizes:
+        if (tr.get("kernel_sha") == kernel_sha() and tr.get("workload") == args.workload and not args.sizes
+                and not args.shapes):
             traffic = tr["dram_bytes_per_launch"]
     except Exception:
         traffic = None
@@ -571,7 +598,7 @@ def run_ours(args, rank, local, world):
         return kbf + (1 if c > 1 or (kbf > 1 and m["C"].dtype != torch.float32) else 0)
 
     launches = args.steps * sum(launches_per_call(m) for m in mats)
-    desc = WORKLOADS[args.workload]["desc"] if not args.sizes else "square sweep sizes %s" % args.sizes
+    desc = describe(args)
     result = {
         "metric": METRIC, "value": round(value, 1), "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4), "higher_is_better": True,
@@ -634,6 +661,14 @@ def run_cublas_compare(args, mats, stream, call):
                 cublas(m)
     except Exception as e:  # e.g. a shape cuBLAS's 8-bit GEMM does not take
         return {"unavailable": "cuBLAS comparison failed: %s" % str(e).splitlines()[0][:200]}
+    # every step of both arms is issued before one synchronisation (the host runs ahead of the
+    # device, so each event pair holds device time only); one untimed step of each arm goes first
+    torch.cuda.synchronize()
+    for m in mats:
+        call(m, m["c"])
+    for m in mats:
+        cublas(m)
+    evs = []
     for k in range(steps):
         for which in (0, 1):
             ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in mats]
@@ -644,9 +679,11 @@ def run_cublas_compare(args, mats, stream, call):
                 else:
                     cublas(m)
                 ev[i][1].record(stream)
-            torch.cuda.synchronize()
-            for i in range(len(mats)):
-                t[i][which] += ev[i][0].elapsed_time(ev[i][1])
+            evs.append((which, ev))
+    torch.cuda.synchronize()
+    for which, ev in evs:
+        for i in range(len(mats)):
+            t[i][which] += ev[i][0].elapsed_time(ev[i][1])
     fl = [2.0 * m["s"]["M"] * m["s"]["N"] * m["s"]["K"] * steps for m in mats]
     ours, cub = sum(x[0] for x in t), sum(x[1] for x in t)
     return {"cublas_tflops": round(sum(fl) / (cub * 1e-3) / 1e12, 1),
@@ -654,7 +691,8 @@ def run_cublas_compare(args, mats, stream, call):
             "per_shape": [{"M": m["s"]["M"], "N": m["s"]["N"], "K": m["s"]["K"],
                            "ours": round(f / (x[0] * 1e-3) / 1e12, 1), "cublas": round(f / (x[1] * 1e-3) / 1e12, 1)}
                           for m, f, x in zip(mats, fl, t)],
-            "note": "alternating steps, same stream; cuBLAS output is bf16 (fp32 rows: bf16 GEMM then cast)"}
+            "note": "alternating steps, same stream, issued ahead of the device (one synchronisation at the end); "
+                    "cuBLAS output is bf16 (fp32 rows: bf16 GEMM then cast)"}
 
 
 def run_e2e(args, mats, stream, world):
@@ -806,7 +844,7 @@ def run_reference(args, rank, world):
     value = flops / secs / 1e12
     cores = int(os.environ["OMP_NUM_THREADS"])
     sample = "%d evenly spaced rows of C per shape per step" % rows
-    desc = WORKLOADS[args.workload]["desc"] if not args.sizes else "square sweep sizes %s" % args.sizes
+    desc = describe(args)
     return {"impl": "reference", "metric": METRIC, "value": round(value, 6), "unit": "TFLOP/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(1e3 * secs / args.steps, 2),
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
