@@ -317,7 +317,11 @@ def make_inputs(s, synth, torch, ab="bf16"):
         return full.contiguous().cuda()[:, : t.shape[1]]
 
     out_dtype = torch.float32 if s["out"] == "f32" else torch.bfloat16
-    C = torch.empty((s["M"], s["N"]), dtype=out_dtype, device="cuda")
+    # C's rows padded to 16 bytes like those of A and B (the caller's layout; unpadded rows
+    # take the library's slower direct-store epilogue, which the parity tests cover)
+    esz = 4 if s["out"] == "f32" else 2
+    ldc = (s["N"] * esz + 15) // 16 * 16 // esz
+    C = torch.empty((s["M"], ldc), dtype=out_dtype, device="cuda")[:, : s["N"]]
     if s.get("shared"):
         def operand(rows, cols, seed):
             key = (rows, cols, seed)
@@ -456,10 +460,14 @@ def run_ours(args, rank, local, world):
     time.sleep(0.2 if clocks.proc else 0)
     barrier(world)
     torch.cuda.synchronize()
+    # an NVTX range around the timed steps lets a profiler capture exactly them
+    # (ncu --nvtx --nvtx-include "sfc_timed_steps/")
+    torch.cuda.nvtx.range_push("sfc_timed_steps")
     t0.record(stream)
     for k in range(args.steps):
         step()
     t1.record(stream)
+    torch.cuda.nvtx.range_pop()
     torch.cuda.synchronize()
     barrier(world)
     clock_info = clocks.stop()

@@ -338,20 +338,27 @@ int64_t auto_layer_cap(int64_t M, int64_t N, int64_t K, int ab = SFC_AB_BF16) {
     return cap < 1 ? 1 : cap;
 }
 
-double plan_cost(int64_t M, int64_t N, int64_t K, int c, int v, const Machine& m, int out_bytes, int ab) {
+// The model's tensor time and DRAM time of the GEMM launch (the reduction not included).
+void gemm_times(int64_t M, int64_t N, int64_t K, int c, int v, const Machine& m, int out_bytes, int ab,
+                double* t_tensor_out, double* t_dram_out) {
     const int64_t items = ceil_div(M, variant_bm(v)) * ceil_div(N, variant_bn(v)) * c;
     const int64_t waves = ceil_div(items, m.workers[v]);
-    // a slab of 8-bit inputs holds twice the k at twice the rate: the same time per slab
     const int64_t slabs = ceil_div(ceil_div(K, slab_k(ab)), c);
     const double slab_ns = 128.0 * variant_bn(v) * kBK * 2.0 / (8192.0 * kEff[v]) / m.sm_ghz;
-    const double t_tensor = static_cast<double>(waves) * static_cast<double>(slabs) * slab_ns;
-    const double mn = static_cast<double>(M) * static_cast<double>(N);
+    *t_tensor_out = static_cast<double>(waves) * static_cast<double>(slabs) * slab_ns;
     const double ab_bytes = in_bytes(ab) * (static_cast<double>(M) * K + static_cast<double>(K) * N);
     const double out_gemm = (c > 1) ? 4.0 * c * static_cast<double>(M) * static_cast<double>(ws_ld(N))
-                                    : out_bytes * mn;
-    const double t_dram = (ab_bytes + out_gemm) / m.hbm_bytes_per_ns;
+                                    : out_bytes * static_cast<double>(M) * static_cast<double>(N);
+    *t_dram_out = (ab_bytes + out_gemm) / m.hbm_bytes_per_ns;
+}
+
+double plan_cost(int64_t M, int64_t N, int64_t K, int c, int v, const Machine& m, int out_bytes, int ab) {
+    double t_tensor = 0.0, t_dram = 0.0;
+    gemm_times(M, N, K, c, v, m, out_bytes, ab, &t_tensor, &t_dram);
     double t = t_tensor > t_dram ? t_tensor : t_dram;
-    if (c > 1) t += kReduceLaunchNs + (4.0 * c + out_bytes) * mn / m.hbm_bytes_per_ns;
+    if (c > 1)
+        t += kReduceLaunchNs + (4.0 * c + out_bytes) * static_cast<double>(M) * static_cast<double>(N) /
+                                   m.hbm_bytes_per_ns;
     return t;
 }
 

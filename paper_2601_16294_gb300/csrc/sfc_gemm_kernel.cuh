@@ -247,34 +247,6 @@ __device__ __forceinline__ float cvt_out<float>(float v) { return v; }
 template <>
 __device__ __forceinline__ __nv_bfloat16 cvt_out<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
 
-// Store 32 consecutive columns v[0..31] of one row, starting at column col0.
-template <typename OutT>
-__device__ __forceinline__ void store_chunk(OutT* row_ptr, int64_t col0, int64_t N, const float* v, bool vec) {
-    if (vec && col0 + 32 <= N) {
-        if constexpr (sizeof(OutT) == 4) {
-            float4* dst = reinterpret_cast<float4*>(row_ptr + col0);
-#pragma unroll
-            for (int j = 0; j < 8; ++j) dst[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
-        } else {
-            uint4* dst = reinterpret_cast<uint4*>(row_ptr + col0);
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-                uint32_t w[4];
-#pragma unroll
-                for (int h = 0; h < 4; ++h) {
-                    __nv_bfloat162 b = __floats2bfloat162_rn(v[8 * j + 2 * h], v[8 * j + 2 * h + 1]);
-                    w[h] = *reinterpret_cast<uint32_t*>(&b);
-                }
-                dst[j] = make_uint4(w[0], w[1], w[2], w[3]);
-            }
-        }
-    } else {
-#pragma unroll
-        for (int j = 0; j < 32; ++j)
-            if (col0 + j < N) row_ptr[col0 + j] = cvt_out<OutT>(v[j]);
-    }
-}
-
 // beta * C_in + bias for columns [col0, col0 + n) of one row of K layer
 // `layer`, added into v (fp32, before rounding to the output type).  Columns
 // >= N are left alone.
@@ -618,13 +590,31 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
                 }
             }
         } else {
-            const int64_t row = warp_row + lane;
-            if (row < p.M) {
-                OutT* row_ptr = out + static_cast<int64_t>(w.layer) * p.layer_stride + row * p.ldo;
+            // C rows the TMA cannot store (C's base or row stride not a multiple of 16 bytes): each
+            // 32-row box is staged in the warp's buffer as for the TMA, then read back so that one
+            // warp store covers consecutive columns of one row (of two rows for fp32), not one
+            // value in each of 32 rows
+            constexpr int kCols = box_cols<OutT>();    // 32 bf16 or 16 fp32 columns: 64 bytes per row
+            constexpr int kRowsPerStore = 32 / kCols;  // rows one warp store covers
+            uint8_t* box = staging + ew * kStageBufBytes;
+            OutT* base = out + static_cast<int64_t>(w.layer) * p.layer_stride;
+            const int c = lane % kCols;                // this lane's column within the box
+            const int cbyte = c * static_cast<int>(sizeof(OutT));
 #pragma unroll
-                for (int g = 0; g < kEpiCols / 32; ++g) {
-                    if (affine) apply_affine<OutT, 32>(p, row, col_base + g * 32, w.layer, run + g * 32);
-                    store_chunk<OutT>(row_ptr, col_base + g * 32, p.N, run + g * 32, p.vec_store != 0);
+            for (int g = 0; g < kEpiCols / kCols; ++g) {  // unrolled: run[] stays in registers
+                const int64_t col0 = col_base + g * kCols;
+                if (col0 >= p.N) break;  // warp-uniform
+                if (affine) apply_affine<OutT, kCols>(p, warp_row + lane, col0, w.layer, run + g * kCols);
+                __syncwarp();  // the previous box has been read back by every lane
+                stage_row<OutT>(box, lane, run + g * kCols);
+                __syncwarp();
+                const int64_t col = col0 + c;
+#pragma unroll 4
+                for (int r0 = 0; r0 < 32; r0 += kRowsPerStore) {
+                    const int r = r0 + lane / kCols;
+                    const int64_t row = warp_row + r;
+                    const int off = r * 64 + (((cbyte >> 4) ^ ((r >> 1) & 3)) << 4) + (cbyte & 15);
+                    if (row < p.M && col < p.N) base[row * p.ldo + col] = *reinterpret_cast<const OutT*>(box + off);
                 }
             }
         }
