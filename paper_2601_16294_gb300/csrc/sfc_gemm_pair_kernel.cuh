@@ -23,8 +23,9 @@
 //
 // Waits are bounded as in the single-SM kernel.  The pair meets at a cluster
 // barrier after set-up (barriers initialised before any remote signal) and
-// before exit (no CTA leaves while its peer may still signal it); then both
-// CTAs free their tensor memory.
+// before exit (no CTA leaves while its peer may still signal it; each warp
+// arrives as soon as its role is done); then both CTAs free their tensor
+// memory.
 #pragma once
 
 #include "sfc_gemm_kernel.cuh"
@@ -82,14 +83,13 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
     src.q_empty0 = ptx::map_to_cta(B.q_empty(0), 0);
     src.q_entry = reinterpret_cast<volatile int*>(smem + L::kQueueOffset);
     // CTA 0's scheduler deals the cluster's items.  The first needs no memory
-    // at all: it is decoded while the other warps set up and published before
-    // the wait for the previous grid.
+    // at all and no message: the scheduler warp of each CTA decodes it into its
+    // own queue's slot 0 while the other warps set up.
     const bool sched_thread = (rank == 0 && warp == scheduler_warp(BN) && lane == 0);
     int item0 = -1;
-    QueueEntry entry0{};
-    if (sched_thread) {
+    if (warp == scheduler_warp(BN) && lane == 0) {
         item0 = sched_next(src, 0, p);
-        entry0 = sched_entry(item0, p);
+        sched_local_first(src, sched_entry(item0, p));
     }
 
     if (threadIdx.x == 0) {
@@ -129,7 +129,7 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
     ptx::tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
 
-    if (sched_thread) sched_send(src, 0, entry0, kCtas);
+    if (sched_thread) sched_mark_first(src, kCtas);
     ptx::pdl_wait();  // on-chip set-up above overlaps the previous kernel; global memory only after it
 
     if (warp == 0) {
@@ -248,15 +248,20 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
     } else if (warp < scheduler_warp(BN)) {
         run_epilogue<BN, OutT, true>(p, B, tmem_base, abort_flag, src, kItemRows,
                                      static_cast<int>(r * 128), warp, lane, &tmap_c,
-                                     smem + L::kStagingOffset, pair_leader);
+                                     smem + L::kStagingOffset, smem, L::kRingBytes / kEpiWarps, pair_leader);
     } else if (sched_thread) {
         // -------------------------------------------------------- scheduler
         run_scheduler(src, item0, p, B, abort_flag, kCtas);
     }
 
+    // No CTA leaves while another CTA of the cluster may still signal it: each warp arrives at
+    // the cluster barrier as soon as its role is done (its remote signals are released then),
+    // and the block waits for the whole cluster before freeing its tensor memory.
+    __syncwarp();
+    ptx::cluster_arrive();
     ptx::tc_fence_before();
     __syncthreads();
-    ptx::cluster_sync();  // no CTA leaves while another CTA of the cluster may still signal it
+    ptx::cluster_wait();
     ptx::tc_fence_after();
     if (warp == 1) ptx::tmem_dealloc_pair(tmem_base, kTmemCols);
 }

@@ -24,7 +24,7 @@ def lib():
 def declared_functions():
     text = open(HEADER).read()
     text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
-    return sorted(set(re.findall(r"^\s*(?:int|size_t|void)\s+\**(sfc_\w+)\s*\(", text, flags=re.M)))
+    return sorted(set(re.findall(r"^\s*(?:int|size_t|void|long long)\s+\**(sfc_\w+)\s*\(", text, flags=re.M)))
 
 
 def test_header_declares_the_boundary():
