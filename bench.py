@@ -47,6 +47,12 @@ KERNEL_SOURCES = ("paper_2601_16294_gb300/csrc/sfc_gemm_kernel.cuh", "paper_2601
                   "paper_2601_16294_gb300/csrc/sfc_curve.cuh", "paper_2601_16294_gb300/csrc/sfc_gemm.cu",
                   "paper_2601_16294_gb300/csrc/sfc_gemm_pair_kernel.cuh")
 TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic_square_sweep.json")
+# per-shape DRAM bytes of the GEMM launches of a workload's timed step (one ncu capture), keyed
+# like the square record by the kernel sources' hash
+TRAFFIC_FILES = {"configs": os.path.join(ROOT, "profiles", "traffic_configs.json")}
+# the kernel name a tile label launches (the record says which kernel each capture measured)
+TILE_KERNEL = {"pair256": "sfc_gemm_pair_kernel<256", "pair128": "sfc_gemm_pair_kernel<128",
+               "256": "sfc_gemm_kernel<256", "128": "sfc_gemm_kernel<128"}
 CS = (1, 2, 4, 8)
 
 
@@ -568,11 +574,25 @@ def run_ours(args, rank, local, world):
         achieved = flops_step * args.steps / (tot_ms * 1e-3) / 1e12
     traffic = None
     try:
-        with open(TRAFFIC_FILE) as f:
+        with open(TRAFFIC_FILES.get(args.workload, TRAFFIC_FILE)) as f:
             tr = json.load(f)
         if (tr.get("kernel_sha") == kernel_sha() and tr.get("workload") == args.workload and not args.sizes
                 and not args.shapes):
-            traffic = tr["dram_bytes_per_launch"]
+            if "per_shape" in tr:
+                # the one-layer calls of this run, each matched to the capture of the same shape
+                # and the same kernel; any call without such a capture leaves traffic unknown
+                got = []
+                for row in per_shape:
+                    if row["ca_c"] != 1:
+                        continue
+                    want = TILE_KERNEL.get(str(row["tile"]), "?")
+                    hit = [e for e in tr["per_shape"] if (e["M"], e["N"], e["K"]) == (row["M"], row["N"], row["K"])
+                           and want in e["kernel"]]
+                    got.append(hit[0]["dram_bytes"] if hit else None)
+                if got and all(g is not None for g in got):
+                    traffic = int(round(sum(got) / len(got)))
+            else:
+                traffic = tr["dram_bytes_per_launch"]
     except Exception:
         traffic = None
     # burst peak for a short timed region, sustained (power-capped) peak for a long one;

@@ -169,7 +169,7 @@ size_t sfc_gemm_workspace_size(int64_t M, int64_t N, int64_t K, int ca_c);
  * sum is restarted every 4096 values of k and the partial sums are added with
  * round-to-nearest fp32 adds, which bounds the error growth of very long K.
  * Memory: besides the layer workspace, a call whose items outnumber the
- * workers (dynamic dealing over more than one wave) takes a 16 KB counter area
+ * workers (dynamic dealing over more than one wave) takes a 256-byte counter
  * from the library's stream-ordered ticket pool and frees it after its kernels
  * (both kept by the pools for the next call).  The counter's words are tagged
  * with a per-call value, so nothing is written to clear it before the kernels.
@@ -390,7 +390,7 @@ int sfc_num_workers(void);
  * handed all device memory to its own arena.  For them this entry point takes
  * the fp32 partial copies of C (ca_c > 1) and the workers' item counter from a
  * fixed scratch area compiled into the library: SFC_NOALLOC_SCRATCH_BYTES
- * bytes for the partials plus 16 KB for the counter, device memory that
+ * bytes for the partials plus 256 bytes for the counter, device memory that
  * every GPU which loads the library holds until the process exits.  It calls
  * no cudaMalloc, cudaFree or allocating library routine, and takes nothing
  * from the library's pools.
@@ -523,27 +523,6 @@ int sfc_debug_pool_used_high(size_t *used_high_bytes, int reset);
  */
 int sfc_debug_force_timeout(const void *A, const void *B, void *C, int limit_ms, void *stream);
 
-/*
- * sfc_debug_set_fused -- test hook: enable = 1 lets a call with 2..4 K layers
- * whose items all fit in one wave of workers sum its layers inside the GEMM
- * launch (each 32 x 128 region of a tile is summed by one of the tile's layer
- * workers, in layer order, the order of the reduction kernel, so the bits are
- * the same); enable = 0 (the default: measured slower on GB300) sends every
- * K-layer call through the reduction kernel.
- * The setting is process-wide and applies to calls made after it.  Returns
- * the previous setting (0 or 1), or SFC_ERR_INVALID_ARG for another value.
- * No counterpart in the paper: it exists so that tests can compare the two
- * reductions bit for bit.
- */
-int sfc_debug_set_fused(int enable);
-
-/*
- * sfc_debug_fused_launches -- test hook: how many GEMM launches of this
- * process (all devices) summed their K layers inside the launch so far.  Tests
- * read it before and after a call to learn which reduction the call took.  No
- * counterpart in the paper.
- */
-long long sfc_debug_fused_launches(void);
 
 #ifdef __cplusplus
 }

@@ -62,8 +62,7 @@ EXPORTS = ("sfc_tile_order", "sfc_tile_order_device", "sfc_gemm_workspace_size",
            "sfc_get_device_status", "sfc_last_cuda_error", "sfc_num_workers", "sfc_debug_force_timeout",
            "sfc_gemm_noalloc", "sfc_gemm_plan", "sfc_release", "sfc_gemm_ex2", "sfc_gemm_host", "sfc_gemm_ex3",
            "sfc_gemm_workspace_size2", "sfc_gemm_tune", "sfc_gemm_tune_forget",
-           "sfc_gemm_tune_lookup", "sfc_mma_peak", "sfc_debug_pool_used_high", "sfc_gemm_plan_desc",
-           "sfc_debug_set_fused", "sfc_debug_fused_launches")
+           "sfc_gemm_tune_lookup", "sfc_mma_peak", "sfc_debug_pool_used_high", "sfc_gemm_plan_desc")
 NOALLOC_SCRATCH_BYTES = 32 << 20
 
 
@@ -126,13 +125,11 @@ def load():
         lib.sfc_mma_peak.argtypes = [i32, vp, vp, vp]
         lib.sfc_debug_pool_used_high.argtypes = [vp, i32]
         lib.sfc_gemm_plan_desc.argtypes = [vp, i64, i64, i64, i32, i32, i32, i32, vp, vp, vp]
-        lib.sfc_debug_set_fused.argtypes = [i32]
-        lib.sfc_debug_fused_launches.argtypes = []
+
         lib.sfc_gemm_workspace_size2.restype = sz
         for name in EXPORTS:
-            if name not in ("sfc_gemm_workspace_size", "sfc_gemm_workspace_size2", "sfc_debug_fused_launches"):
+            if name not in ("sfc_gemm_workspace_size", "sfc_gemm_workspace_size2"):
                 getattr(lib, name).restype = ctypes.c_int
-        lib.sfc_debug_fused_launches.restype = ctypes.c_longlong
         _lib = lib
         return lib
 
@@ -388,20 +385,6 @@ def device_status(stream=None) -> int:
 def debug_force_timeout(A, B, C, limit_ms: int = 20, stream=None) -> int:
     return load().sfc_debug_force_timeout(ctypes.c_void_p(A.data_ptr()), ctypes.c_void_p(B.data_ptr()),
                                           ctypes.c_void_p(C.data_ptr()), int(limit_ms), _stream_ptr(stream))
-
-
-def set_fused(enable: bool) -> bool:
-    """Test hook: whether K-layer calls that fit one wave sum their layers inside the GEMM
-    launch (the default) or through the reduction kernel.  Returns the previous setting."""
-    rc = load().sfc_debug_set_fused(1 if enable else 0)
-    if rc < 0:
-        _check(rc, "sfc_debug_set_fused")
-    return bool(rc)
-
-
-def fused_launches() -> int:
-    """Test hook: GEMM launches of this process that summed their K layers in the launch."""
-    return int(load().sfc_debug_fused_launches())
 
 
 def gemm_host(A_host, B_host, C_host=None, *, ca_c: int = 0, out_dtype=None, tile=0, b_layout: str = "kn",

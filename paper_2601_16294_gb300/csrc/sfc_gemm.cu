@@ -52,16 +52,7 @@ constexpr int kMaxLayers = 4096;  // keeps the kernels' layer arithmetic in 32 b
 constexpr int kMaxKBlocks = 64;   // k_block_factor bound (keeps the kernels' pass arithmetic in 32 bits)
 constexpr uint64_t kDefaultTimeoutNs = 2000000000ull;  // 2 s per wait
 
-// one call's ticket allocation: the two 64-bit counter words, then (from kFlagOffset) the
-// flags of K layers summed in the launch
-constexpr size_t kTicketBytes = 16384;
-constexpr size_t kFlagOffset = 64;
-constexpr int kFusedMaxLayers = 4;  // K layers a launch may sum itself (above: the reduction kernel)
-// Off by default: measured slower than the reduction kernel on GB300 (the two-kernel path with
-// programmatic dependent launch hides the reduction's launch; the in-launch sum serialises the
-// owners' waits behind the slowest contributor).  sfc_debug_set_fused(1) switches it on.
-std::atomic<int> g_fused_enabled{0};
-std::atomic<long long> g_fused_launches{0};  // GEMM launches that summed their K layers themselves
+constexpr size_t kTicketBytes = 256;  // one call's ticket allocation (two 64-bit counter words used)
 constexpr double kSlabClockGhz = 1.9;     // SM clock the time model's slab times assume
 constexpr double kHbmBytesPerNs = 6700.0; // attainable DRAM bandwidth of GB300 (a copy's, GB/s)
 
@@ -110,13 +101,10 @@ constexpr int variant_smem(int v) {
                              : pair_smem<256, kStagesPair256>();
 }
 
-// attr must hold three entries.  With `pdl` the kernel may begin launching
+// attr must hold two entries.  With `pdl` the kernel may begin launching
 // while the previous kernel in the stream finishes (programmatic dependent
-// launch); the kernels wait for it before touching global memory.  With
-// `cooperative` every block of the grid is resident at once (launches whose
-// blocks wait for one another: K layers summed in the launch).
-cudaLaunchConfig_t launch_config(int v, int grid, cudaStream_t s, cudaLaunchAttribute* attr, bool pdl,
-                                 bool cooperative = false) {
+// launch); the kernels wait for it before touching global memory.
+cudaLaunchConfig_t launch_config(int v, int grid, cudaStream_t s, cudaLaunchAttribute* attr, bool pdl) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid, 1, 1);
     cfg.blockDim = dim3(block_threads(variant_bn(v)), 1, 1);
@@ -134,11 +122,6 @@ cudaLaunchConfig_t launch_config(int v, int grid, cudaStream_t s, cudaLaunchAttr
     if (pdl) {
         attr[cfg.numAttrs].id = cudaLaunchAttributeProgrammaticStreamSerialization;
         attr[cfg.numAttrs].val.programmaticStreamSerializationAllowed = 1;
-        ++cfg.numAttrs;
-    }
-    if (cooperative) {
-        attr[cfg.numAttrs].id = cudaLaunchAttributeCooperative;
-        attr[cfg.numAttrs].val.cooperative = 1;
         ++cfg.numAttrs;
     }
     return cfg;
@@ -220,7 +203,7 @@ int device_setup(DeviceInfo** info) {
                 d.workers[v] = d.num_sms;
                 continue;
             }
-            cudaLaunchAttribute attr[3];
+            cudaLaunchAttribute attr[2];
             cudaLaunchConfig_t cfg = launch_config(v, d.num_sms, nullptr, attr, false);
             int clusters = 0;
             e = cudaOccupancyMaxActiveClusters(&clusters, Kernels<float, false>::get(v), &cfg);
@@ -327,14 +310,9 @@ int64_t ws_ld(int64_t N) { return (N + 3) / 4 * 4; }
 //     the c fp32 partial copies of C: the launch takes at least those bytes /
 //     DRAM bandwidth, and the longer of the two times is the GEMM's;
 //   - for c > 1 the reduction adds its launch and its own DRAM traffic (the c
-//     copies read back, C written); where the launch sums its few layers itself
-//     (one item per worker) each SM instead stores and reads back (c-1)/c of
-//     its fp32 tile through L2 at the per-SM intake rate, after a fixed
-//     hand-over latency.
+//     copies read back, C written).
 // The tile and layer count with the least time win (ties keep fewer layers).
 constexpr double kReduceLaunchNs = 3000.0;   // reduction kernel launch and ramp
-constexpr double kFusedHandoverNs = 1500.0;  // flag wait, partial loads' latency, final stores
-constexpr double kIntakeBytesPerClk = 64.0;  // one SM's operand intake from L2
 // relative tensor-pipe efficiency measured on GB300, back to back at 8192 x
 // 8192 x 4096 and 6144^2 x 4096 (256-wide tiles feed the tensor core with fewer
 // shared-memory bytes per flop)
@@ -356,13 +334,6 @@ int64_t auto_layer_cap(int64_t M, int64_t N, int64_t K, int ab = SFC_AB_BF16) {
     return cap < 1 ? 1 : cap;
 }
 
-// Whether a call of c layers on variant v sums them inside the GEMM launch (C assumed aligned).
-bool fused_layers(int64_t M, int64_t N, int c, int v, const Machine& m) {
-    const int64_t items = ceil_div(M, variant_bm(v)) * ceil_div(N, variant_bn(v)) * c;
-    return c >= 2 && c <= kFusedMaxLayers && items <= m.workers[v] &&
-           g_fused_enabled.load(std::memory_order_relaxed) != 0;
-}
-
 // The model's tensor time and DRAM time of the GEMM launch (the reduction not included).
 void gemm_times(int64_t M, int64_t N, int64_t K, int c, int v, const Machine& m, int out_bytes, int ab,
                 double* t_tensor_out, double* t_dram_out) {
@@ -372,11 +343,8 @@ void gemm_times(int64_t M, int64_t N, int64_t K, int c, int v, const Machine& m,
     const double slab_ns = 128.0 * variant_bn(v) * kBK * 2.0 / (8192.0 * kEff[v]) / m.sm_ghz;
     *t_tensor_out = static_cast<double>(waves) * static_cast<double>(slabs) * slab_ns;
     const double ab_bytes = in_bytes(ab) * (static_cast<double>(M) * K + static_cast<double>(K) * N);
-    const double mn = static_cast<double>(M) * static_cast<double>(N);
-    const double out_gemm = (c <= 1)                       ? out_bytes * mn
-                            : fused_layers(M, N, c, v, m) ? 4.0 * (c - 1) * M * static_cast<double>(ws_ld(N)) +
-                                                                out_bytes * mn
-                                                          : 4.0 * c * M * static_cast<double>(ws_ld(N));
+    const double out_gemm = (c > 1) ? 4.0 * c * static_cast<double>(M) * static_cast<double>(ws_ld(N))
+                                    : out_bytes * static_cast<double>(M) * static_cast<double>(N);
     *t_dram_out = (ab_bytes + out_gemm) / m.hbm_bytes_per_ns;
 }
 
@@ -384,11 +352,7 @@ double plan_cost(int64_t M, int64_t N, int64_t K, int c, int v, const Machine& m
     double t_tensor = 0.0, t_dram = 0.0;
     gemm_times(M, N, K, c, v, m, out_bytes, ab, &t_tensor, &t_dram);
     double t = t_tensor > t_dram ? t_tensor : t_dram;
-    if (c > 1 && fused_layers(M, N, c, v, m)) {
-        // each SM stores (c-1)/c of its 128 x bn fp32 partial tile and reads as much back
-        const double part_ns = 128.0 * variant_bn(v) * 4.0 / (kIntakeBytesPerClk * m.sm_ghz);
-        t += kFusedHandoverNs + 2.0 * (c - 1) / c * part_ns;
-    } else if (c > 1) {
+    if (c > 1) {
         t += kReduceLaunchNs + (4.0 * c + out_bytes) * static_cast<double>(M) * static_cast<double>(N) /
                                    m.hbm_bytes_per_ns;
     }
@@ -480,9 +444,9 @@ size_t workspace_bytes_for(int64_t M, int64_t N, int c, int kbf, int c_dtype) {
 
 template <typename OutT>
 cudaError_t launch_gemm(int v, bool f8, const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc,
-                        const GemmParams& p, int grid, cudaStream_t s, bool pdl = true) {
-    cudaLaunchAttribute attr[3];
-    cudaLaunchConfig_t cfg = launch_config(v, grid, s, attr, pdl, p.fused != 0);
+                        const GemmParams& p, int grid, cudaStream_t s) {
+    cudaLaunchAttribute attr[2];
+    cudaLaunchConfig_t cfg = launch_config(v, grid, s, attr, true);
     cudaError_t e = cudaLaunchKernelEx(&cfg, f8 ? Kernels<OutT, true>::get(v) : Kernels<OutT, false>::get(v), ta, tb,
                                        tc, p);
     return e;
@@ -748,24 +712,12 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
     p.kbf = 1;
     p.pass = 0;
     p.accumulate = 0;
-    p.fused = 0;
-    p.flags = nullptr;
     const int64_t workers = dev->workers[v];
     const int64_t used = p.num_items < workers ? p.num_items : workers;
     const int grid = static_cast<int>(variant_cluster(v) * used);
     // one item per worker: dynamic dealing would hand worker w item w and nothing else, which is
     // the static wave deal (the same items, the same bits) without a counter
     if (p.dynamic && p.num_items <= workers) p.dynamic = 0;
-    // K layers summed inside the GEMM launch instead of by the reduction kernel: every worker
-    // holds one item (all resident at once, cooperative launch), few layers, one K block, and a
-    // C the TMA can store; the flags (one word per tile, CTA, epilogue warp and layer) must fit
-    // the call's ticket allocation
-    const int c_esz = (c_dtype == SFC_F32) ? 4 : 2;
-    const int64_t flag_words = static_cast<int64_t>(p.grid_tiles) * variant_cluster(v) * (bn / 32) * ca_c;
-    const bool want_fused = ca_c >= 2 && ca_c <= kFusedMaxLayers && kbf == 1 && p.num_items <= workers &&
-                            aligned16(C) && (ldc * c_esz) % 16 == 0 &&
-                            flag_words * 4 <= static_cast<int64_t>(kTicketBytes - kFlagOffset) &&
-                            g_fused_enabled.load(std::memory_order_relaxed) != 0;
 
     void* ws = workspace;
     bool pooled = false;
@@ -777,11 +729,10 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
         }
         pooled = true;
     }
-    // dynamic dealing, or K layers summed in the launch: the call's own ticket allocation (the
-    // K-block passes share it: each kernel leaves its counter zero, and a pass touches it only
-    // after the previous pass has finished)
+    // dynamic dealing: the call's own ticket counter (the K-block passes share it: each kernel
+    // leaves it zero, and a pass touches it only after the previous pass has finished)
     bool own_ticket = false;
-    if (p.dynamic || want_fused) {
+    if (p.dynamic) {
         if (fixed_ticket) {
             p.ticket = fixed_ticket;
         } else {
@@ -825,63 +776,29 @@ int run_gemm(int64_t M, int64_t N, int64_t K, const void* A, const void* B, void
                                      : launch_gemm<__nv_bfloat16>(v, f8, ta, tb, tc, p, grid, stream);
         }
     } else {
-        bool fused_done = false;
-        if (want_fused) {
-            // each region's owner layer adds the other layers' fp32 partials (stored in their
-            // workspace copies) and writes C; beta C + bias applied there, as the reduction kernel would
-            p.out = ws;
-            p.ldo = ws_ld(N);
-            p.layer_stride = M * p.ldo;
-            p.vec_store = 1;
-            p.tma_store = 1;
-            p.fused = 1;
-            p.flags = reinterpret_cast<unsigned int*>(reinterpret_cast<unsigned char*>(p.ticket) + kFlagOffset);
-            if (make_out_map(&tc, C, M, N, ldc, c_esz, 1) == SFC_OK) {
-                // cooperative launch, with programmatic dependent launch when the runtime takes both
-                for (int attempt = 0; attempt < 2 && !fused_done; ++attempt) {
-                    const bool pdl = attempt == 0;
-                    e = (c_dtype == SFC_F32) ? launch_gemm<float>(v, f8, ta, tb, tc, p, grid, stream, pdl)
-                                             : launch_gemm<__nv_bfloat16>(v, f8, ta, tb, tc, p, grid, stream, pdl);
-                    if (e == cudaSuccess) {
-                        fused_done = true;
-                        g_fused_launches.fetch_add(1, std::memory_order_relaxed);
-                    }
-                    else (void)cudaGetLastError();  // a configuration the runtime refused: try the next
-                }
+        // fp32 copies of C, one per K layer (K blocks added in place), then the reduction
+        p.out = ws;
+        p.ldo = ws_ld(N);
+        p.layer_stride = M * p.ldo;
+        p.vec_store = 1;
+        p.tma_store = make_out_map(&tc, ws, M, N, p.ldo, 4, ca_c) == SFC_OK;
+        p.beta = 0.0f;
+        p.bias = nullptr;
+        for (int pass = 0; pass < kbf && e == cudaSuccess; ++pass) {
+            if (pass > 0) {
+                p.accumulate = p.tma_store;
+                p.beta = p.tma_store ? 0.0f : 1.0f;
+                p.c_in = ws;
+                p.ldc_in = p.ldo;
+                p.c_in_layer_stride = p.layer_stride;
             }
-            if (!fused_done) {
-                // not launchable this way: the reduction kernel's path below
-                e = cudaSuccess;
-                p.fused = 0;
-                p.flags = nullptr;
-                std::memset(&tc, 0, sizeof(tc));
-            }
+            p.kbf = kbf;
+            p.pass = pass;
+            e = launch_gemm<float>(v, f8, ta, tb, tc, p, grid, stream);
         }
-        if (!fused_done) {
-            // fp32 copies of C, one per K layer (K blocks added in place), then the reduction
-            p.out = ws;
-            p.ldo = ws_ld(N);
-            p.layer_stride = M * p.ldo;
-            p.vec_store = 1;
-            p.tma_store = make_out_map(&tc, ws, M, N, p.ldo, 4, ca_c) == SFC_OK;
-            p.beta = 0.0f;
-            p.bias = nullptr;
-            for (int pass = 0; pass < kbf && e == cudaSuccess; ++pass) {
-                if (pass > 0) {
-                    p.accumulate = p.tma_store;
-                    p.beta = p.tma_store ? 0.0f : 1.0f;
-                    p.c_in = ws;
-                    p.ldc_in = p.ldo;
-                    p.c_in_layer_stride = p.layer_stride;
-                }
-                p.kbf = kbf;
-                p.pass = pass;
-                e = launch_gemm<float>(v, f8, ta, tb, tc, p, grid, stream);
-            }
-            if (e == cudaSuccess)
-                e = launch_reduce(dev, static_cast<const float*>(ws), p.ldo, p.layer_stride, ca_c, M, N, C, ldc, c_dtype,
-                                  beta, bias, stream);
-        }
+        if (e == cudaSuccess)
+            e = launch_reduce(dev, static_cast<const float*>(ws), p.ldo, p.layer_stride, ca_c, M, N, C, ldc, c_dtype,
+                              beta, bias, stream);
     }
     if (pooled) {
         cudaError_t f = cudaFreeAsync(ws, stream);
@@ -1197,13 +1114,6 @@ SFC_API int sfc_get_device_status(void* stream) {
 }
 
 SFC_API int sfc_last_cuda_error(void) { return t_last_cuda_error; }
-
-SFC_API int sfc_debug_set_fused(int enable) {
-    if (enable != 0 && enable != 1) return SFC_ERR_INVALID_ARG;
-    return g_fused_enabled.exchange(enable);
-}
-
-SFC_API long long sfc_debug_fused_launches(void) { return g_fused_launches.load(std::memory_order_relaxed); }
 
 SFC_API int sfc_num_workers(void) {
     DeviceInfo* dev = nullptr;

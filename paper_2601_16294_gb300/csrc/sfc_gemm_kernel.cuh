@@ -76,7 +76,6 @@ enum WaitSite : unsigned int {
     kWaitDrain = 1u << 13,
     kWaitQueueFull = 1u << 14,
     kWaitQueueEmpty = 1u << 15,
-    kWaitPartial = 1u << 16,
 };
 
 // Item dealing.  One scheduler thread per worker decodes the worker's items
@@ -94,6 +93,16 @@ enum WaitSite : unsigned int {
 // scheduler to finish sets both words to zero (also after a wait gave up), so
 // that a replay of a captured launch, which keeps its epoch, starts from zero.
 constexpr int kQueue = 4;
+
+// At a launch's start (after the wait for the previous grid): tag the word with
+// this epoch and a count of zero unless it carries the epoch already, so that
+// the first tickets find their tag and take one atomic add.  One attempt: a
+// failed swap means another worker changed the word first.
+__device__ __forceinline__ void epoch_claim(unsigned long long* word, unsigned int epoch) {
+    const unsigned long long tag = static_cast<unsigned long long>(epoch) << 32;
+    const unsigned long long cur = atomicOr(word, 0ull);
+    if ((cur & 0xffffffff00000000ull) != tag) atomicCAS(word, cur, tag);
+}
 
 // Next value of an epoch-tagged counter (see above); 32-bit counts.  The
 // common case is one atomic add.  An add that finds another tag is void: the
@@ -144,9 +153,6 @@ struct GemmParams {
     int ab_fmt;            // A/B format code of the instruction descriptor (bf16: 1; e4m3: 0, e5m2: 1)
     int kbf, pass;         // k_block_factor > 1: this launch contracts K block `pass` of every layer
     int accumulate;        // 1: the TMA stores add into `out` (fp32, in L2) instead of overwriting it
-    int fused;             // 1: the K layers are summed inside this launch (one item per worker)
-    unsigned int* flags;   // fused: per (tile, CTA, epilogue warp, layer < ca_c - 1), the epoch once
-                           // that layer's partial of the warp's 32 x 128 region is stored
 };
 
 struct WorkItem {
@@ -338,13 +344,18 @@ struct ItemSource {
 
 // Item j of a consuming role: fills w (tile, K layer and range; K order from
 // j) and returns the item index >= 0, or -1 when there are no more, -2 when a
-// bounded wait gave up.  Item 0 needs no wait: every CTA decodes it into its
-// own slot 0 during set-up (sched_local_first), before the block barrier.
+// bounded wait gave up.  Item 0 needs no wait (`first_local`, for the roles on
+// the start-up path: producer and MMA issuer): every CTA decodes it into its
+// own slot 0 during set-up (sched_local_first), before the block barrier.  The
+// epilogue waits for the slot's first phase as for any other item (it needs
+// item 0 only microseconds later, and the branch would cost it registers).
+template <bool kFirstLocal = false>
 __device__ __forceinline__ int64_t src_take(const ItemSource& S, int j, const GemmParams& p, volatile int* abort_flag,
                                             WorkItem& w) {
     const int q = j % kQueue;
-    if (j > 0 && !wait_bounded(S.q_full0 + 8u * q, static_cast<uint32_t>((j / kQueue) & 1), abort_flag, p.timeout_ns,
-                               kWaitQueueFull))
+    if ((!kFirstLocal || j > 0) &&
+        !wait_bounded(S.q_full0 + 8u * q, static_cast<uint32_t>((j / kQueue) & 1), abort_flag, p.timeout_ns,
+                      kWaitQueueFull))
         return -2;
     const int item = S.q_entry[4 * q];
     w.tm = S.q_entry[4 * q + 1];
@@ -355,22 +366,6 @@ __device__ __forceinline__ int64_t src_take(const ItemSource& S, int j, const Ge
     w.k1 = (p.ca_c == 1) ? p.Kt : layer_k0(w.layer + 1, p);
     narrow_to_pass(w, p);
     return item;
-}
-
-// Whether the worker has an item after item j: waits (bounded) for queue
-// entry j + 1 and reads its item index without consuming it (the later
-// src_take of j + 1 reads it again).  Returns 1 (more items), 0 (item j is the
-// worker's last) or -1 when a bounded wait gave up.  The scheduler publishes
-// entry j + 1 as soon as the producer has taken item j, long before any
-// epilogue is done with item j, so the wait is short.
-__device__ __forceinline__ int src_has_next(const ItemSource& S, int j, const GemmParams& p,
-                                            volatile int* abort_flag) {
-    const int jn = j + 1;
-    const int q = jn % kQueue;
-    if (!wait_bounded(S.q_full0 + 8u * q, static_cast<uint32_t>((jn / kQueue) & 1), abort_flag, p.timeout_ns,
-                      kWaitQueueFull))
-        return -1;
-    return S.q_entry[4 * q] >= 0 ? 1 : 0;
 }
 
 // Scheduler: the queue entry of an item (decoded tile and K layer).
@@ -442,6 +437,10 @@ __device__ __forceinline__ int sched_next(const ItemSource& S, int j, const Gemm
 __device__ __forceinline__ bool run_scheduler(const ItemSource& S, int item0, const GemmParams& p, const Barriers& B,
                                               volatile int* abort_flag, int n_ctas) {
     bool ok = true;
+    if (S.dynamic) {
+        epoch_claim(&p.ticket[0], p.epoch);
+        epoch_claim(&p.ticket[1], p.epoch);
+    }
     for (int j = 1; ok && item0 >= 0; ++j) {
         if (!wait_bounded_idle(B.q_taken(), static_cast<uint32_t>((j - 1) & 1), abort_flag, p.timeout_ns,
                                kWaitQueueEmpty, 256) ||
@@ -480,7 +479,7 @@ __device__ __forceinline__ bool produce(const ItemSource& src, const GemmParams&
     uint32_t phase = 0;
     for (int j = 0;; ++j) {
         WorkItem w;
-        const int64_t it = src_take(src, j, p, abort_flag, w);
+        const int64_t it = src_take<true>(src, j, p, abort_flag, w);
         if (it < 0) return it == -1;
         if (signal_taken) ptx::mbar_arrive(B.q_taken());
         const int nq = w.k1 - w.k0;
@@ -530,186 +529,6 @@ __device__ __forceinline__ void stage_row(uint8_t* box, int lane, const float* v
 }
 
 // -------------------------------------------------------------------------
-// K layers summed inside the launch (GemmParams::fused).  The host sets it
-// only when every worker holds exactly one item and all workers are resident
-// at once (a cooperative launch), so no item waits for one that has not
-// started.  A tile's c layers run on c workers at the same time, and the
-// tile's 32 x 128 warp regions are shared out among them: region q (q =
-// CTA * epilogue warps + warp) belongs to layer q mod c.  The warp that holds
-// a region of another layer stores its fp32 partial of it in that layer's
-// workspace copy and publishes the call's epoch in the region's flag for its
-// layer; the warp that owns a region waits for the c-1 flags, loads those
-// partials with the TMA into its share of the (then idle) operand ring, sums
-// all c partials in layer order 0, 1, ..., c-1 -- its own from registers, in
-// its place -- which is the order of ca_reduce_kernel, so the result has the
-// same bits, and writes C.  Every worker thus stores and sums a 1/c share of
-// its tile.  Flags hold epochs, not counts, so memory of earlier calls needs
-// no clearing; the owner clears each flag it consumed, so that a replay of a
-// captured launch, which keeps its epoch, waits again.
-// -------------------------------------------------------------------------
-
-// Bounded wait until *flag holds `epoch` (acquire at GPU scope).
-__device__ __forceinline__ bool wait_flag(const unsigned int* flag, unsigned int epoch, volatile int* abort_flag,
-                                          uint64_t limit_ns) {
-    if (ptx::ld_acquire_gpu(flag) == epoch) return true;
-    const uint64_t t0 = ptx::global_timer_ns();
-    for (;;) {
-        if (ptx::ld_acquire_gpu(flag) == epoch) return true;
-        if (*abort_flag) return false;
-        if (ptx::global_timer_ns() - t0 > limit_ns) {
-            *abort_flag = 1;
-            atomicOr(&g_sfc_status, 1u | kWaitPartial);
-            return false;
-        }
-    }
-}
-
-// Boxes of 16 fp32 columns (of the warp's kEpiCols) that hold columns < N.
-__device__ __forceinline__ int f32_boxes(int64_t col_base, int64_t N) {
-    const int64_t cols = N - col_base;
-    if (cols <= 0) return 0;
-    return cols >= kEpiCols ? kEpiCols / 16 : static_cast<int>((cols + 15) / 16);
-}
-
-// A warp holding another layer's region: store its fp32 partial of the region
-// in the layer's workspace copy, then publish the epoch in the region's flag
-// for this layer.  The partial goes out through ordinary (generic-proxy)
-// stores, ordered before the flag's release by a warp barrier:
-// a tensor-memory-accelerator store, even after its bulk-group wait and a
-// proxy fence, was measured to become visible to another SM's tensor loads
-// only after the flag (they then read the memory's old contents).  The rows
-// are staged in `buf` (the warp's share of the idle ring, swizzled boxes of
-// 16 columns) and written back 16 bytes per thread, eight full 64-byte row
-// pieces per warp store.
-__device__ __forceinline__ void fused_put_partial(const GemmParams& p, uint8_t* buf, int lane, int64_t warp_row,
-                                                  int64_t col_base, int layer, const float* run,
-                                                  unsigned int* flag) {
-    const int nbox = f32_boxes(col_base, p.N);
-#pragma unroll
-    for (int g = 0; g < kEpiCols / 16; ++g) {
-        if (g >= nbox) break;  // warp-uniform
-        stage_row<float>(buf + g * kBoxBytes, lane, run + g * 16);
-    }
-    __syncwarp();
-    float* ws = static_cast<float*>(p.out) + static_cast<int64_t>(layer) * p.layer_stride;
-    const int j = lane & 3;  // this thread's 16-byte piece of a 64-byte box row
-    for (int g = 0; g < nbox; ++g) {
-        const int64_t col = col_base + g * 16 + j * 4;  // < round_up(N, 4) = the copy's row stride when < N
-#pragma unroll
-        for (int t = 0; t < 4; ++t) {
-            const int r = t * 8 + (lane >> 2);
-            const int64_t row = warp_row + r;
-            const float4 v = *reinterpret_cast<const float4*>(buf + g * kBoxBytes + r * 64 + ((j ^ ((r >> 1) & 3)) << 4));
-            if (row < p.M && col < p.N) *reinterpret_cast<float4*>(ws + row * p.ldo + col) = v;
-        }
-    }
-    __syncwarp();  // every lane's stores happen before lane 0's release (which is cumulative)
-    if (lane == 0) ptx::st_release_gpu(flag + layer, p.epoch);
-}
-
-// Columns 8h..8h+7 of this lane's row of a 32-row fp32 box (16 columns, the
-// 64-byte swizzled layout of stage_row).
-__device__ __forceinline__ void box_half_row_f32(const uint8_t* box, int lane, int h, float* v) {
-    const uint8_t* row = box + lane * 64;
-    const int sw = (lane >> 1) & 3;
-#pragma unroll
-    for (int j = 0; j < 2; ++j) {
-        const float4 u = *reinterpret_cast<const float4*>(row + (((2 * h + j) ^ sw) * 16));
-        v[4 * j] = u.x;
-        v[4 * j + 1] = u.y;
-        v[4 * j + 2] = u.z;
-        v[4 * j + 3] = u.w;
-    }
-}
-
-// The warp owning its region (layer `own`): wait for the other layers'
-// partials of the region, copy them box by box into `buf` (its share of the
-// idle ring; rounds of as many 16-column boxes as fit, a power of two) and sum
-// all layers' values in layer order into run[], its own from registers in its
-// place.  The copies are ordinary L1-bypassing loads (cp.async), coalesced, one
-// 512-byte row piece per warp instruction, issued after lane 0's acquire of
-// the flags and a warp barrier: writer and reader stay in the generic proxy,
-// where the release/acquire pairing orders them.  False when a wait gave up.
-__device__ __forceinline__ bool fused_take_partials(const GemmParams& p, uint8_t* buf, int ring_share, int lane,
-                                                    int64_t warp_row, int64_t col_base, int own, float* run,
-                                                    unsigned int* flag, volatile int* abort_flag) {
-    const int L = p.ca_c - 1;  // layers copied: every layer but `own`, in order
-    const int nbox = f32_boxes(col_base, p.N);
-    if (nbox == 0) return true;
-    int ok = 1;
-    if (lane == 0) {
-        for (int l = 0; l < p.ca_c && ok; ++l)
-            if (l != own) ok = wait_flag(flag + l, p.epoch, abort_flag, p.timeout_ns);
-        if (ok) {
-            // each flag has one writer and this one reader per launch: clear it, so that a replay
-            // of a captured launch (same epoch) waits for its own partials
-            for (int l = 0; l < p.ca_c; ++l)
-                if (l != own) flag[l] = 0u;
-        }
-    }
-    ok = __shfl_sync(0xffffffffu, ok, 0);
-    __syncwarp();  // the lanes' loads below come after lane 0's acquire
-    if (!ok) return false;
-    int per_round = kEpiCols / 16;  // boxes per round: a power of two whose copies fit in buf
-    while (per_round > 1 && per_round * L * kBoxBytes > ring_share) per_round >>= 1;
-    const int pieces = per_round * 4;     // 16-byte pieces of a row in one round (4 .. 32)
-    const int rows_per_op = 32 / pieces;  // rows one warp instruction covers
-    const int piece = lane % pieces;
-#pragma unroll
-    for (int g = 0; g < kEpiCols / 16; ++g) {  // unrolled: run[] stays in registers
-        if (g >= nbox) break;                   // warp-uniform
-        const int slot = g % per_round;
-        if (slot == 0) {
-            // copy boxes g .. g + per_round - 1 of every other layer (rows past M and pieces past
-            // N are skipped: those outputs are not stored)
-            const int bx_in_round = piece >> 2, j = piece & 3;
-            const int64_t col = col_base + (g + bx_in_round) * 16 + j * 4;
-            for (int l = 0, li = 0; l < p.ca_c; ++l) {
-                if (l == own) continue;
-                const float* src = static_cast<const float*>(p.out) + l * p.layer_stride + col;
-                uint8_t* dst = buf + (bx_in_round * L + li) * kBoxBytes;
-                for (int r0 = 0; r0 < 32; r0 += rows_per_op) {
-                    const int r = r0 + lane / pieces;
-                    const int64_t row = warp_row + r;
-                    if (row < p.M && col < p.N)
-                        ptx::cp_async_16(ptx::smem_addr(dst + r * 64 + ((j ^ ((r >> 1) & 3)) << 4)), src + row * p.ldo);
-                }
-                ++li;
-            }
-            ptx::cp_async_wait_all();
-            __syncwarp();
-        }
-        // layers before `own` (copied slots 0..own-1), then its own partial, then the layers after
-        // it (copied slots own..L-1): P_0 + P_1 + ... + P_(c-1), left to right
-        const uint8_t* bx = buf + (slot * L) * kBoxBytes;
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {        // 8 columns at a time (fewer registers beside run[])
-            float* r = run + g * 16 + h * 8;  // g and h are constants here: r[] stays in registers
-            if (own > 0) {
-                float v[8];
-                box_half_row_f32(bx, lane, h, v);
-                for (int li = 1; li < own; ++li) {
-                    float u[8];
-                    box_half_row_f32(bx + li * kBoxBytes, lane, h, u);
-#pragma unroll
-                    for (int k = 0; k < 8; ++k) v[k] = __fadd_rn(v[k], u[k]);
-                }
-#pragma unroll
-                for (int k = 0; k < 8; ++k) r[k] = __fadd_rn(v[k], r[k]);
-            }
-            for (int li = own; li < L; ++li) {
-                float u[8];
-                box_half_row_f32(bx + li * kBoxBytes, lane, h, u);
-#pragma unroll
-                for (int k = 0; k < 8; ++k) r[k] = __fadd_rn(r[k], u[k]);
-            }
-        }
-        if (slot == per_round - 1 || g == nbox - 1) __syncwarp();  // buf is read before it is reused
-    }
-    return true;
-}
-
-// -------------------------------------------------------------------------
 // Epilogue of one block: drain chunks, promote, store.  `rows_base` is the
 // first output row this block's TMEM lanes map to for tile row tm.
 // -------------------------------------------------------------------------
@@ -717,8 +536,7 @@ template <int BN, typename OutT, bool PAIR>
 __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers& B, uint32_t tmem_base,
                                              volatile int* abort_flag, const ItemSource& src,
                                              int tile_rows, int row_offset, int warp, int lane,
-                                             const CUtensorMap* tmap_c, uint8_t* staging, uint8_t* ring_smem,
-                                             int ring_share, uint32_t pair_leader = 0) {
+                                             const CUtensorMap* tmap_c, uint8_t* staging, uint32_t pair_leader = 0) {
     const int ew = warp - 2;                 // epilogue warp index
     const int quarter = warp & 3;            // TMEM lane quarter this warp may access
     const int half = ew / 4;                 // which 128-column half of the tile
@@ -728,10 +546,8 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
     const uint32_t acce_target = PAIR ? ptx::map_to_cta(B.acc_empty(0), pair_leader) : B.acc_empty(0);
     float run[kEpiCols];
     // beta C_in + bias in this epilogue only without K layers (else the reduction applies
-    // it), when a later K block adds into the layer copies (k_block_factor > 1), or in the
-    // receiver of K layers summed in the launch (contributors return before it is applied)
-    const bool affine =
-        (p.ca_c == 1 || p.c_in_layer_stride != 0 || p.fused) && (p.beta != 0.0f || p.bias != nullptr);
+    // it), or when a later K block adds into the layer copies (k_block_factor > 1)
+    const bool affine = (p.ca_c == 1 || p.c_in_layer_stride != 0) && (p.beta != 0.0f || p.bias != nullptr);
     for (int j = 0;; ++j) {
         // lane 0 takes the item, the warp follows (tcgen05.ld needs the whole warp)
         int64_t it = 0;
@@ -794,60 +610,7 @@ __device__ __forceinline__ void run_epilogue(const GemmParams& p, const Barriers
         if (!ok) break;
         const int64_t warp_row = static_cast<int64_t>(w.tm) * tile_rows + row_offset + quarter * 32;
         const int64_t col_base = static_cast<int64_t>(w.tn) * BN + half * kEpiCols;
-        // The worker's last item: no loads follow it and the accumulator-full signal of its last
-        // chunk means every MMA has finished reading the operand ring, so the ring is idle and
-        // the warp stages all of its boxes at once in its share of it (one fence, one warp sync,
-        // one bulk group) instead of reusing its two-box buffer round after round.
-        constexpr int kAllBoxes = kEpiCols / box_cols<OutT>();
-        int last = 0;
-        if (p.fused) {
-            // one item per worker: every item is the worker's last
-            const int s_idx = static_cast<int>(it - static_cast<int64_t>(w.layer) * p.grid_tiles);
-            const int q = (PAIR ? (row_offset >> 7) : 0) * (BN / 32) + ew;  // region within the tile
-            const int region = s_idx * (PAIR ? 2 : 1) * (BN / 32) + q;
-            const int owner = q % p.ca_c;
-            unsigned int* flag = p.flags + static_cast<int64_t>(region) * p.ca_c;  // one word per layer
-            uint8_t* buf = ring_smem + ew * ring_share;
-            if (w.layer != owner) {
-                fused_put_partial(p, buf, lane, warp_row, col_base, w.layer, run, flag);
-                continue;
-            }
-            if (!fused_take_partials(p, buf, ring_share, lane, warp_row, col_base, w.layer, run, flag, abort_flag))
-                break;
-            last = 1;  // C (2-D map) is stored from the ring below
-        } else if (p.tma_store && ring_share >= kAllBoxes * kBoxBytes && lane == 0) {
-            last = src_has_next(src, j, p, abort_flag) == 0 ? 1 : 0;
-        }
-        last = __shfl_sync(0xffffffffu, last, 0);
-        if (last) {
-            constexpr int kCols = box_cols<OutT>();
-            uint8_t* buf = ring_smem + ew * ring_share;
-            int nbox = 0;
-#pragma unroll
-            for (int g = 0; g < kAllBoxes; ++g) {
-                if (col_base + g * kCols >= p.N) break;  // warp-uniform
-                if (affine) apply_affine<OutT, kCols>(p, warp_row + lane, col_base + g * kCols, w.layer, run + g * kCols);
-                stage_row<OutT>(buf + g * kBoxBytes, lane, run + g * kCols);
-                nbox = g + 1;
-            }
-            ptx::fence_proxy_async_smem();
-            __syncwarp();
-            if (lane == 0) {
-                for (int g = 0; g < nbox; ++g) {
-                    const uint32_t box_addr = ptx::smem_addr(buf + g * kBoxBytes);
-                    const int32_t x = static_cast<int32_t>(col_base + g * kCols);
-                    const int32_t y = static_cast<int32_t>(warp_row);
-                    if (p.ca_c > 1 && !p.fused) {
-                        if (p.accumulate) ptx::tma_reduce_add_3d(tmap_c, box_addr, x, y, w.layer);
-                        else ptx::tma_store_3d(tmap_c, box_addr, x, y, w.layer);
-                    } else {
-                        if (p.accumulate) ptx::tma_reduce_add_2d(tmap_c, box_addr, x, y);
-                        else ptx::tma_store_2d(tmap_c, box_addr, x, y);
-                    }
-                }
-                ptx::bulk_commit();
-            }
-        } else if (p.tma_store) {
+        if (p.tma_store) {
             // stage 32-row boxes and let the TMA write them (edges clipped by the map);
             // the two boxes of the buffer alternate
             constexpr int kCols = box_cols<OutT>();
@@ -1047,7 +810,7 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
             if (p.debug_never) ok = wait_bounded(B.never(), 0, abort_flag, p.timeout_ns, kWaitDebugNever);
             for (int j = 0; ok; ++j) {
                 WorkItem w;
-                const int64_t it = src_take(src, j, p, abort_flag, w);
+                const int64_t it = src_take<true>(src, j, p, abort_flag, w);
                 if (it < 0) {
                     ok = (it == -1);
                     break;
@@ -1105,7 +868,7 @@ sfc_gemm_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_constan
         }
     } else if (warp < scheduler_warp(BN)) {
         run_epilogue<BN, OutT, false>(p, B, tmem_base, abort_flag, src, kBM, 0, warp, lane, &tmap_c,
-                                      smem + L::kStagingOffset, smem, L::kRingBytes / kEpiWarps);
+                                      smem + L::kStagingOffset);
     } else if (sched_thread) {
         // -------------------------------------------------------- scheduler
         run_scheduler(src, item0, p, B, abort_flag, 1);

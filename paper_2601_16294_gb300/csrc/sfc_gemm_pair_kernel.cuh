@@ -23,9 +23,8 @@
 //
 // Waits are bounded as in the single-SM kernel.  The pair meets at a cluster
 // barrier after set-up (barriers initialised before any remote signal) and
-// before exit (no CTA leaves while its peer may still signal it; each warp
-// arrives as soon as its role is done); then both CTAs free their tensor
-// memory.
+// before exit (no CTA leaves while its peer may still signal it); then both
+// CTAs free their tensor memory.
 #pragma once
 
 #include "sfc_gemm_kernel.cuh"
@@ -190,7 +189,7 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
             if (p.debug_never) ok = wait_bounded(B.never(), 0, abort_flag, p.timeout_ns, kWaitDebugNever);
             for (int j = 0; ok; ++j) {
                 WorkItem w;
-                const int64_t it = src_take(src, j, p, abort_flag, w);
+                const int64_t it = src_take<true>(src, j, p, abort_flag, w);
                 if (it < 0) {
                     ok = (it == -1);
                     break;
@@ -248,20 +247,15 @@ sfc_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmap_a, const __grid_co
     } else if (warp < scheduler_warp(BN)) {
         run_epilogue<BN, OutT, true>(p, B, tmem_base, abort_flag, src, kItemRows,
                                      static_cast<int>(r * 128), warp, lane, &tmap_c,
-                                     smem + L::kStagingOffset, smem, L::kRingBytes / kEpiWarps, pair_leader);
+                                     smem + L::kStagingOffset, pair_leader);
     } else if (sched_thread) {
         // -------------------------------------------------------- scheduler
         run_scheduler(src, item0, p, B, abort_flag, kCtas);
     }
 
-    // No CTA leaves while another CTA of the cluster may still signal it: each warp arrives at
-    // the cluster barrier as soon as its role is done (its remote signals are released then),
-    // and the block waits for the whole cluster before freeing its tensor memory.
-    __syncwarp();
-    ptx::cluster_arrive();
     ptx::tc_fence_before();
     __syncthreads();
-    ptx::cluster_wait();
+    ptx::cluster_sync();  // no CTA leaves while another CTA of the cluster may still signal it
     ptx::tc_fence_after();
     if (warp == 1) ptx::tmem_dealloc_pair(tmem_base, kTmemCols);
 }
