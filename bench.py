@@ -54,6 +54,7 @@ TRAFFIC_FILES = {"configs": os.path.join(ROOT, "profiles", "traffic_configs.json
 TILE_KERNEL = {"pair256": "sfc_gemm_pair_kernel<256", "pair128": "sfc_gemm_pair_kernel<128",
                "256": "sfc_gemm_kernel<256", "128": "sfc_gemm_kernel<128"}
 CS = (1, 2, 4, 8)
+HOLD_HZ = 2.07e9  # GB300's maximum SM clock: cycles per second of the hold kernel's spin
 
 
 def _shape(M, N, K, kind="uniform", out="bf16", cs=(1,), shared=False):
@@ -150,6 +151,9 @@ def parse_args():
                          "smaller calls' copies then overlap the largest call's GEMMs)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-clocks", action="store_true")
+    ap.add_argument("--traffic-capture", action="store_true",
+                    help="the timed step runs every shape once with each tile at one K layer, for a profiler's "
+                         "per-tile DRAM record (prints the launch list instead of a bench line)")
     ap.add_argument("--no-cublas", action="store_true",
                     help="skip the comparison with torch.matmul (cuBLAS) in the same power window")
     return ap.parse_args()
@@ -389,6 +393,10 @@ def run_ours(args, rank, local, world):
         sfc.gemm(m["Ad"], m["Bd"], m["C"], ca_c=c, order=args.order, assign=args.assign, stream=stream,
                  b_layout=args.b_layout, k_block_factor=args.k_block_factor)
 
+    def hold(host_s):
+        # a spin kernel of about twice host_s at the maximum SM clock (longer at a lower clock)
+        torch.cuda._sleep(int(min(max(2.0 * host_s, 1e-4), 0.2) * HOLD_HZ))
+
     # the tensor cores' per-SM rate from resident operands (untimed), for the clock-based peak
     mma_per_clk = None
     if args.ab == "bf16":
@@ -411,41 +419,48 @@ def run_ours(args, rank, local, world):
                                 b_layout=args.b_layout, stream=stream)
         torch.cuda.synchronize()
 
-    # pick the K-layer count per shape where several are listed (timed, warm)
+    # pick the K-layer count per shape where several are listed (timed, warm), and time the
+    # library's own choice (ca_c = 0) beside them: three interleaved rounds of 5 calls per count,
+    # the minimum kept, so that a clock or power change during one round does not decide
+    def timed5(m, c):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(5):
+            call(m, c)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        return e0.elapsed_time(e1) / 5
+
     cs_report = {}
     for i, m in enumerate(mats):
         if len(m["s"]["cs"]) == 1:
             continue
         Kt = (m["s"]["K"] + 63) // 64
-        best = None
-        for c in [c for c in m["s"]["cs"] if c * args.k_block_factor <= Kt]:
+        cands = [c for c in m["s"]["cs"] if c * args.k_block_factor <= Kt] + [0]
+        for c in cands:
             for _ in range(2):
                 call(m, c)
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-            for _ in range(5):
-                call(m, c)
-            e1.record(stream)
-            torch.cuda.synchronize()
-            t = e0.elapsed_time(e1) / 5
-            cs_report.setdefault(i, {})[c] = round(t, 4)
-            if best is None or t < best[1]:
-                best = (c, t)
-        m["c"] = best[0]
-        # the library's own choice (ca_c = 0), reported beside the configured set
+        t_min = {c: float("inf") for c in cands}
+        for _ in range(3):
+            for c in cands:
+                t_min[c] = min(t_min[c], timed5(m, c))
+        configured = {c: t for c, t in t_min.items() if c != 0}
+        m["c"] = min(configured, key=configured.get)
+        cs_report[i] = {c: round(t, 4) for c, t in configured.items()}
         tile, c_auto = sfc.plan(m["s"]["M"], m["s"]["N"], m["s"]["K"], 0, out_dtype=m["C"].dtype,
                                 in_dtype=m["Ad"].dtype, b_layout=args.b_layout)
-        for _ in range(2):
-            call(m, 0)
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        for _ in range(5):
-            call(m, 0)
-        e1.record(stream)
-        torch.cuda.synchronize()
-        cs_report[i]["auto"] = {"ca_c": c_auto, "tile": str(tile), "ms": round(e0.elapsed_time(e1) / 5, 4)}
+        cs_report[i]["auto"] = {"ca_c": c_auto, "tile": str(tile), "ms": round(t_min[0], 4),
+                                "vs_best_configured": round(t_min[0] / configured[m["c"]], 3)}
+
+    capture_tiles = (128, 256, "pair128", "pair256")
 
     def step(events=None):
+        if args.traffic_capture:
+            for m in mats:
+                for t in capture_tiles:
+                    sfc.gemm(m["Ad"], m["Bd"], m["C"], ca_c=1, order=args.order, assign=args.assign, tile=t,
+                             stream=stream, b_layout=args.b_layout)
+            return
         for i, m in enumerate(mats):
             if events is not None:
                 events[i][0].record(stream)
@@ -455,6 +470,13 @@ def run_ours(args, rank, local, world):
 
     for _ in range(args.warmup):
         step()
+    torch.cuda.synchronize()
+    # the host's time to issue one step with an event pair around every launch (the device is
+    # idle meanwhile), for the hold kernel of the per-launch pass below
+    pairs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in mats]
+    h0 = time.perf_counter()
+    step(pairs)
+    issue_s = time.perf_counter() - h0
     torch.cuda.synchronize()
     if sfc.device_status() != 0:
         raise RuntimeError("device-side timeout during warm-up")
@@ -480,6 +502,10 @@ def run_ours(args, rank, local, world):
     status = sfc.device_status()
     if status != 0:
         raise RuntimeError("device-side timeout in the timed region (status %d)" % status)
+    if args.traffic_capture:
+        return {"traffic_capture": [{"M": m["s"]["M"], "N": m["s"]["N"], "K": m["s"]["K"], "ca_c": 1, "tile": str(t)}
+                                    for _ in range(args.steps) for m in mats for t in capture_tiles],
+                "kernel_sha": kernel_sha(), "workload": args.workload}
 
     elapsed_ms = max_over_ranks(t0.elapsed_time(t1), world)
     flops_step = sum(2.0 * m["s"]["M"] * m["s"]["N"] * m["s"]["K"] for m in mats)
@@ -492,10 +518,12 @@ def run_ours(args, rank, local, world):
     per_launch = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
                    for _ in mats] for _ in range(args.steps)]
     torch.cuda.synchronize()
-    # one untimed step first: the recorded launches then find the device busy with earlier work,
-    # so each event pair holds the launch's device time, not the host's issue of the first call
-    step()
+    # each step is issued behind a hold kernel that keeps the stream busy for twice the host's
+    # issue time, so every launch is queued before the device reaches it and each event pair
+    # holds the launch's device time (started after the previous launch finished), not gaps
+    # where the device waited for the host
     for k in range(args.steps):
+        hold(issue_s)
         step(per_launch[k])
     torch.cuda.synchronize()
 
@@ -587,7 +615,7 @@ def run_ours(args, rank, local, world):
                         continue
                     want = TILE_KERNEL.get(str(row["tile"]), "?")
                     hit = [e for e in tr["per_shape"] if (e["M"], e["N"], e["K"]) == (row["M"], row["N"], row["K"])
-                           and want in e["kernel"]]
+                           and e.get("ca_c") == 1 and want in e["kernel"]]
                     got.append(hit[0]["dram_bytes"] if hit else None)
                 if got and all(g is not None for g in got):
                     traffic = int(round(sum(got) / len(got)))
@@ -640,17 +668,27 @@ def run_ours(args, rank, local, world):
                    "l2": "inputs larger than L2 between reuses: one step runs every shape once, so a shape's "
                          "operands are re-read only after the other shapes' traffic has passed through L2",
                    "timing": "value: one event pair around the K steps; per_shape ms_mean: a second pass of the "
-                             "same steps with an event pair around each launch; ms_back_to_back: each shape alone, "
+                             "same steps with an event pair around each call, each step issued behind a hold "
+                             "kernel so that the pairs hold device time, not host issue; ms_back_to_back: each shape alone, "
                              "launches back to back over rotating input copies (> 256 MB between reuses)",
                    "pct_of_dense_peak": round(100.0 * value / world / burst, 2)},
         "roofline": roofline,
         "gpu_launches": launches,
         "per_shape": per_shape,
     }
+    if cs_report:
+        # the library's own layer count and tile (ca_c = 0) against the best configured count
+        r = [(mats[i]["s"], v["auto"]["vs_best_configured"]) for i, v in cs_report.items()]
+        worst = max(r, key=lambda x: x[1])
+        result["library_choice"] = {
+            "shapes": len(r), "within_5pct_of_best": sum(1 for _, q in r if q <= 1.05),
+            "faster_than_best": sum(1 for _, q in r if q < 1.0),
+            "worst": {"M": worst[0]["M"], "N": worst[0]["N"], "K": worst[0]["K"], "ratio": worst[1]},
+            "timing": "min over three interleaved rounds of 5 warm back-to-back calls per count"}
     if clock_info is not None:
         result["clocks"] = clock_info
     if not args.no_cublas and world == 1:
-        result["cublas_same_window"] = run_cublas_compare(args, mats, stream, call)
+        result["cublas_same_window"] = run_cublas_compare(args, mats, stream, call, hold)
     if not args.no_e2e:
         result["e2e"] = run_e2e(args, mats, stream, world)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -658,7 +696,7 @@ def run_ours(args, rank, local, world):
     return result
 
 
-def run_cublas_compare(args, mats, stream, call):
+def run_cublas_compare(args, mats, stream, call, hold):
     """Comparison only: torch.matmul (cuBLAS) on the same shapes, alternating
     step by step with this library so both see the same clocks and power."""
     import torch
@@ -689,38 +727,62 @@ def run_cublas_compare(args, mats, stream, call):
                 cublas(m)
     except Exception as e:  # e.g. a shape cuBLAS's 8-bit GEMM does not take
         return {"unavailable": "cuBLAS comparison failed: %s" % str(e).splitlines()[0][:200]}
-    # every step of both arms is issued before one synchronisation (the host runs ahead of the
-    # device, so each event pair holds device time only); one untimed step of each arm goes first
+    arms = (lambda m: call(m, m["c"]), cublas)
+    # one untimed step of each arm first, its host issue time measured (the device is busy)
     torch.cuda.synchronize()
-    for m in mats:
-        call(m, m["c"])
-    for m in mats:
-        cublas(m)
+    issue_s = []
+    for arm in arms:
+        h0 = time.perf_counter()
+        for m in mats:
+            arm(m)
+        issue_s.append(time.perf_counter() - h0)
+    torch.cuda.synchronize()
+    # (1) an event pair around every call; each arm's step is issued behind a hold kernel of
+    # twice its host issue time, so each pair holds the call's device time, started after the
+    # previous call finished
     evs = []
     for k in range(steps):
         for which in (0, 1):
+            hold(issue_s[which])
             ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in mats]
             for i, m in enumerate(mats):
                 ev[i][0].record(stream)
-                if which == 0:
-                    call(m, m["c"])
-                else:
-                    cublas(m)
+                arms[which](m)
                 ev[i][1].record(stream)
             evs.append((which, ev))
     torch.cuda.synchronize()
     for which, ev in evs:
         for i in range(len(mats)):
             t[i][which] += ev[i][0].elapsed_time(ev[i][1])
+    # (2) one event pair around each arm's whole step, calls back to back as a caller issues them
+    # (this library's launches then overlap their start with the previous launch's end)
+    step_ev = []
+    for k in range(steps):
+        for which in (0, 1):
+            hold(issue_s[which])
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for m in mats:
+                arms[which](m)
+            e1.record(stream)
+            step_ev.append((which, e0, e1))
+    torch.cuda.synchronize()
+    t_step = [0.0, 0.0]
+    for which, e0, e1 in step_ev:
+        t_step[which] += e0.elapsed_time(e1)
     fl = [2.0 * m["s"]["M"] * m["s"]["N"] * m["s"]["K"] * steps for m in mats]
     ours, cub = sum(x[0] for x in t), sum(x[1] for x in t)
     return {"cublas_tflops": round(sum(fl) / (cub * 1e-3) / 1e12, 1),
             "ours_tflops": round(sum(fl) / (ours * 1e-3) / 1e12, 1), "steps": steps,
+            "back_to_back": {"cublas_tflops": round(sum(fl) / (t_step[1] * 1e-3) / 1e12, 1),
+                             "ours_tflops": round(sum(fl) / (t_step[0] * 1e-3) / 1e12, 1),
+                             "timing": "one event pair around each arm's step of back-to-back calls"},
             "per_shape": [{"M": m["s"]["M"], "N": m["s"]["N"], "K": m["s"]["K"],
                            "ours": round(f / (x[0] * 1e-3) / 1e12, 1), "cublas": round(f / (x[1] * 1e-3) / 1e12, 1)}
                           for m, f, x in zip(mats, fl, t)],
-            "note": "alternating steps, same stream, issued ahead of the device (one synchronisation at the end); "
-                    "cuBLAS output is bf16 (fp32 rows: bf16 GEMM then cast)"}
+            "note": "alternating steps, same stream, each step issued behind a hold kernel (one synchronisation "
+                    "at the end); cublas_tflops / ours_tflops: an event pair around every call; cuBLAS output is "
+                    "bf16 (fp32 rows: bf16 GEMM then cast)"}
 
 
 def run_e2e(args, mats, stream, world):
