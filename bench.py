@@ -421,7 +421,8 @@ def run_ours(args, rank, local, world):
 
     # pick the K-layer count per shape where several are listed (timed, warm), and time the
     # library's own choice (ca_c = 0) beside them: three interleaved rounds of 5 calls per count,
-    # the minimum kept, so that a clock or power change during one round does not decide
+    # the minimum kept, so that neither a clock or power change during one round nor the order
+    # decides
     def timed5(m, c):
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
@@ -437,12 +438,13 @@ def run_ours(args, rank, local, world):
             continue
         Kt = (m["s"]["K"] + 63) // 64
         cands = [c for c in m["s"]["cs"] if c * args.k_block_factor <= Kt] + [0]
-        for c in cands:
-            for _ in range(2):
-                call(m, c)
         t_min = {c: float("inf") for c in cands}
-        for _ in range(3):
-            for c in cands:
+        for r in range(3):
+            # each round in another order, each count after two untimed calls of its own (the
+            # previous count's partials may still be dirty in L2)
+            for c in cands[r % len(cands):] + cands[:r % len(cands)]:
+                for _ in range(2):
+                    call(m, c)
                 t_min[c] = min(t_min[c], timed5(m, c))
         configured = {c: t for c, t in t_min.items() if c != 0}
         m["c"] = min(configured, key=configured.get)
@@ -684,7 +686,8 @@ def run_ours(args, rank, local, world):
             "shapes": len(r), "within_5pct_of_best": sum(1 for _, q in r if q <= 1.05),
             "faster_than_best": sum(1 for _, q in r if q < 1.0),
             "worst": {"M": worst[0]["M"], "N": worst[0]["N"], "K": worst[0]["K"], "ratio": worst[1]},
-            "timing": "min over three interleaved rounds of 5 warm back-to-back calls per count"}
+            "timing": "min over three interleaved rounds (rotated order) of 5 back-to-back calls per count, "
+                      "each after two untimed calls"}
     if clock_info is not None:
         result["clocks"] = clock_info
     if not args.no_cublas and world == 1:
