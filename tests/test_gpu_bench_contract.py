@@ -48,3 +48,30 @@ def test_default_line_keys():
     assert len(d["per_shape"]) == 2 and all(p["tile"] for p in d["per_shape"])
     assert all(p["ms_min"] <= p["ms_median"] for p in d["per_shape"])
 
+
+
+def test_traffic_capture_runs_every_tile_of_every_shape():
+    d = run_bench("--shapes", "512x512x512,256x384x128", "--traffic-capture", "--no-tune", "--ca-c", "1",
+                  "--steps", "1", "--warmup", "3", "--no-cublas", "--no-e2e", "--no-cpu-baseline", "--no-clocks")
+    sys.path.insert(0, ROOT)
+    import bench
+    assert d["kernel_sha"] == bench.kernel_sha()
+    calls = d["traffic_capture"]
+    assert len(calls) == 2 * 4
+    assert {(c["M"], c["N"], c["K"]) for c in calls} == {(512, 512, 512), (256, 384, 128)}
+    assert {c["tile"] for c in calls} == {"128", "256", "pair128", "pair256"}
+    assert all(c["ca_c"] == 1 for c in calls)
+
+
+def test_layer_counts_library_choice_and_both_cublas_modes():
+    d = run_bench("--shapes", "512x512x8192", "--steps", "3", "--warmup", "3", "--no-e2e", "--no-cpu-baseline",
+                  "--no-clocks")
+    row = d["per_shape"][0]
+    assert {"1", "2", "4", "8", "auto"} <= set(row["ms_by_ca_c"])
+    assert row["ca_c"] in (1, 2, 4, 8)
+    assert row["ms_by_ca_c"][str(row["ca_c"])] == min(v for k, v in row["ms_by_ca_c"].items() if k != "auto")
+    lc = d["library_choice"]
+    assert lc["shapes"] == 1 and 0 < lc["worst"]["ratio"] < 10
+    c = d["cublas_same_window"]
+    assert c["ours_tflops"] > 0 and c["cublas_tflops"] > 0
+    assert c["back_to_back"]["ours_tflops"] > 0 and c["back_to_back"]["cublas_tflops"] > 0
