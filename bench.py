@@ -394,8 +394,10 @@ def run_ours(args, rank, local, world):
                  b_layout=args.b_layout, k_block_factor=args.k_block_factor)
 
     def hold(host_s):
-        # a spin kernel of about twice host_s at the maximum SM clock (longer at a lower clock)
-        torch.cuda._sleep(int(min(max(2.0 * host_s, 1e-4), 0.2) * HOLD_HZ))
+        # a spin kernel of about twice host_s at the maximum SM clock (longer at a lower clock);
+        # without torch's spin kernel the pairs may also hold gaps where the device waited
+        if hasattr(torch.cuda, "_sleep"):
+            torch.cuda._sleep(int(min(max(2.0 * host_s, 1e-4), 0.2) * HOLD_HZ))
 
     # the tensor cores' per-SM rate from resident operands (untimed), for the clock-based peak
     mma_per_clk = None
