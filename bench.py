@@ -46,10 +46,10 @@ FALLBACK_PEAKS = {"bf16_tflops": 1900.0, "hbm_gbs": 6800.0, "bf16_tflops_sustain
 KERNEL_SOURCES = ("paper_2601_16294_gb300/csrc/sfc_gemm_kernel.cuh", "paper_2601_16294_gb300/csrc/ptx.cuh",
                   "paper_2601_16294_gb300/csrc/sfc_curve.cuh", "paper_2601_16294_gb300/csrc/sfc_gemm.cu",
                   "paper_2601_16294_gb300/csrc/sfc_gemm_pair_kernel.cuh")
-TRAFFIC_FILE = os.path.join(ROOT, "profiles", "traffic_square_sweep.json")
-# per-shape DRAM bytes of the GEMM launches of a workload's timed step (one ncu capture), keyed
-# like the square record by the kernel sources' hash
-TRAFFIC_FILES = {"configs": os.path.join(ROOT, "profiles", "traffic_configs.json")}
+# per-shape DRAM bytes of each tile's GEMM launch on a workload's shapes (one ncu capture of
+# --traffic-capture), keyed by the kernel sources' hash
+TRAFFIC_FILES = {"configs": os.path.join(ROOT, "profiles", "traffic_configs.json"),
+                 "square": os.path.join(ROOT, "profiles", "traffic_square_sweep.json")}
 # the kernel name a tile label launches (the record says which kernel each capture measured)
 TILE_KERNEL = {"pair256": "sfc_gemm_pair_kernel<256", "pair128": "sfc_gemm_pair_kernel<128",
                "256": "sfc_gemm_kernel<256", "128": "sfc_gemm_kernel<128"}
@@ -606,7 +606,7 @@ def run_ours(args, rank, local, world):
         achieved = flops_step * args.steps / (tot_ms * 1e-3) / 1e12
     traffic = None
     try:
-        with open(TRAFFIC_FILES.get(args.workload, TRAFFIC_FILE)) as f:
+        with open(TRAFFIC_FILES[args.workload]) as f:
             tr = json.load(f)
         if (tr.get("kernel_sha") == kernel_sha() and tr.get("workload") == args.workload and not args.sizes
                 and not args.shapes):
