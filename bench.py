@@ -198,6 +198,25 @@ def kernel_sha() -> str:
     return h.hexdigest()[:16]
 
 
+def traffic_per_launch(record, rows, workload, sha):
+    """Mean DRAM bytes per launch over the one-layer calls in `rows` (bench per-shape rows with
+    M, N, K, ca_c and tile), each matched to the record's capture of the same shape and kernel;
+    None when the record belongs to other kernel sources or another workload, or lacks a call."""
+    if record.get("kernel_sha") != sha or record.get("workload") != workload:
+        return None
+    got = []
+    for row in rows:
+        if row["ca_c"] != 1:
+            continue
+        want = TILE_KERNEL.get(str(row["tile"]))
+        hit = [e for e in record.get("per_shape", []) if want and (e["M"], e["N"], e["K"]) == (row["M"], row["N"], row["K"])
+               and e.get("ca_c") == 1 and want in e["kernel"]]
+        if not hit:
+            return None
+        got.append(hit[0]["dram_bytes"])
+    return int(round(sum(got) / len(got))) if got else None
+
+
 def load_peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -605,28 +624,12 @@ def run_ours(args, rank, local, world):
     else:
         achieved = flops_step * args.steps / (tot_ms * 1e-3) / 1e12
     traffic = None
-    try:
-        with open(TRAFFIC_FILES[args.workload]) as f:
-            tr = json.load(f)
-        if (tr.get("kernel_sha") == kernel_sha() and tr.get("workload") == args.workload and not args.sizes
-                and not args.shapes):
-            if "per_shape" in tr:
-                # the one-layer calls of this run, each matched to the capture of the same shape
-                # and the same kernel; any call without such a capture leaves traffic unknown
-                got = []
-                for row in per_shape:
-                    if row["ca_c"] != 1:
-                        continue
-                    want = TILE_KERNEL.get(str(row["tile"]), "?")
-                    hit = [e for e in tr["per_shape"] if (e["M"], e["N"], e["K"]) == (row["M"], row["N"], row["K"])
-                           and e.get("ca_c") == 1 and want in e["kernel"]]
-                    got.append(hit[0]["dram_bytes"] if hit else None)
-                if got and all(g is not None for g in got):
-                    traffic = int(round(sum(got) / len(got)))
-            else:
-                traffic = tr["dram_bytes_per_launch"]
-    except Exception:
-        traffic = None
+    if not args.sizes and not args.shapes and args.workload in TRAFFIC_FILES:
+        try:
+            with open(TRAFFIC_FILES[args.workload]) as f:
+                traffic = traffic_per_launch(json.load(f), per_shape, args.workload, kernel_sha())
+        except (OSError, ValueError):
+            traffic = None
     # burst peak for a short timed region, sustained (power-capped) peak for a long one;
     # 8-bit inputs: the measured bf16 peak times the nominal 8-bit / bf16 ratio
     sustained = elapsed_ms > 500.0
